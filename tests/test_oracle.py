@@ -1,0 +1,359 @@
+"""Pins for the fp64 CPU oracle, against facts that do not come from the oracle.
+
+Each check ties the oracle to something independent of its own code: a
+worked example derived by hand, closed forms (zero heads, identical student
+and teacher), library routines on special cases (``torch.nn.functional``
+cross-entropy, soft-target cross-entropy, KL, logsumexp, numpy argmax),
+central finite differences, autograd of the loss written from Eq. 2/3, and
+invariants of the gradient (rows of dL/dz sum to zero, linearity).
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+import torch.nn.functional as F
+
+from oracle import oracle as orc
+
+
+def normal(shape, seed, scale=1.0, dtype=np.float64):
+    return (np.random.default_rng(seed).standard_normal(shape) * scale).astype(dtype)
+
+
+def problem(T, d, V, seed=0, hs=1.0, ws=0.3, dtype=np.float64):
+    H = [normal((T, dm), seed + 10 * m, hs, dtype) for m, dm in enumerate(d)]
+    W = [normal((V, dm), seed + 10 * m + 5, ws, dtype) for m, dm in enumerate(d)]
+    y = np.random.default_rng(seed + 99).integers(0, V, T).astype(np.int32)
+    return H, W, y
+
+
+def logits(H, W):
+    return [torch.from_numpy(h.astype(np.float64)) @ torch.from_numpy(w.astype(np.float64)).T
+            for h, w in zip(H, W)]
+
+
+def sig(x):
+    return 1.0 / (1.0 + math.exp(-x))
+
+
+# ---------------------------------------------------------------- worked example
+@pytest.mark.parametrize("tau", [1.0, 2.0])
+def test_hand_worked_example(tau):
+    """Two sub-models, V = 2, width 1, one token with target 0, derived by hand.
+
+    student logits z_s = (1, 0), teacher logits z_T = (2, -2), alpha = 1/2.
+    """
+    H = [np.array([[1.0]]), np.array([[2.0]])]
+    W = [np.array([[1.0], [0.0]]), np.array([[1.0], [-1.0]])]
+    y = np.array([0], np.int32)
+    alpha = 0.5
+    out = orc.forward(H, W, y, teacher=1, tau=tau, alpha=alpha)
+    dH, dW = orc.backward(H, W, y, teacher=1, tau=tau, alpha=alpha)
+
+    ce_s = math.log1p(math.exp(-1.0))                 # log(e + 1) - 1
+    ce_t = math.log1p(math.exp(-4.0))                 # log(e^2 + e^-2) - 2
+    q0, q1 = sig(4.0 / tau), sig(-4.0 / tau)          # softmax((2, -2) / tau)
+    lp0 = -math.log1p(math.exp(-1.0 / tau))           # log softmax((1, 0) / tau)
+    lp1 = -1.0 / tau - math.log1p(math.exp(-1.0 / tau))
+    ld_s = -(q0 * lp0 + q1 * lp1)
+    hq = -(q0 * math.log(q0) + q1 * math.log(q1))
+    assert out["ce"][0, 0] == pytest.approx(ce_s, abs=1e-14)
+    assert out["ce"][1, 0] == pytest.approx(ce_t, abs=1e-14)
+    assert out["ld"][0, 0] == pytest.approx(ld_s, abs=1e-14)
+    assert out["kl"][0, 0] == pytest.approx(ld_s - hq, abs=1e-14)
+    assert out["tok_loss"][0, 0] == pytest.approx(0.5 * ce_s + 0.5 * ld_s, abs=1e-14)
+    assert out["tok_loss"][1, 0] == pytest.approx(ce_t, abs=1e-14)
+    assert out["loss"] == pytest.approx(0.5 * ce_s + 0.5 * ld_s + ce_t, abs=1e-14)
+    assert list(out["argmax"][:, 0]) == [0, 0]
+
+    # gradients: student G = (1-a)(p - e_y) + (a/tau)(p^tau - q); teacher G = p - e_y
+    p0, p1 = sig(1.0), sig(-1.0)
+    pt0, pt1 = sig(1.0 / tau), sig(-1.0 / tau)
+    gs = [0.5 * (p0 - 1.0) + 0.5 / tau * (pt0 - q0), 0.5 * p1 + 0.5 / tau * (pt1 - q1)]
+    gt = [sig(4.0) - 1.0, sig(-4.0)]
+    assert dH[0][0, 0] == pytest.approx(gs[0] * 1.0 + gs[1] * 0.0, abs=1e-14)
+    assert dW[0][:, 0] == pytest.approx([gs[0] * 1.0, gs[1] * 1.0], abs=1e-14)
+    assert dH[1][0, 0] == pytest.approx(gt[0] * 1.0 + gt[1] * -1.0, abs=1e-14)
+    assert dW[1][:, 0] == pytest.approx([gt[0] * 2.0, gt[1] * 2.0], abs=1e-14)
+
+
+# ---------------------------------------------------------------- closed forms
+@pytest.mark.parametrize("tau", [0.5, 1.0, 2.0])
+def test_zero_heads_give_log_v(tau):
+    T, d, V = 7, (8, 16, 12), 37
+    H, W, y = problem(T, d, V, seed=1)
+    W = [np.zeros_like(w) for w in W]
+    w = (0.5, 2.0, 1.5)
+    out = orc.forward(H, W, y, tau=tau, alpha=0.3, w=w)
+    lv = math.log(V)
+    np.testing.assert_allclose(out["ce"], lv, atol=1e-12)
+    np.testing.assert_allclose(out["ld"], lv, atol=1e-12)
+    np.testing.assert_allclose(out["kl"], 0.0, atol=1e-12)
+    np.testing.assert_allclose(out["lse"], lv, atol=1e-12)
+    np.testing.assert_allclose(out["lse_tau"], lv, atol=1e-12)
+    assert out["loss"] == pytest.approx(sum(w) * lv, rel=1e-13)
+    assert (out["argmax"] == 0).all()
+
+
+@pytest.mark.parametrize("tau", [0.5, 1.0, 3.0])
+def test_student_equal_teacher(tau):
+    """Identical student and teacher: KL = 0, Ld = H(q) and the distillation
+    gradient vanishes, so the student's gradients are (1 - alpha) times the
+    teacher's."""
+    T, V, dm = 9, 29, 12
+    H, W, y = problem(T, (dm,), V, seed=2, ws=0.5)
+    H2, W2 = [H[0], H[0].copy()], [W[0], W[0].copy()]
+    alpha = 0.35
+    out = orc.forward(H2, W2, y, teacher=1, tau=tau, alpha=alpha)
+    np.testing.assert_allclose(out["kl"][0], 0.0, atol=1e-13)
+    z = logits(H, W)[0]
+    q = torch.softmax(z / tau, -1)
+    Hq = -(q * torch.log(q)).sum(-1).numpy()
+    np.testing.assert_allclose(out["ld"][0], Hq, rtol=1e-12)
+    dH, dW = orc.backward(H2, W2, y, teacher=1, tau=tau, alpha=alpha)
+    np.testing.assert_allclose(dH[0], (1 - alpha) * dH[1], rtol=1e-10, atol=1e-15)
+    np.testing.assert_allclose(dW[0], (1 - alpha) * dW[1], rtol=1e-10, atol=1e-15)
+
+
+# ---------------------------------------------------------------- library routines
+def test_alpha_zero_is_library_cross_entropy():
+    T, d, V = 16, (8, 24, 16), 50
+    H, W, y = problem(T, d, V, seed=3)
+    w = (1.0, 0.25, 3.0)
+    out = orc.forward(H, W, y, tau=1.7, alpha=0.0, w=w)
+    zs = logits(H, W)
+    yt = torch.from_numpy(y.astype(np.int64))
+    total = 0.0
+    for m, z in enumerate(zs):
+        ce = F.cross_entropy(z, yt, reduction="none").numpy()
+        np.testing.assert_allclose(out["ce"][m], ce, rtol=1e-12)
+        np.testing.assert_allclose(out["tok_loss"][m], ce, rtol=1e-12)
+        total += w[m] * ce.mean()
+    assert out["loss"] == pytest.approx(total, rel=1e-12)
+
+
+@pytest.mark.parametrize("tau", [0.5, 1.0, 2.0])
+def test_distillation_is_soft_target_cross_entropy(tau):
+    T, d, V = 11, (8, 16, 24), 64
+    H, W, y = problem(T, d, V, seed=4, ws=0.4)
+    out = orc.forward(H, W, y, teacher=2, tau=tau, alpha=0.5)
+    zs = logits(H, W)
+    q = torch.softmax(zs[2] / tau, -1)
+    for m in range(3):
+        ld = F.cross_entropy(zs[m] / tau, q, reduction="none").numpy()
+        kl = F.kl_div(torch.log_softmax(zs[m] / tau, -1), q, reduction="none").sum(-1).numpy()
+        np.testing.assert_allclose(out["ld"][m], ld, rtol=1e-11)
+        np.testing.assert_allclose(out["kl"][m], kl, rtol=1e-9, atol=1e-13)
+        np.testing.assert_allclose(out["lse"][m], torch.logsumexp(zs[m], -1).numpy(), rtol=1e-13)
+        np.testing.assert_allclose(out["lse_tau"][m], torch.logsumexp(zs[m] / tau, -1).numpy(),
+                                   rtol=1e-13)
+        np.testing.assert_array_equal(out["argmax"][m], np.argmax(zs[m].numpy(), -1))
+        ce = F.cross_entropy(zs[m], torch.from_numpy(y.astype(np.int64)), reduction="none").numpy()
+        want = ce if m == 2 else 0.5 * ce + 0.5 * ld
+        np.testing.assert_allclose(out["tok_loss"][m], want, rtol=1e-11)
+
+
+def test_integer_exact_argmax_and_ties():
+    """One-hot hidden rows and small-integer heads make every logit an exact
+    integer; argmax then must equal numpy's (first maximum on ties)."""
+    T, V, dm = 24, 40, 16
+    rng = np.random.default_rng(5)
+    H = np.zeros((T, dm), np.float32)
+    H[np.arange(T), rng.integers(0, dm, T)] = 1.0
+    W = rng.integers(-3, 4, (V, dm)).astype(np.float32)
+    W[7] = W[3]          # duplicate rows -> exact ties between v=3 and v=7
+    Hs, Ws = [H, H], [W, np.flip(W, 0).copy()]
+    y = rng.integers(0, V, T).astype(np.int32)
+    out = orc.forward(Hs, Ws, y)
+    for m in range(2):
+        z = Hs[m].astype(np.int64) @ Ws[m].astype(np.int64).T
+        np.testing.assert_array_equal(out["argmax"][m], np.argmax(z, -1))
+        ce = out["lse"][m] - z[np.arange(T), y]
+        np.testing.assert_allclose(out["ce"][m], ce, rtol=0, atol=1e-12)
+
+
+def test_bf16_storage_decodes_exactly():
+    T, d, V = 5, (8, 16), 33
+    H, W, y = problem(T, d, V, seed=6, dtype=np.float32)
+    Hb = [torch.from_numpy(h).to(torch.bfloat16) for h in H]
+    Wb = [torch.from_numpy(w).to(torch.bfloat16) for w in W]
+    bits = lambda ts: [t.view(torch.int16).numpy().view(np.uint16) for t in ts]
+    f32 = lambda ts: [t.float().numpy() for t in ts]
+    a = orc.forward(bits(Hb), bits(Wb), y, tau=0.7)
+    b = orc.forward(f32(Hb), f32(Wb), y, tau=0.7)
+    assert a["loss"] == b["loss"]
+    np.testing.assert_array_equal(a["tok_loss"], b["tok_loss"])
+
+
+# ---------------------------------------------------------------- gradients
+def _fd_case():
+    T, d, V = 4, (8, 16), 32
+    H, W, y = problem(T, d, V, seed=7, ws=0.5)
+    y[2] = -1            # one ignored token
+    return H, W, y, dict(teacher=1, tau=0.8, alpha=0.4, w=(1.3, 0.7))
+
+
+def test_finite_differences():
+    """Central differences in fp64 of the objective.  Student parameters see
+    the whole loss; the teacher's see only its own term, because Eq. 2 stops
+    the gradient through the teacher's distribution."""
+    H, W, y, kw = _fd_case()
+    dH, dW = orc.backward(H, W, y, grad_scale=1.0, **kw)
+    eps = 1e-6
+    T = H[0].shape[0]
+    n = int((y >= 0).sum())
+    tmask = y >= 0
+
+    def objective(Hc, Wc, m):
+        out = orc.forward(Hc, Wc, y, **kw)
+        if m == kw["teacher"]:
+            return kw["w"][m] * out["tok_loss"][m][tmask].sum() / n
+        return out["loss"]
+
+    for m in range(2):
+        for which, grad in (("H", dH[m]), ("W", dW[m])):
+            base = H if which == "H" else W
+            fd = np.zeros_like(grad)
+            for idx in np.ndindex(*grad.shape):
+                vals = []
+                for sgn in (1, -1):
+                    arrs = [a.copy() for a in base]
+                    arrs[m][idx] += sgn * eps
+                    vals.append(objective(arrs, W, m) if which == "H" else objective(H, arrs, m))
+                fd[idx] = (vals[0] - vals[1]) / (2 * eps)
+            scale = np.abs(grad).max()
+            assert np.abs(fd - grad).max() <= 1e-6 * scale, (m, which)
+
+
+def test_autograd_of_eq2_eq3():
+    """Gradients from torch autograd applied to the objective written from
+    Eq. 2/3 with q detached (stop_grad)."""
+    T, d, V = 12, (16, 24, 8), 40
+    H, W, y = problem(T, d, V, seed=8, ws=0.4)
+    y[[3, 9]] = -1
+    teacher, tau, alpha, w, g = 1, 0.7, 0.3, (0.5, 1.5, 2.0), 1.3
+    dH, dW = orc.backward(H, W, y, teacher=teacher, tau=tau, alpha=alpha, w=w, grad_scale=g)
+    Ht = [torch.tensor(h, requires_grad=True) for h in H]
+    Wt = [torch.tensor(x, requires_grad=True) for x in W]
+    yt = torch.from_numpy(y.astype(np.int64))
+    valid = yt >= 0
+    n = valid.sum()
+    z = [h @ x.T for h, x in zip(Ht, Wt)]
+    q = torch.softmax(z[teacher] / tau, -1).detach()
+    loss = 0.0
+    for m in range(3):
+        ce = torch.logsumexp(z[m], -1) - z[m].gather(1, yt.clamp(min=0)[:, None])[:, 0]
+        if m == teacher:
+            lm = ce
+        else:
+            ld = -(q * torch.log_softmax(z[m] / tau, -1)).sum(-1)
+            lm = (1 - alpha) * ce + alpha * ld
+        loss = loss + w[m] * (lm * valid).sum() / n
+    (g * loss).backward()
+    for m in range(3):
+        np.testing.assert_allclose(dH[m], Ht[m].grad.numpy(), rtol=1e-10, atol=1e-14)
+        np.testing.assert_allclose(dW[m], Wt[m].grad.numpy(), rtol=1e-10, atol=1e-14)
+
+
+def test_gradient_invariants_and_linearity():
+    T, d, V = 10, (8, 16, 24), 30
+    H, W, y = problem(T, d, V, seed=9, ws=0.4)
+    y[4] = -1
+    kw = dict(teacher=2, tau=1.5, alpha=0.6)
+    dH, dW = orc.backward(H, W, y, w=(1.0, 1.0, 1.0), grad_scale=1.0, **kw)
+    for m in range(3):
+        # every row of dL/dz sums to zero, so the columns of dW do too
+        assert np.abs(dW[m].sum(0)).max() <= 1e-13 * max(1.0, np.abs(dW[m]).max()) * V
+        assert np.abs(dH[m][4]).max() == 0.0          # ignored token
+    dH2, dW2 = orc.backward(H, W, y, w=(2.0, 1.0, 3.0), grad_scale=1.5, **kw)
+    for m, f in enumerate((3.0, 1.5, 4.5)):
+        np.testing.assert_allclose(dH2[m], f * dH[m], rtol=1e-12, atol=1e-16)
+        np.testing.assert_allclose(dW2[m], f * dW[m], rtol=1e-12, atol=1e-16)
+    a = orc.forward(H, W, y, w=(1.0, 1.0, 1.0), **kw)["loss"]
+    b = orc.forward(H, W, y, w=(2.0, 2.0, 2.0), **kw)["loss"]
+    assert b == pytest.approx(2 * a, rel=1e-14)
+    # the teacher's gradient depends on neither alpha nor tau
+    dH3, dW3 = orc.backward(H, W, y, w=(1.0, 1.0, 1.0), teacher=2, tau=0.4, alpha=0.1)
+    np.testing.assert_allclose(dH3[2], dH[2], rtol=1e-12, atol=1e-16)
+    np.testing.assert_allclose(dW3[2], dW[2], rtol=1e-12, atol=1e-16)
+
+
+def test_ignored_tokens_equal_dropping_them():
+    T, d, V = 14, (8, 16), 26
+    H, W, y = problem(T, d, V, seed=10, ws=0.4)
+    drop = np.array([1, 5, 6, 13])
+    y2 = y.copy()
+    y2[drop] = -1
+    keep = np.setdiff1d(np.arange(T), drop)
+    kw = dict(tau=0.9, alpha=0.45)
+    full = orc.forward(H, W, y2, **kw)
+    sub = orc.forward([h[keep] for h in H], W, y[keep], **kw)
+    assert full["loss"] == pytest.approx(sub["loss"], rel=1e-13)
+    dHf, dWf = orc.backward(H, W, y2, **kw)
+    dHs, dWs = orc.backward([h[keep] for h in H], W, y[keep], **kw)
+    for m in range(2):
+        np.testing.assert_allclose(dWf[m], dWs[m], rtol=1e-11, atol=1e-15)
+        np.testing.assert_allclose(dHf[m][keep], dHs[m], rtol=1e-11, atol=1e-15)
+        assert np.abs(dHf[m][drop]).max() == 0.0
+        assert (full["tok_loss"][m][drop] == 0).all()
+
+
+def test_rows_match_full_problem():
+    T, d, V = 9, (8, 16, 8), 21
+    H, W, y = problem(T, d, V, seed=11, ws=0.4)
+    y[0] = -1
+    kw = dict(teacher=1, tau=1.2, alpha=0.5, w=(1.0, 0.5, 2.0))
+    full = orc.forward(H, W, y, **kw)
+    dH, _ = orc.backward(H, W, y, grad_scale=0.7, **kw)
+    sel = [8, 0, 3]
+    r = orc.rows(H, W, y, sel, grad_scale=0.7, **kw)
+    for key in ("tok_loss", "ce", "ld", "kl", "lse", "lse_tau"):
+        np.testing.assert_allclose(r[key], full[key][:, sel], rtol=1e-13, atol=1e-15)
+    np.testing.assert_array_equal(r["argmax"], full["argmax"][:, sel])
+    for m in range(3):
+        np.testing.assert_allclose(r["dH"][m], dH[m][sel], rtol=1e-12, atol=1e-16)
+
+
+def test_degenerate_cases():
+    T, d, V = 6, (8, 8), 10
+    H, W, y = problem(T, d, V, seed=12)
+    none = np.full(T, -1, np.int32)
+    out = orc.forward(H, W, none)
+    assert out["loss"] == 0.0
+    dH, dW = orc.backward(H, W, none)
+    assert all(np.abs(x).max() == 0 for x in dH + dW)
+    bad = y.copy()
+    bad[2] = V
+    with pytest.raises(RuntimeError):
+        orc.forward(H, W, bad)
+    # a single sub-model is plain cross-entropy
+    one = orc.forward(H[:1], W[:1], y, alpha=0.9)
+    ce = F.cross_entropy(logits(H[:1], W[:1])[0], torch.from_numpy(y.astype(np.int64)))
+    assert one["loss"] == pytest.approx(float(ce), rel=1e-13)
+    # zero tokens
+    empty = orc.forward([h[:0] for h in H], W, y[:0])
+    assert empty["loss"] == 0.0
+
+
+def test_golden_regression_fixture():
+    """The oracle still reproduces tests/golden/oracle_small.json (written by
+    tests/golden/make_golden.py, which calls only the oracle)."""
+    import json
+    import os
+
+    path = os.path.join(os.path.dirname(__file__), "golden", "oracle_small.json")
+    fx = json.load(open(path))
+    H = [np.asarray(h, np.float32) for h in fx["H"]]
+    W = [np.asarray(x, np.float32) for x in fx["W"]]
+    y = np.asarray(fx["y"], np.int32)
+    kw = dict(teacher=fx["teacher"], tau=fx["tau"], alpha=fx["alpha"], w=fx["w"])
+    f = orc.forward(H, W, y, **kw)
+    assert f["loss"] == pytest.approx(fx["loss"], rel=1e-12)
+    for k in ("tok_loss", "ce", "ld", "kl", "lse", "lse_tau"):
+        np.testing.assert_allclose(f[k], np.asarray(fx[k]), rtol=1e-12, atol=1e-15)
+    np.testing.assert_array_equal(f["argmax"], np.asarray(fx["argmax"]))
+    dH, dW = orc.backward(H, W, y, **kw)
+    for m in range(3):
+        np.testing.assert_allclose(dH[m], np.asarray(fx["dH"][m]), rtol=1e-11, atol=1e-15)
+        np.testing.assert_allclose(dW[m], np.asarray(fx["dW"][m]), rtol=1e-11, atol=1e-15)
