@@ -1,0 +1,407 @@
+#!/usr/bin/env python
+"""Benchmark of the fused Matryoshka-suite output stage on GB300.
+
+One step = one forward + backward of the whole hot path (LM heads of every
+sub-model, cross-entropy, distillation from the teacher, dH and dW) over one
+batch of T tokens of the 3-level suite shaped like 500M/1.5B/3B:
+T = 8192 (4 x 2048), d = (1024, 2048, 3072), V = 50304, bf16, tau = 1,
+alpha = 0.5, synthetic seeded inputs (the paper's FineWeb-Edu batches are
+not available).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl mls|reference]
+
+Under torchrun each rank runs its own batch on its own GPU (no collective on
+the data path: the loss of one batch needs nothing from another), so scaling
+is weak and `value` is the tokens of all ranks per second of the slowest rank.
+`--impl reference` times the fp64 CPU oracle (the reference definition of the
+method) on the host cores, on a bounded sample of the same workload.
+Rank 0 prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "tokens/s fused head+CE+KL fwd+bwd (3-level suite) and % of dense BF16 tensor peak"
+UNIT = "tokens/s"
+WORKLOAD = "suite3"
+KERNELS = ("head_fwd", "head_bwd", "gemm_dw", "gemm_dh")   # each does 2*T*V*sum(d) FLOPs per step
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as fh:
+            d = json.load(fh)
+        return d, "measured"
+    except Exception:
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+def source_hash() -> str:
+    csrc = os.path.join(ROOT, "paper_2608_09703_gb300", "csrc")
+    h = hashlib.sha256()
+    for name in sorted(os.listdir(csrc)):
+        if name.endswith((".cu", ".cuh", ".h")):
+            with open(os.path.join(csrc, name), "rb") as fh:
+                h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def traffic_for(kernel: str):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken
+    on the current kernel sources (else None)."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as fh:
+            d = json.load(fh)
+    except Exception:
+        return None
+    e = d.get(kernel)
+    if not e or e.get("source_hash") != source_hash():
+        return None
+    return e.get("traffic_bytes_per_launch")
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason samples while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.out = None
+
+    def start(self):
+        try:
+            self.out = tempfile.NamedTemporaryFile("w+", delete=False, suffix=".csv")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-i", str(self.gpu), "-lms", "100"], stdout=self.out, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.out.flush()
+        self.out.seek(0)
+        rows = [l.strip().split(",") for l in self.out.read().splitlines() if l.strip()]
+        self.out.close()
+        os.unlink(self.out.name)
+        sm, mx, power, reasons = [], None, [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for r in rows:
+            r = [x.strip() for x in r]
+            if len(r) < 9:
+                continue
+            try:
+                sm.append(float(r[1]))
+                mx = float(r[2])
+                power.append(float(r[3]))
+            except ValueError:
+                continue
+            for name, val in zip(names, r[5:9]):
+                if val.lower() == "active":
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx,
+                "reasons": sorted(reasons), "samples": len(sm),
+                "power_w_max": max(power) if power else None}
+
+
+def dist_setup():
+    import torch
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
+    return rank, world, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ------------------------------------------------------------------------- oracle timing
+def oracle_sample(wl, ntok: int, seed: int = 1234):
+    """The first `ntok` tokens of the workload's seeded inputs, as oracle arrays."""
+    import numpy as np
+
+    from paper_2608_09703_gb300 import synth
+
+    H, W, y = synth.make_inputs(wl, seed=seed)
+    Hs = synth.as_oracle_arrays([h[:ntok] for h in H])
+    Ws = synth.as_oracle_arrays(W)
+    return Hs, Ws, y[:ntok].numpy().astype(np.int32)
+
+
+def oracle_step(wl, Hs, Ws, ys):
+    from oracle import oracle
+
+    kw = dict(teacher=wl.teacher_index, tau=wl.tau, alpha=wl.alpha, w=wl.weights)
+    oracle.forward(Hs, Ws, ys, **kw)
+    oracle.backward(Hs, Ws, ys, **kw)
+
+
+def oracle_rate(wl, budget_s: float, seed: int = 1234):
+    """Calibrates the sample size to ~budget_s of CPU work, then times one
+    forward+backward of the oracle on it.  Returns (tokens/s, tokens, seconds)."""
+    from oracle import oracle
+
+    oracle.build()
+    Hs, Ws, ys = oracle_sample(wl, 2, seed)
+    t0 = time.perf_counter()
+    oracle_step(wl, Hs, Ws, ys)
+    per_tok = (time.perf_counter() - t0) / 2
+    ntok = int(max(2, min(wl.T, budget_s / max(per_tok, 1e-6))))
+    Hs, Ws, ys = oracle_sample(wl, ntok, seed)
+    t0 = time.perf_counter()
+    oracle_step(wl, Hs, Ws, ys)
+    dt = time.perf_counter() - t0
+    return ntok / dt, ntok, dt
+
+
+def reference_arm(args, rank, world):
+    from oracle import oracle
+    from paper_2608_09703_gb300 import synth
+
+    if rank != 0:
+        return
+    wl = synth.WORKLOADS[args.workload]
+    oracle.build()
+    # size each step so that warmup + steps fit in about three minutes
+    Hs, Ws, ys = oracle_sample(wl, 2)
+    t0 = time.perf_counter()
+    oracle_step(wl, Hs, Ws, ys)
+    per_tok = (time.perf_counter() - t0) / 2
+    per_step_budget = max(1.0, 180.0 / (args.steps + args.warmup))
+    ntok = int(max(1, min(wl.T, per_step_budget / max(per_tok, 1e-6))))
+    Hs, Ws, ys = oracle_sample(wl, ntok)
+    for _ in range(args.warmup):
+        oracle_step(wl, Hs, Ws, ys)
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        oracle_step(wl, Hs, Ws, ys)
+        times.append(time.perf_counter() - t0)
+    step_s = sum(times) / len(times)
+    value = ntok / step_s
+    sample = (f"first {ntok} of {wl.T} tokens of {wl.name} per step (full V={wl.V} and widths "
+              f"{list(wl.d)}); fp64 forward+backward")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_s * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": workload_config(wl, world),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": oracle.threads(), "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def workload_config(wl, world):
+    return {"workload": f"{wl.name}: 3-level Matryoshka suite head+CE+distillation, T={wl.T} tokens "
+                        f"(4x2048), d={list(wl.d)}, V={wl.V}, bf16, tau={wl.tau}, alpha={wl.alpha}",
+            "T": wl.T, "d": list(wl.d), "V": wl.V, "tau": wl.tau, "alpha": wl.alpha,
+            "global_batch": wl.T * world, "seq_len": 2048, "parallelism": f"dp{world}",
+            "l2": "inputs larger than L2 (W 618 MB bf16), no flush"}
+
+
+# ------------------------------------------------------------------------- GPU arm
+def gpu_arm(args, rank, world, local):
+    import numpy as np
+    import torch
+
+    from paper_2608_09703_gb300 import binding as B
+    from paper_2608_09703_gb300 import synth
+
+    dev = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(dev)
+    wl = synth.WORKLOADS[args.workload]
+    H, W, y = synth.make_inputs(wl, seed=1234 + rank, device=dev)
+    op = B.HeadLoss(wl.d, wl.T, wl.V, teacher=wl.teacher_index, tau=wl.tau, alpha=wl.alpha,
+                    w=wl.weights, dtype=torch.bfloat16, device=dev)
+
+    def step():
+        op.forward(H, W, y)
+        op.backward(H, W, y)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    status = B.mls_get_status()
+    if status:
+        raise RuntimeError(f"device status after warm-up: {B.mls_strerror(status)}")
+
+    # ---- timed region
+    sampler = ClockSampler(dev.index if dev.index is not None else 0)
+    stream = torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    torch.cuda.synchronize()
+    sampler.start()
+    time.sleep(0.25)
+    B.mls_profile_enable(True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    kern = B.mls_profile_read()
+    B.mls_profile_enable(False)
+    clocks = sampler.stop()
+    barrier(world)
+    ms = e0.elapsed_time(e1) / args.steps
+    ms_max = max_over_ranks(ms, world)
+    value = world * wl.T / (ms_max / 1e3)
+
+    pk, pk_src = peaks()
+    step_flops = wl.flops_fwd_bwd()
+    per_kernel = {}
+    for name, (launches, total_ms) in kern.items():
+        entry = {"launches_per_step": launches / args.steps, "ms_per_step": total_ms / args.steps}
+        if name in KERNELS:
+            flops_launch = (step_flops / 4) / (launches / args.steps)
+            entry["tflops"] = flops_launch / (total_ms / launches / 1e3) / 1e12
+        per_kernel[name] = entry
+    dom = max((k for k in KERNELS if k in kern), key=lambda k: kern[k][1])
+    launches, total_ms = kern[dom]
+    flops_launch = (step_flops / 4) / (launches / args.steps)
+    achieved = flops_launch / (total_ms / launches / 1e3) / 1e12
+    peak = float(pk["bf16_tflops"])
+    roofline = {"bound": "tensor", "kernel": dom, "achieved": achieved, "peak": peak,
+                "unit": "TFLOP/s", "frac": achieved / peak,
+                "frac_of_sustained": achieved / float(pk["bf16_tflops_sustained"]),
+                "peak_source": f"{pk_src} bf16 dense burst (MEASURED_PEAKS.json)" if pk_src == "measured"
+                else "fallback 1.9 PFLOP/s bf16",
+                "flops_per_launch": flops_launch,
+                "traffic": traffic_for(dom)}
+    gpu_launches = sum(v[0] for v in kern.values())
+
+    # ---- end to end through the C ABI with host buffers (pinned), copies timed
+    Hh = [h.cpu().pin_memory() for h in H]
+    Wh = [w.cpu().pin_memory() for w in W]
+    yh = y.cpu().pin_memory()
+    loss_h = torch.empty(1, dtype=torch.float32).pin_memory()
+    Hd = [torch.empty_like(h) for h in H]
+    Wd = [torch.empty_like(w) for w in W]
+    yd = torch.empty_like(y)
+    h2d = sum(t.numel() * t.element_size() for t in Hh + Wh) + yh.numel() * yh.element_size()
+    d2h = loss_h.numel() * loss_h.element_size()
+
+    def e2e_step():
+        for src, dst in zip(Hh + Wh + [yh], Hd + Wd + [yd]):
+            dst.copy_(src, non_blocking=True)
+        op.forward(Hd, Wd, yd)
+        op.backward(Hd, Wd, yd)
+        loss_h.copy_(op.loss, non_blocking=True)
+
+    n_e2e = max(3, min(args.steps, 10))
+    e2e_step()
+    torch.cuda.synchronize()
+    barrier(world)
+    t0 = time.perf_counter()
+    e0.record(stream)
+    for _ in range(n_e2e):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = max(e0.elapsed_time(e1), (time.perf_counter() - t0) * 1e3) / n_e2e
+    e2e_ms = max_over_ranks(e2e_ms, world)
+    e2e = {"value": world * wl.T / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+           "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms}
+    status = B.mls_get_status()
+    if status:
+        raise RuntimeError(f"device status: {B.mls_strerror(status)}")
+
+    if rank != 0:
+        return
+    cpu = None
+    if world == 1 and not args.no_cpu_baseline:
+        rate, ntok, secs = oracle_rate(wl, budget_s=15.0)
+        from oracle import oracle
+
+        cpu = {"value": rate, "unit": UNIT, "cores": oracle.threads(), "kind": "oracle",
+               "sample": f"first {ntok} of {wl.T} tokens of {wl.name} (full V and widths), "
+                         f"fp64 forward+backward, {secs:.1f} s"}
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded N(0,1) hidden states, "
+        "N(0,0.02^2) heads, uniform targets; FineWeb-Edu not available)",
+        "config": workload_config(wl, world),
+        "tensor_frac_step": step_flops / (ms_max / 1e3) / 1e12 / peak,
+        "roofline": roofline, "kernels": per_kernel, "gpu_launches": gpu_launches,
+        "clocks": clocks, "e2e": e2e, "cpu_baseline": cpu,
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="mls", choices=["mls", "reference"])
+    ap.add_argument("--workload", default=WORKLOAD)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        # rank 0 alone times the CPU oracle; other ranks exit without work
+        reference_arm(args, int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")))
+        return
+    rank, world, local = dist_setup()
+    try:
+        gpu_arm(args, rank, world, local)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

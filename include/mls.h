@@ -1,0 +1,150 @@
+/*
+ * mls.h -- C ABI of the fused Matryoshka-suite output stage on GB300 (sm_103a).
+ *
+ * The operation (paper: "Matryoshka Language Model Suites", Sec. 2):
+ *   for every nested sub-model m = 0..M-1 with hidden states H_m [T, d_m] and
+ *   LM head W_m [V, d_m] (Sec. 2, "Inter-model Junction": W^m in R^{V x D_m}),
+ *     z_m    = H_m W_m^T                                    (never stored)
+ *     CE_m   = logsumexp(z_m) - z_m[y]                      (Sec. 2, "Modeling")
+ *     Ld_m   = -sum_v q_v log softmax(z_m / tau)_v,  q = stop_grad(softmax(z_t / tau))
+ *              with t the teacher sub-model                 (Eq. 2)
+ *     L_m    = (1 - alpha) CE_m + alpha Ld_m  for m != t;  L_t = CE_t   (Eq. 3)
+ *     loss   = sum_m w_m (1/N) sum_{tokens with y >= 0} L_m           (sum after Eq. 3, App. G)
+ *   and its gradients dH_m, dW_m (teacher distribution under stop-gradient).
+ *   tau is an extension: Eq. 2 is the case tau = 1.  The [T, V] logits of a
+ *   sub-model are never written to memory.
+ *
+ * Conventions shared by every entry point:
+ *   - Pointer arguments named H, W, targets, loss, tok_loss, tok_diag, argmax,
+ *     stats, dH, dW and ws are DEVICE pointers owned by the caller; the arrays
+ *     H, W, dH, dW themselves (the pointer lists, length M) and everything in
+ *     mls_problem are HOST memory read during the call only.
+ *   - All matrices are row-major and dense: H_m has row pitch d_m elements,
+ *     W_m row pitch d_m, dH_m and dW_m row pitch d_m floats.  H_m and W_m must be
+ *     16-byte aligned and d_m * sizeof(element) a multiple of 16 bytes.
+ *   - Calls are asynchronous on `stream`; nothing is allocated and the host
+ *     never synchronises.  The caller provides a workspace of at least
+ *     mls_workspace_size() bytes (256-byte aligned); its contents need not be
+ *     preserved between calls.
+ *   - Return value: 0 on success or a negative MLS_ERR_* code, in which case
+ *     nothing was launched.  Conditions only the device can see (a target >= V,
+ *     an internal wait that timed out) are recorded in a status word read by
+ *     mls_get_status().
+ */
+#ifndef MLS_H
+#define MLS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same object as cudaStream_t; NULL is the legacy default stream. */
+typedef struct CUstream_st* mls_stream_t;
+
+/* Storage type of H and W.  Outputs are always fp32. */
+enum { MLS_BF16 = 0, MLS_FP32 = 1 };
+
+/* Return codes (negative) and status bits (positive, from mls_get_status). */
+enum {
+  MLS_OK = 0,
+  MLS_ERR_ARG = -1,          /* null pointer, size or parameter out of range */
+  MLS_ERR_ALIGN = -2,        /* a device pointer breaks the alignment rules above */
+  MLS_ERR_UNSUPPORTED = -3,  /* shape the kernels do not handle (see mls_problem) */
+  MLS_ERR_WORKSPACE = -4,    /* workspace NULL, misaligned or smaller than required */
+  MLS_ERR_CUDA = -5,         /* a CUDA runtime call or kernel launch failed */
+  MLS_ERR_DEVICE = -6,       /* current device is not a compute-capability 10.3 GPU */
+  MLS_STATUS_BAD_TARGET = 1, /* some target was >= V; that token was treated as ignored */
+  MLS_STATUS_TIMEOUT = 2     /* a pipeline wait exceeded its bound; outputs are invalid */
+};
+
+/* Maximum number of sub-models per call. */
+#define MLS_MAX_MODELS 4
+
+typedef struct {
+  int32_t M;            /* sub-models, 1..MLS_MAX_MODELS */
+  int64_t T;            /* tokens, >= 0 */
+  int64_t V;            /* vocabulary size, 1 .. 2^31 - 1 */
+  const int32_t* d;     /* host array [M]: width d_m of sub-model m (> 0) */
+  int32_t teacher;      /* distillation teacher, 0..M-1 (paper: M-1, the largest) */
+  float tau;            /* distillation temperature > 0 (paper: 1) */
+  float alpha;          /* alpha_d of Eq. 3, in [0, 1] */
+  const float* w;       /* host array [M] of loss weights (App. G), or NULL for all 1 */
+  int32_t in_dtype;     /* MLS_BF16 or MLS_FP32: storage type of every H_m and W_m */
+  int64_t vocab_group;  /* backward vocabulary group (columns), multiple of 256, or 0 = automatic */
+} mls_problem;
+
+/*
+ * Bytes of device workspace that mls_head_loss_fwd and mls_head_loss_bwd need
+ * for this problem (the larger of the two).  Returns 0 if the problem is
+ * invalid.  The backward keeps the gradient of the logits for one vocabulary
+ * group, bf16 [M, T, group] (fp32 for MLS_FP32 inputs), in this workspace.
+ */
+size_t mls_workspace_size(const mls_problem* p);
+
+/*
+ * Forward (Eq. 2, Eq. 3, weighted sum over sub-models).
+ *   H[m]      device, [T, d_m] in_dtype      hidden states of sub-model m
+ *   W[m]      device, [V, d_m] in_dtype      LM head of sub-model m
+ *   targets   device, int32 [T]; < 0 = ignored token
+ *   loss      device, fp32 [1]               the scalar objective
+ *   tok_loss  device, fp32 [M, T]            L_m per token (0 for ignored tokens)
+ *   tok_diag  device, fp32 [3, M, T] or NULL CE_m, Ld_m and KL_m = Ld_m - H(q) per token
+ *   argmax    device, int32 [M, T] or NULL   argmax_v z_m (lowest index on ties)
+ *   stats     device, fp32 [2, M, T]         logsumexp(z_m) and logsumexp(z_m / tau);
+ *                                            the backward needs them
+ *   ws        device workspace, ws_bytes >= mls_workspace_size(p)
+ */
+int mls_head_loss_fwd(const mls_problem* p, const void* const* H, const void* const* W,
+                      const int32_t* targets, float* loss, float* tok_loss, float* tok_diag,
+                      int32_t* argmax, float* stats, void* ws, size_t ws_bytes,
+                      mls_stream_t stream);
+
+/*
+ * Backward: gradients of grad_scale * loss.
+ *   stats     device, fp32 [2, M, T] as written by mls_head_loss_fwd for the same inputs
+ *   dH[m]     device, fp32 [T, d_m]    overwritten with d(loss)/dH_m
+ *   dW[m]     device, fp32 [V, d_m]    overwritten with d(loss)/dW_m
+ * The teacher's parameters get only the gradient of w_t * mean CE_t: Eq. 2 stops
+ * the gradient through q.  The logits are recomputed, never read from memory.
+ */
+int mls_head_loss_bwd(const mls_problem* p, const void* const* H, const void* const* W,
+                      const int32_t* targets, const float* stats, float grad_scale,
+                      float* const* dH, float* const* dW, void* ws, size_t ws_bytes,
+                      mls_stream_t stream);
+
+/*
+ * Synchronises `stream`, then returns the status bits (MLS_STATUS_*) recorded by
+ * the device on the current device since the last call and clears them; returns
+ * a negative MLS_ERR_CUDA if the synchronisation or the read failed.
+ */
+int mls_get_status(mls_stream_t stream);
+
+/* Static description of a return code or status bit. */
+const char* mls_strerror(int code);
+
+/*
+ * Kernel timing (a tracing aid; not part of the paper's method).  While
+ * enabled, every kernel the library launches is bracketed by two CUDA events
+ * recorded on the launch stream.  mls_profile_read synchronises on the last
+ * event, then fills up to `n` records (kernel name, launch count, summed
+ * device time in ms), aggregated by kernel since the last enable/read, and
+ * returns how many kernels it saw; the records are cleared.  Host-side state
+ * only; thread-unsafe with concurrent calls on other threads.
+ */
+typedef struct {
+  const char* name;   /* static string, e.g. "head_fwd" */
+  int launches;
+  double total_ms;
+} mls_kernel_time;
+
+int mls_profile_enable(int on);
+int mls_profile_read(mls_kernel_time* out, int n);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MLS_H */

@@ -88,13 +88,30 @@ static int check_problem(const mls_oracle_problem* p) {
 
 static double weight(const mls_oracle_problem* p, int m) { return p->w ? p->w[m] : 1.0; }
 
-/* z[v] = sum_k H[t,k] W[v,k] for every v: the full logit row of one token. */
+/* z[v] = sum_k H[t,k] W[v,k] for every v: the full logit row of one token.
+   (The storage type is switched on outside the loops; every product and the
+   order of the sum over k are the same as elem(H) * elem(W) summed k = 0..d-1.) */
 static void logits_row(const mls_oracle_problem* p, const void* H, const void* W, int dm,
                        long long t, double* z) {
+  double h[dm > 0 ? dm : 1];
+  for (int k = 0; k < dm; ++k) h[k] = elem(H, p->in_dtype, t * dm + k);
   for (long long v = 0; v < p->V; ++v) {
     double acc = 0.0;
-    for (int k = 0; k < dm; ++k)
-      acc += elem(H, p->in_dtype, t * dm + k) * elem(W, p->in_dtype, v * dm + k);
+    if (p->in_dtype == 0) {
+      const uint16_t* w = (const uint16_t*)W + v * dm;
+      for (int k = 0; k < dm; ++k) {
+        uint32_t bits = ((uint32_t)w[k]) << 16;
+        float f;
+        memcpy(&f, &bits, sizeof f);
+        acc += h[k] * (double)f;
+      }
+    } else if (p->in_dtype == 1) {
+      const float* w = (const float*)W + v * dm;
+      for (int k = 0; k < dm; ++k) acc += h[k] * (double)w[k];
+    } else {
+      const double* w = (const double*)W + v * dm;
+      for (int k = 0; k < dm; ++k) acc += h[k] * w[k];
+    }
     z[v] = acc;
   }
 }

@@ -1,0 +1,17 @@
+"""GB300-native fused output stage of Matryoshka language-model suites.
+
+For every nested sub-model the LM-head logits, the next-token cross-entropy
+and the distillation term from the teacher sub-model (paper Eq. 2, Eq. 3),
+forward and backward, in hand-written sm_103a kernels behind the C ABI of
+include/mls.h.  ``binding`` is the Python face of that ABI.
+"""
+from .binding import (  # noqa: F401
+    HeadLoss,
+    MLSError,
+    Problem,
+    mls_get_status,
+    mls_head_loss_bwd,
+    mls_head_loss_fwd,
+    mls_strerror,
+    mls_workspace_size,
+)

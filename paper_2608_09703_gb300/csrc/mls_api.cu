@@ -1,0 +1,562 @@
+// Host side of the C ABI declared in include/mls.h: argument validation,
+// workspace planning, TMA tensor-map encoding and the launch sequences of the
+// forward and backward passes.  Nothing here allocates device memory.
+#include <cudaTypedefs.h>
+
+#include <climits>
+#include <cmath>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+#include <vector>
+
+#include "mls.h"
+#include "mls_kernels.h"
+
+namespace mls {
+namespace {
+
+__device__ int g_status;  // MLS_STATUS_* bits raised by the kernels
+
+constexpr int kMaxDevices = 64;
+
+struct DeviceState {
+  bool ready = false;
+  int err = 0;
+  int sms = 0;
+  int* status = nullptr;
+};
+
+std::mutex g_mu;
+DeviceState g_dev[kMaxDevices];
+
+// With MLS_DEBUG set in the environment, failures are described on stderr.
+int fail(int code, const char* what, cudaError_t e = cudaSuccess) {
+  static const bool verbose = std::getenv("MLS_DEBUG") != nullptr;
+  if (verbose)
+    std::fprintf(stderr, "[mls] %s failed: %s%s%s\n", what, e != cudaSuccess ? cudaGetErrorName(e) : "",
+                 e != cudaSuccess ? " " : "", e != cudaSuccess ? cudaGetErrorString(e) : "");
+  return code;
+}
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+// Checks the current device once and prepares the kernels for it.
+int device_state(DeviceState** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return MLS_ERR_CUDA;
+  if (dev < 0 || dev >= kMaxDevices) return MLS_ERR_DEVICE;
+  std::lock_guard<std::mutex> lk(g_mu);
+  DeviceState& s = g_dev[dev];
+  if (!s.ready) {
+    s.ready = true;
+    int major = 0, minor = 0;
+    cudaError_t e;
+    if ((e = cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev)) != cudaSuccess ||
+        (e = cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev)) != cudaSuccess ||
+        (e = cudaDeviceGetAttribute(&s.sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) {
+      s.err = fail(MLS_ERR_CUDA, "device query", e);
+    } else if (major != 10 || minor != 3) {
+      s.err = fail(MLS_ERR_DEVICE, "device check (need compute capability 10.3)");
+    } else if ((e = cudaGetSymbolAddress(reinterpret_cast<void**>(&s.status), g_status)) != cudaSuccess) {
+      s.err = fail(MLS_ERR_CUDA, "cudaGetSymbolAddress(status)", e);
+    } else if ((e = setup_head_kernels()) != cudaSuccess) {
+      s.err = fail(MLS_ERR_CUDA, "head kernel attributes", e);
+    } else if ((e = setup_gemm_kernels()) != cudaSuccess) {
+      s.err = fail(MLS_ERR_CUDA, "gemm kernel attributes", e);
+    } else if (!g_encode) {
+      void* fn = nullptr;
+      cudaDriverEntryPointQueryResult q;
+      if ((e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000,
+                                                cudaEnableDefault, &q)) != cudaSuccess ||
+          q != cudaDriverEntryPointSuccess || !fn) {
+        s.err = fail(MLS_ERR_CUDA, "cuTensorMapEncodeTiled entry point", e);
+      } else {
+        g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+      }
+    }
+  }
+  *out = &s;
+  return s.err;
+}
+
+int current_sms() {
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) == cudaSuccess &&
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && sms > 0)
+    return sms;
+  cudaGetLastError();
+  return 152;  // GB300
+}
+
+// ------------------------------------------------------------------ planning
+constexpr size_t kAlign = 256;
+size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+long long ceil_div(long long a, long long b) { return (a + b - 1) / b; }
+
+struct Plan {
+  int elt = 2;
+  int ntt = 0, nvt = 0;
+  // forward
+  int S = 1, nparts = 0, merge_blocks = 0;
+  size_t off_part = 0, off_bsum = 0, off_bcnt = 0, fwd_bytes = 0;
+  // backward
+  long long group = 0, ngroups = 0;
+  size_t off_invn = 0, off_G = 0, bwd_bytes = 0;
+  // fp32 inputs only: K-major copies G^T [M][group][t_pitch], H_m^T [d_m][t_pitch],
+  // W_m^T [d_m][v_pitch] for the tf32 GEMMs
+  long long t_pitch = 0, v_pitch = 0;
+  size_t off_GT = 0, off_HT[kMaxModels] = {}, off_WT[kMaxModels] = {};
+  size_t total = 0;
+};
+
+// CTAs per token tile: about eight waves of one CTA per SM.
+int choose_splits(int ntt, long long tiles, int sms) {
+  long long s = std::llround(8.0 * sms / (ntt > 0 ? ntt : 1));
+  if (s < 1) s = 1;
+  if (s > tiles) s = tiles;
+  return static_cast<int>(s < 1 ? 1 : s);
+}
+
+int validate(const mls_problem* p) {
+  if (!p || p->M < 1 || p->M > MLS_MAX_MODELS || p->T < 0 || p->V < 1 || p->V > INT_MAX ||
+      p->T > INT_MAX || !p->d)
+    return MLS_ERR_ARG;
+  if (p->teacher < 0 || p->teacher >= p->M) return MLS_ERR_ARG;
+  if (!(p->tau > 0.f) || !std::isfinite(p->tau)) return MLS_ERR_ARG;
+  if (!(p->alpha >= 0.f && p->alpha <= 1.f)) return MLS_ERR_ARG;
+  if (p->in_dtype != MLS_BF16 && p->in_dtype != MLS_FP32) return MLS_ERR_ARG;
+  if (p->vocab_group < 0 || p->vocab_group % kHeadBN != 0) return MLS_ERR_ARG;
+  const int elt = p->in_dtype == MLS_BF16 ? 2 : 4;
+  for (int m = 0; m < p->M; ++m) {
+    if (p->d[m] < 1) return MLS_ERR_ARG;
+    if ((static_cast<long long>(p->d[m]) * elt) % 16 != 0) return MLS_ERR_UNSUPPORTED;
+  }
+  if (p->w)
+    for (int m = 0; m < p->M; ++m)
+      if (!std::isfinite(p->w[m])) return MLS_ERR_ARG;
+  return MLS_OK;
+}
+
+Plan make_plan(const mls_problem* p, int sms) {
+  Plan pl;
+  pl.elt = p->in_dtype == MLS_BF16 ? 2 : 4;
+  const long long T = p->T, V = p->V, M = p->M;
+  pl.ntt = static_cast<int>(ceil_div(T, kHeadBM));
+  pl.nvt = static_cast<int>(ceil_div(V, kHeadBN));
+  pl.S = choose_splits(pl.ntt, pl.nvt, sms);
+  pl.nparts = 2 * pl.S;
+  pl.merge_blocks = static_cast<int>(ceil_div(T, kMergeThreads));
+  size_t o = 0;
+  pl.off_part = o;
+  o = align_up(o + sizeof(float) * static_cast<size_t>(pl.nparts) * kPartFields * M * T);
+  pl.off_bsum = o;
+  o = align_up(o + sizeof(double) * static_cast<size_t>(pl.merge_blocks + 1));
+  pl.off_bcnt = o;
+  o = align_up(o + sizeof(long long) * static_cast<size_t>(pl.merge_blocks + 1));
+  pl.fwd_bytes = o;
+
+  // Backward vocabulary groups: the bf16 (fp32) gradient of the logits of one
+  // group of columns for every sub-model stays within ~2 GiB unless the caller
+  // chose the group width.
+  const long long vpad = static_cast<long long>(pl.nvt) * kHeadBN;
+  long long gmax = p->vocab_group;
+  if (gmax == 0) {
+    const long long budget = 2LL << 30;
+    const long long per_col = M * (T > 0 ? T : 1) * pl.elt;
+    gmax = budget / per_col / kHeadBN * kHeadBN;
+    if (gmax < 2048) gmax = 2048;
+  }
+  if (gmax > vpad) gmax = vpad;
+  pl.ngroups = ceil_div(vpad, gmax);
+  pl.group = ceil_div(ceil_div(vpad, pl.ngroups), kHeadBN) * kHeadBN;
+  pl.ngroups = ceil_div(vpad, pl.group);
+  o = 0;
+  pl.off_invn = o;
+  o = align_up(o + sizeof(float));
+  pl.off_G = o;
+  o = align_up(o + static_cast<size_t>(pl.elt) * M * T * pl.group);
+  if (pl.elt == 4) {
+    pl.t_pitch = ceil_div(T, 4) * 4;
+    pl.v_pitch = ceil_div(V, 4) * 4;
+    pl.off_GT = o;
+    o = align_up(o + sizeof(float) * static_cast<size_t>(M) * pl.group * pl.t_pitch);
+    for (int m = 0; m < p->M; ++m) {
+      pl.off_HT[m] = o;
+      o = align_up(o + sizeof(float) * static_cast<size_t>(p->d[m]) * pl.t_pitch);
+      pl.off_WT[m] = o;
+      o = align_up(o + sizeof(float) * static_cast<size_t>(p->d[m]) * pl.v_pitch);
+    }
+  }
+  pl.bwd_bytes = o;
+  pl.total = pl.fwd_bytes > pl.bwd_bytes ? pl.fwd_bytes : pl.bwd_bytes;
+  return pl;
+}
+
+bool aligned16(const void* ptr) { return (reinterpret_cast<uintptr_t>(ptr) & 15u) == 0; }
+
+// 2-D row-major tensor [rows, cols] of `elt`-byte elements, 128-byte swizzle.
+int encode(CUtensorMap* map, const void* ptr, int elt, long long cols, long long rows,
+           long long pitch_elems, int box_cols, int box_rows) {
+  const cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(pitch_elems) * elt};
+  const cuuint32_t box[2] = {static_cast<cuuint32_t>(box_cols), static_cast<cuuint32_t>(box_rows)};
+  const cuuint32_t estr[2] = {1, 1};
+  const CUresult r = g_encode(
+      map, elt == 2 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2,
+      const_cast<void*>(ptr), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+      CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+      CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    char what[160];
+    std::snprintf(what, sizeof what, "cuTensorMapEncodeTiled (CUresult %d, %lld x %lld, box %d x %d)",
+                  static_cast<int>(r), cols, rows, box_cols, box_rows);
+    return fail(MLS_ERR_CUDA, what);
+  }
+  return MLS_OK;
+}
+
+void fill_head_common(HeadParams& hp, const mls_problem* p, const Plan& pl, const int* y,
+                      int* status) {
+  const int KE = 128 / pl.elt;
+  hp.M = p->M;
+  hp.order[0] = p->teacher;
+  for (int m = 0, j = 1; m < p->M; ++m)
+    if (m != p->teacher) hp.order[j++] = m;
+  for (int m = 0; m < p->M; ++m) hp.nk[m] = static_cast<int>(ceil_div(p->d[m], KE));
+  hp.ntt = pl.ntt;
+  hp.T = p->T;
+  hp.V = p->V;
+  hp.L1 = 1.4426950408889634f;
+  hp.Ltau = static_cast<float>(1.4426950408889634 / static_cast<double>(p->tau));
+  hp.y = y;
+  hp.status = status;
+}
+
+int encode_head_maps(HeadParams& hp, const mls_problem* p, const Plan& pl, const void* const* H,
+                     const void* const* W) {
+  const int KE = 128 / pl.elt;
+  for (int m = 0; m < p->M; ++m) {
+    if (encode(&hp.mapH[m], H[m], pl.elt, p->d[m], p->T, p->d[m], KE, kHeadBM) ||
+        encode(&hp.mapW[m], W[m], pl.elt, p->d[m], p->V, p->d[m], KE, kHeadBN))
+      return MLS_ERR_CUDA;
+  }
+  return MLS_OK;
+}
+
+int check_ws(const Plan& pl, void* ws, size_t ws_bytes, size_t need) {
+  if (need == 0) return MLS_OK;
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)) != 0 || ws_bytes < need)
+    return MLS_ERR_WORKSPACE;
+  return MLS_OK;
+}
+
+int launch_ok(cudaError_t e) { return e == cudaSuccess ? MLS_OK : fail(MLS_ERR_CUDA, "launch", e); }
+
+// ------------------------------------------------------------------ kernel timing
+struct ProfRec {
+  const char* name;
+  cudaEvent_t a, b;
+};
+std::mutex g_prof_mu;
+bool g_prof_on = false;
+std::vector<ProfRec> g_prof;
+std::vector<cudaEvent_t> g_event_pool;
+
+cudaEvent_t pool_event() {
+  if (!g_event_pool.empty()) {
+    cudaEvent_t e = g_event_pool.back();
+    g_event_pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+  return e;
+}
+
+// Runs `launch` (which returns a cudaError_t), bracketed by events when timing is on.
+template <class F>
+int timed(const char* name, cudaStream_t s, F&& launch) {
+  if (!g_prof_on) return launch_ok(launch());
+  std::lock_guard<std::mutex> lk(g_prof_mu);
+  cudaEvent_t a = pool_event(), b = pool_event();
+  if (a) cudaEventRecord(a, s);
+  const int rc = launch_ok(launch());
+  if (a && b) {
+    cudaEventRecord(b, s);
+    g_prof.push_back({name, a, b});
+  }
+  return rc;
+}
+
+}  // namespace
+}  // namespace mls
+
+using namespace mls;
+
+extern "C" size_t mls_workspace_size(const mls_problem* p) {
+  if (validate(p) != MLS_OK) return 0;
+  return make_plan(p, current_sms()).total;
+}
+
+extern "C" int mls_head_loss_fwd(const mls_problem* p, const void* const* H, const void* const* W,
+                                 const int32_t* targets, float* loss, float* tok_loss,
+                                 float* tok_diag, int32_t* argmax, float* stats, void* ws,
+                                 size_t ws_bytes, mls_stream_t stream) {
+  int rc = validate(p);
+  if (rc) return rc;
+  if (!H || !W || !loss || (p->T > 0 && (!targets || !tok_loss || !stats))) return MLS_ERR_ARG;
+  for (int m = 0; m < p->M; ++m) {
+    if (!H[m] || !W[m]) return MLS_ERR_ARG;
+    if (!aligned16(H[m]) || !aligned16(W[m])) return MLS_ERR_ALIGN;
+  }
+  DeviceState* dev = nullptr;
+  if ((rc = device_state(&dev))) return rc;
+  const Plan pl = make_plan(p, dev->sms);
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (p->T == 0) return launch_ok(cudaMemsetAsync(loss, 0, sizeof(float), s));
+  if ((rc = check_ws(pl, ws, ws_bytes, pl.total))) return rc;
+  char* wsb = static_cast<char*>(ws);
+
+  HeadParams hp;
+  std::memset(&hp, 0, sizeof hp);
+  fill_head_common(hp, p, pl, targets, dev->status);
+  if ((rc = encode_head_maps(hp, p, pl, H, W))) return rc;
+  hp.vt_begin = 0;
+  hp.vt_end = pl.nvt;
+  hp.S = pl.S;
+  hp.part = reinterpret_cast<float*>(wsb + pl.off_part);
+  if ((rc = timed("head_fwd", s, [&] { return launch_head_fwd(hp, pl.elt == 4, p->tau == 1.0f, s); }))) return rc;
+
+  MergeParams mp;
+  std::memset(&mp, 0, sizeof mp);
+  mp.part = hp.part;
+  mp.nparts = pl.nparts;
+  mp.M = p->M;
+  mp.teacher = p->teacher;
+  mp.T = p->T;
+  mp.V = p->V;
+  mp.L1 = hp.L1;
+  mp.Ltau = hp.Ltau;
+  mp.tau = p->tau;
+  mp.alpha = p->alpha;
+  for (int m = 0; m < p->M; ++m) mp.w[m] = p->w ? p->w[m] : 1.0f;
+  mp.y = targets;
+  mp.tok_loss = tok_loss;
+  mp.tok_diag = tok_diag;
+  mp.argmax = argmax;
+  mp.stats = stats;
+  mp.block_sum = reinterpret_cast<double*>(wsb + pl.off_bsum);
+  mp.block_cnt = reinterpret_cast<long long*>(wsb + pl.off_bcnt);
+  mp.status = dev->status;
+  if ((rc = timed("merge", s, [&] { return launch_merge(mp, pl.merge_blocks, s); }))) return rc;
+  return timed("final", s, [&] { return launch_final(mp.block_sum, mp.block_cnt, pl.merge_blocks, loss, s); });
+}
+
+extern "C" int mls_head_loss_bwd(const mls_problem* p, const void* const* H, const void* const* W,
+                                 const int32_t* targets, const float* stats, float grad_scale,
+                                 float* const* dH, float* const* dW, void* ws, size_t ws_bytes,
+                                 mls_stream_t stream) {
+  int rc = validate(p);
+  if (rc) return rc;
+  if (!H || !W || !dH || !dW || (p->T > 0 && (!targets || !stats))) return MLS_ERR_ARG;
+  if (!std::isfinite(grad_scale)) return MLS_ERR_ARG;
+  for (int m = 0; m < p->M; ++m) {
+    if (!H[m] || !W[m] || !dW[m] || (p->T > 0 && !dH[m])) return MLS_ERR_ARG;
+    if (!aligned16(H[m]) || !aligned16(W[m]) || !aligned16(dW[m]) || !aligned16(dH[m]))
+      return MLS_ERR_ALIGN;
+  }
+  DeviceState* dev = nullptr;
+  if ((rc = device_state(&dev))) return rc;
+  const Plan pl = make_plan(p, dev->sms);
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (p->T == 0) {
+    for (int m = 0; m < p->M; ++m)
+      if ((rc = launch_ok(cudaMemsetAsync(dW[m], 0, sizeof(float) * p->V * p->d[m], s)))) return rc;
+    return MLS_OK;
+  }
+  if ((rc = check_ws(pl, ws, ws_bytes, pl.total))) return rc;
+  char* wsb = static_cast<char*>(ws);
+  const bool tf32 = pl.elt == 4;
+  const int KE = 128 / pl.elt;
+  float* inv_n = reinterpret_cast<float*>(wsb + pl.off_invn);
+  void* G = wsb + pl.off_G;
+
+  if ((rc = timed("count", s, [&] { return launch_count(targets, p->T, p->V, inv_n, dev->status, s); }))) return rc;
+
+  HeadParams hp;
+  std::memset(&hp, 0, sizeof hp);
+  fill_head_common(hp, p, pl, targets, dev->status);
+  if ((rc = encode_head_maps(hp, p, pl, H, W))) return rc;
+  hp.stats = stats;
+  hp.inv_n = inv_n;
+  for (int m = 0; m < p->M; ++m) hp.coef[m] = grad_scale * (p->w ? p->w[m] : 1.0f);
+  hp.one_minus_alpha = 1.0f - p->alpha;
+  hp.alpha_over_tau = p->alpha / p->tau;
+  hp.G = G;
+  hp.g_pitch = pl.group;
+  hp.g_model_stride = p->T * pl.group;
+
+  // bf16: dW reads A = G viewed M-major and B = H viewed N-major, dH reads
+  // A = G K-major and B = W viewed N-major, all in place.
+  // fp32 (tf32 MMA): dW reads A = G^T and B = H^T, dH reads A = G and B = W^T,
+  // all K-major.
+  GemmParams gw, gh;
+  std::memset(&gw, 0, sizeof gw);
+  std::memset(&gh, 0, sizeof gh);
+  float* GT = tf32 ? reinterpret_cast<float*>(wsb + pl.off_GT) : nullptr;
+  for (int m = 0; m < p->M; ++m) {
+    const void* Gm = static_cast<const char*>(G) + static_cast<size_t>(pl.elt) * hp.g_model_stride * m;
+    if (encode(&gh.mapA[m], Gm, pl.elt, pl.group, p->T, pl.group, KE, kGemmBM)) return MLS_ERR_CUDA;
+    if (!tf32) {
+      if (encode(&gw.mapA[m], Gm, pl.elt, pl.group, p->T, pl.group, KE, KE) ||
+          encode(&gw.mapB[m], H[m], pl.elt, p->d[m], p->T, p->d[m], KE, KE) ||
+          encode(&gh.mapB[m], W[m], pl.elt, p->d[m], p->V, p->d[m], KE, KE))
+        return MLS_ERR_CUDA;
+    } else {
+      float* HT = reinterpret_cast<float*>(wsb + pl.off_HT[m]);
+      float* WT = reinterpret_cast<float*>(wsb + pl.off_WT[m]);
+      if ((rc = launch_ok(launch_transpose(static_cast<const float*>(H[m]), p->T, p->d[m], p->d[m],
+                                           HT, pl.t_pitch, s))) ||
+          (rc = launch_ok(launch_transpose(static_cast<const float*>(W[m]), p->V, p->d[m], p->d[m],
+                                           WT, pl.v_pitch, s))))
+        return rc;
+      if (encode(&gw.mapA[m], GT + static_cast<size_t>(m) * pl.group * pl.t_pitch, 4, p->T,
+                 pl.group, pl.t_pitch, KE, kGemmBM) ||
+          encode(&gw.mapB[m], HT, 4, p->T, p->d[m], pl.t_pitch, KE, kGemmBN) ||
+          encode(&gh.mapB[m], WT, 4, p->V, p->d[m], pl.v_pitch, KE, kGemmBN))
+        return MLS_ERR_CUDA;
+    }
+  }
+  gw.nprob = gh.nprob = p->M;
+  gw.status = gh.status = dev->status;
+
+  const long long tiles_per_group = pl.group / kHeadBN;
+  for (long long g = 0; g < pl.ngroups; ++g) {
+    const long long c0 = g * pl.group;
+    const long long gc = (p->V - c0 < pl.group) ? p->V - c0 : pl.group;  // columns of this group
+    hp.vt_begin = static_cast<int>(g * tiles_per_group);
+    hp.vt_end = static_cast<int>(ceil_div(c0 + gc, kHeadBN));
+    hp.S = choose_splits(pl.ntt, hp.vt_end - hp.vt_begin, dev->sms);
+    hp.g_col0 = c0;
+    if ((rc = timed("head_bwd", s, [&] { return launch_head_bwd(hp, tf32, p->tau == 1.0f, s); }))) return rc;
+    if (tf32)
+      for (int m = 0; m < p->M; ++m)
+        if ((rc = launch_ok(launch_transpose(
+                 reinterpret_cast<const float*>(G) + static_cast<size_t>(m) * hp.g_model_stride,
+                 p->T, pl.group, pl.group, GT + static_cast<size_t>(m) * pl.group * pl.t_pitch,
+                 pl.t_pitch, s))))
+          return rc;
+
+    int tw = 0, th = 0;
+    for (int m = 0; m < p->M; ++m) {
+      GemmProblem& a = gw.prob[m];
+      a.Mrows = static_cast<int>(gc);
+      a.Ncols = p->d[m];
+      a.K = static_cast<int>(p->T);
+      a.a_map = a.b_map = m;
+      a.C = dW[m] + c0 * p->d[m];
+      a.ldc = p->d[m];
+      a.accumulate = 0;
+      a.tiles_n = static_cast<int>(ceil_div(p->d[m], kGemmBN));
+      a.tile_begin = tw;
+      tw += static_cast<int>(ceil_div(gc, kGemmBM)) * a.tiles_n;
+
+      GemmProblem& b = gh.prob[m];
+      b.Mrows = static_cast<int>(p->T);
+      b.Ncols = p->d[m];
+      b.K = static_cast<int>(gc);
+      b.a_map = b.b_map = m;
+      b.b_k0 = static_cast<int>(c0);
+      b.C = dH[m];
+      b.ldc = p->d[m];
+      b.accumulate = g > 0 ? 1 : 0;
+      b.tiles_n = static_cast<int>(ceil_div(p->d[m], kGemmBN));
+      b.tile_begin = th;
+      th += static_cast<int>(ceil_div(p->T, kGemmBM)) * b.tiles_n;
+    }
+    gw.total_tiles = tw;
+    gh.total_tiles = th;
+    const int grid_w = tw < dev->sms ? tw : dev->sms, grid_h = th < dev->sms ? th : dev->sms;
+    if (tf32) {
+      if ((rc = timed("gemm_dw", s, [&] { return launch_gemm_kk(gw, true, grid_w, s); }))) return rc;
+      if ((rc = timed("gemm_dh", s, [&] { return launch_gemm_kk(gh, true, grid_h, s); }))) return rc;
+    } else {
+      if ((rc = timed("gemm_dw", s, [&] { return launch_gemm_dw(gw, false, grid_w, s); }))) return rc;
+      if ((rc = timed("gemm_dh", s, [&] { return launch_gemm_dh(gh, false, grid_h, s); }))) return rc;
+    }
+  }
+  return MLS_OK;
+}
+
+extern "C" int mls_get_status(mls_stream_t stream) {
+  DeviceState* dev = nullptr;
+  const int rc = device_state(&dev);
+  if (rc) return rc;
+  if (cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
+    return MLS_ERR_CUDA;
+  int v = 0;
+  if (cudaMemcpy(&v, dev->status, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess)
+    return MLS_ERR_CUDA;
+  const int zero = 0;
+  if (cudaMemcpy(dev->status, &zero, sizeof zero, cudaMemcpyHostToDevice) != cudaSuccess)
+    return MLS_ERR_CUDA;
+  return v;
+}
+
+extern "C" const char* mls_strerror(int code) {
+  switch (code) {
+    case MLS_OK: return "success";
+    case MLS_ERR_ARG: return "invalid argument";
+    case MLS_ERR_ALIGN: return "device pointer not 16-byte aligned";
+    case MLS_ERR_UNSUPPORTED: return "unsupported shape (row of H/W not a multiple of 16 bytes)";
+    case MLS_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+    case MLS_ERR_CUDA: return "CUDA runtime or launch failure";
+    case MLS_ERR_DEVICE: return "current device is not compute capability 10.3";
+    case MLS_STATUS_BAD_TARGET: return "a target was >= V (token ignored)";
+    case MLS_STATUS_TIMEOUT: return "a pipeline wait timed out; outputs are invalid";
+    case MLS_STATUS_BAD_TARGET | MLS_STATUS_TIMEOUT: return "target >= V and a pipeline timeout";
+    default: return "unknown code";
+  }
+}
+
+extern "C" int mls_profile_enable(int on) {
+  std::lock_guard<std::mutex> lk(g_prof_mu);
+  g_prof_on = on != 0;
+  for (auto& r : g_prof) {
+    g_event_pool.push_back(r.a);
+    g_event_pool.push_back(r.b);
+  }
+  g_prof.clear();
+  return MLS_OK;
+}
+
+extern "C" int mls_profile_read(mls_kernel_time* out, int n) {
+  std::lock_guard<std::mutex> lk(g_prof_mu);
+  if (!g_prof.empty() && cudaEventSynchronize(g_prof.back().b) != cudaSuccess) return MLS_ERR_CUDA;
+  int k = 0;
+  const char* names[32];
+  int launches[32];
+  double ms[32];
+  for (auto& r : g_prof) {
+    float t = 0.f;
+    cudaEventElapsedTime(&t, r.a, r.b);
+    int i = 0;
+    while (i < k && std::strcmp(names[i], r.name) != 0) ++i;
+    if (i == k && k < 32) {
+      names[k] = r.name;
+      launches[k] = 0;
+      ms[k] = 0.0;
+      ++k;
+    }
+    if (i < 32) {
+      launches[i] += 1;
+      ms[i] += t;
+    }
+    g_event_pool.push_back(r.a);
+    g_event_pool.push_back(r.b);
+  }
+  g_prof.clear();
+  for (int i = 0; i < k && i < n; ++i) out[i] = {names[i], launches[i], ms[i]};
+  return k;
+}

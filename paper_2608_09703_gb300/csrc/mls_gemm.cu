@@ -1,0 +1,306 @@
+// Gradient GEMMs of the backward pass, on tcgen05 tensor cores:
+//   dW_m[v, :] = sum_t G_m[t, v] H_m[t, :]     A = G_m viewed M-major (M = v), B = H_m N-major
+//   dH_m[t, :] = sum_v G_m[t, v] W_m[v, :]     A = G_m K-major (K = v),       B = W_m N-major
+// where G_m = dL/dz_m is the bf16 (fp32 for fp32 inputs) gradient tile written
+// by the backward head kernel.  For bf16 both products read the row-major
+// tensors in place: the shared-memory descriptors say which dimension is
+// contiguous, so no transposed copy of G, H or W is made.  The tf32 MMA is
+// only used with K-major operands here, so fp32 inputs go through transposed
+// copies (G^T, H^T, W^T) instead.
+//
+// Persistent CTAs walk a list of 128x256 output tiles over up to four
+// problems (one per sub-model): warp 4 streams A/B k-blocks with TMA, warp 5
+// issues the MMAs into one of two TMEM accumulators, warps 0-3 drain the other
+// accumulator to global memory (optionally adding to what is there).
+#include "mls_device.cuh"
+#include "mls_kernels.h"
+
+namespace mls {
+namespace {
+
+struct GemmSmem {
+  static constexpr uint32_t kA = 0;
+  static constexpr uint32_t kB = kGemmStages * kGemmABytes;
+  static constexpr uint32_t kBar = kB + kGemmStages * kGemmBBytes;
+  static __device__ __forceinline__ uint32_t full(uint32_t b, int s) { return b + kBar + 8u * s; }
+  static __device__ __forceinline__ uint32_t empty(uint32_t b, int s) {
+    return b + kBar + 8u * (kGemmStages + s);
+  }
+  static __device__ __forceinline__ uint32_t accf(uint32_t b, uint32_t a) {
+    return b + kBar + 8u * (2 * kGemmStages + a);
+  }
+  static __device__ __forceinline__ uint32_t acce(uint32_t b, uint32_t a) {
+    return b + kBar + 8u * (2 * kGemmStages + 2 + a);
+  }
+  static __device__ __forceinline__ uint32_t drain(uint32_t b) {
+    return b + kBar + 8u * (2 * kGemmStages + 4);
+  }
+  static constexpr uint32_t kTmemSlot = kBar + 8u * (2 * kGemmStages + 5);
+  static constexpr uint32_t kAbort = kTmemSlot + 4;
+  static constexpr uint32_t kEnd = kAbort + 4;
+};
+static_assert(GemmSmem::kEnd + 1024 <= kGemmSmem, "gemm shared memory map overflows");
+
+constexpr uint32_t kTmemCols = 512;
+constexpr uint64_t kDrainNs = 100000000ull;
+
+struct TileCoord {
+  int prob, tm, tn;
+};
+
+__device__ __forceinline__ TileCoord decode_tile(const GemmParams& p, int t) {
+  int i = 0;
+  while (i + 1 < p.nprob && t >= p.prob[i + 1].tile_begin) ++i;
+  const int local = t - p.prob[i].tile_begin;
+  return {i, local / p.prob[i].tiles_n, local % p.prob[i].tiles_n};
+}
+
+template <bool kTF32, bool kAMN, bool kBMN>
+__device__ __forceinline__ void gemm_producer(const GemmParams& p, uint32_t base,
+                                              volatile int* abort_flag) {
+  constexpr int KE = kTF32 ? 32 : 64;           // elements per 128-byte row
+  constexpr uint32_t kBox = KE * 128;           // bytes of one MN-major box {KE, KE}
+  int stage = 0;
+  uint32_t phase = 0, filled = 0, lastpar = 0;
+  bool ok = true;
+  for (int t = blockIdx.x; ok && t < p.total_tiles; t += gridDim.x) {
+    const TileCoord tc = decode_tile(p, t);
+    const GemmProblem& pr = p.prob[tc.prob];
+    const CUtensorMap* ma = &p.mapA[pr.a_map];
+    const CUtensorMap* mb = &p.mapB[pr.b_map];
+    const int nkb = (pr.K + KE - 1) / KE;
+    const int m0 = pr.a_m0 + tc.tm * kGemmBM;
+    const int n0 = pr.b_n0 + tc.tn * kGemmBN;
+    for (int kb = 0; kb < nkb; ++kb) {
+      if (!mbar_wait(GemmSmem::empty(base, stage), phase ^ 1u, abort_flag, p.status)) {
+        ok = false;
+        break;
+      }
+      const uint32_t fb = GemmSmem::full(base, stage);
+      mbar_arrive_expect_tx(fb, kGemmABytes + kGemmBBytes);
+      const uint32_t sa = base + GemmSmem::kA + stage * kGemmABytes;
+      const uint32_t sb = base + GemmSmem::kB + stage * kGemmBBytes;
+      const int ka = pr.a_k0 + kb * KE, kbb = pr.b_k0 + kb * KE;
+      if (kAMN) {
+#pragma unroll
+        for (int j = 0; j < kGemmBM / KE; ++j) tma_load_2d(sa + j * kBox, ma, fb, m0 + j * KE, ka);
+      } else {
+        tma_load_2d(sa, ma, fb, ka, m0);
+      }
+      if (kBMN) {
+#pragma unroll
+        for (int j = 0; j < kGemmBN / KE; ++j) tma_load_2d(sb + j * kBox, mb, fb, n0 + j * KE, kbb);
+      } else {
+        tma_load_2d(sb, mb, fb, kbb, n0);
+      }
+      filled |= 1u << stage;
+      lastpar = (lastpar & ~(1u << stage)) | (phase << stage);
+      if (++stage == kGemmStages) {
+        stage = 0;
+        phase ^= 1u;
+      }
+    }
+  }
+  if (!ok) {
+    for (int s = 0; s < kGemmStages; ++s)
+      if ((filled >> s) & 1u) mbar_wait_drain(GemmSmem::full(base, s), (lastpar >> s) & 1u, kDrainNs);
+  }
+}
+
+template <bool kTF32, bool kAMN, bool kBMN>
+__device__ __forceinline__ void gemm_mma(const GemmParams& p, uint32_t base, uint32_t tmem,
+                                         volatile int* abort_flag) {
+  constexpr int KE = kTF32 ? 32 : 64;
+  constexpr uint32_t kIdesc = make_idesc(kGemmBM, kGemmBN, kTF32, kAMN, kBMN);
+  constexpr uint32_t kBox = KE * 128;
+  // Advance per MMA (32 bytes of K): along a 128-byte row for K-major
+  // operands, by (32 / element size) rows of 128 bytes for MN-major ones.
+  constexpr uint32_t kStepK = 32u >> 4;
+  constexpr uint32_t kStepMN = ((32u / (kTF32 ? 4u : 2u)) * 128u) >> 4;
+  int stage = 0;
+  uint32_t phase = 0, acc = 0, acc_par = 0;
+  bool ok = true;
+  for (int t = blockIdx.x; ok && t < p.total_tiles; t += gridDim.x) {
+    const TileCoord tc = decode_tile(p, t);
+    const int nkb = (p.prob[tc.prob].K + KE - 1) / KE;
+    if (!mbar_wait(GemmSmem::acce(base, acc), acc_par ^ 1u, abort_flag, p.status)) {
+      ok = false;
+      break;
+    }
+    tc_fence_after();
+    const uint32_t d = tmem + acc * kGemmBN;
+    for (int kb = 0; kb < nkb; ++kb) {
+      if (!mbar_wait(GemmSmem::full(base, stage), phase, abort_flag, p.status)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint64_t ad = make_sdesc(base + GemmSmem::kA + stage * kGemmABytes, kAMN ? kBox : 16u);
+      const uint64_t bd = make_sdesc(base + GemmSmem::kB + stage * kGemmBBytes, kBMN ? kBox : 16u);
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk)
+        mma_issue<kTF32>(d, ad + kk * (kAMN ? kStepMN : kStepK), bd + kk * (kBMN ? kStepMN : kStepK),
+                         kIdesc, (kb | kk) != 0);
+      mma_commit(GemmSmem::empty(base, stage));
+      if (++stage == kGemmStages) {
+        stage = 0;
+        phase ^= 1u;
+      }
+    }
+    if (!ok) break;
+    mma_commit(GemmSmem::accf(base, acc));
+    acc ^= 1u;
+    if (acc == 0) acc_par ^= 1u;
+  }
+  mma_commit(GemmSmem::drain(base));
+  mbar_wait_drain(GemmSmem::drain(base), 0, kDrainNs);
+}
+
+__device__ __forceinline__ void gemm_epilogue(const GemmParams& p, uint32_t base, uint32_t tmem,
+                                              int warp, int lane, volatile int* abort_flag) {
+  uint32_t acc = 0, acc_par = 0;
+  const uint32_t tl = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+  for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x) {
+    const TileCoord tc = decode_tile(p, t);
+    const GemmProblem& pr = p.prob[tc.prob];
+    const bool ok = mbar_wait(GemmSmem::accf(base, acc), acc_par, abort_flag, p.status);
+    if (!__all_sync(0xffffffffu, ok)) return;
+    tc_fence_after();
+    const long long row = static_cast<long long>(tc.tm) * kGemmBM + warp * 32 + lane;
+    const bool row_ok = row < pr.Mrows;
+    float* crow = pr.C + (row_ok ? row : 0) * pr.ldc;
+    float v[32];
+#pragma unroll 1
+    for (int c = 0; c < kGemmBN / 32; ++c) {
+      tmem_ld32(tl + acc * kGemmBN + c * 32, v);
+      const int col = tc.tn * kGemmBN + c * 32;
+      if (!row_ok || col >= pr.Ncols) continue;
+      float* dst = crow + col;
+      if (col + 32 <= pr.Ncols) {
+        float4* d4 = reinterpret_cast<float4*>(dst);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          float4 o = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+          if (pr.accumulate) {
+            const float4 c4 = d4[i];
+            o.x += c4.x;
+            o.y += c4.y;
+            o.z += c4.z;
+            o.w += c4.w;
+          }
+          d4[i] = o;
+        }
+      } else {
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+          if (col + i < pr.Ncols) dst[i] = pr.accumulate ? dst[i] + v[i] : v[i];
+      }
+    }
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(GemmSmem::acce(base, acc));
+    acc ^= 1u;
+    if (acc == 0) acc_par ^= 1u;
+  }
+}
+
+template <bool kTF32, bool kAMN, bool kBMN>
+__global__ void __launch_bounds__(kGemmThreads, 1) gemm_kernel(const __grid_constant__ GemmParams p) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* gbase = smem_raw + (base - raw);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(gbase + GemmSmem::kAbort);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + GemmSmem::kTmemSlot);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    *abort_flag = 0;
+    for (int s = 0; s < kGemmStages; ++s) {
+      mbar_init(GemmSmem::full(base, s), 1);
+      mbar_init(GemmSmem::empty(base, s), 1);
+    }
+    for (uint32_t a = 0; a < 2; ++a) {
+      mbar_init(GemmSmem::accf(base, a), 1);
+      mbar_init(GemmSmem::acce(base, a), kGemmEpiWarps);
+    }
+    mbar_init(GemmSmem::drain(base), 1);
+    fence_barrier_init();
+  }
+  if (warp == kGemmEpiWarps + 1) {
+    tmem_alloc(base + GemmSmem::kTmemSlot, kTmemCols);
+    tmem_relinquish();
+  }
+  if (warp == kGemmEpiWarps && lane == 0) {
+    for (int i = 0; i < p.nprob; ++i) {
+      tma_prefetch_desc(&p.mapA[p.prob[i].a_map]);
+      tma_prefetch_desc(&p.mapB[p.prob[i].b_map]);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == kGemmEpiWarps) {
+    if (lane == 0) gemm_producer<kTF32, kAMN, kBMN>(p, base, abort_flag);
+  } else if (warp == kGemmEpiWarps + 1) {
+    if (lane == 0) gemm_mma<kTF32, kAMN, kBMN>(p, base, tmem, abort_flag);
+    __syncwarp();
+  } else {
+    gemm_epilogue(p, base, tmem, warp, lane, abort_flag);
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == kGemmEpiWarps + 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+template <bool kAMN, bool kBMN>
+cudaError_t launch(const GemmParams& p, bool tf32, int grid, cudaStream_t s) {
+  if (p.total_tiles <= 0 || grid <= 0) return cudaSuccess;
+  if (tf32)
+    gemm_kernel<true, kAMN, kBMN><<<grid, kGemmThreads, kGemmSmem, s>>>(p);
+  else
+    gemm_kernel<false, kAMN, kBMN><<<grid, kGemmThreads, kGemmSmem, s>>>(p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_gemm_dw(const GemmParams& p, bool tf32, int grid, cudaStream_t s) {
+  return launch<true, true>(p, tf32, grid, s);
+}
+cudaError_t launch_gemm_dh(const GemmParams& p, bool tf32, int grid, cudaStream_t s) {
+  return launch<false, true>(p, tf32, grid, s);
+}
+cudaError_t launch_gemm_kk(const GemmParams& p, bool tf32, int grid, cudaStream_t s) {
+  return launch<false, false>(p, tf32, grid, s);
+}
+
+cudaError_t setup_gemm_kernels() {
+  cudaError_t e;
+#define MLS_SET(TF, AM, BM)                                                                     \
+  e = cudaFuncSetAttribute(gemm_kernel<TF, AM, BM>, cudaFuncAttributeMaxDynamicSharedMemorySize, \
+                           kGemmSmem);                                                          \
+  if (e != cudaSuccess) return e;                                                               \
+  {                                                                                             \
+    cudaFuncAttributes fa;                                                                      \
+    e = cudaFuncGetAttributes(&fa, gemm_kernel<TF, AM, BM>);                                    \
+    if (e != cudaSuccess) return e;                                                             \
+    if (fa.maxThreadsPerBlock < kGemmThreads) return cudaErrorLaunchOutOfResources;             \
+  }
+  MLS_SET(true, true, true)
+  MLS_SET(false, true, true)
+  MLS_SET(true, false, true)
+  MLS_SET(false, false, true)
+  MLS_SET(true, false, false)
+  MLS_SET(false, false, false)
+#undef MLS_SET
+  return cudaSuccess;
+}
+
+}  // namespace mls

@@ -1,0 +1,643 @@
+// Fused LM-head kernels of the Matryoshka-suite output stage.
+//
+// One CTA owns kHeadBM = 128 tokens and a strided set of 256-column vocabulary
+// tiles.  For every vocabulary tile it computes the teacher's logit tile
+// z_t = H_t W_t^T first and then each student's z_m = H_m W_m^T (Sec. 2: each
+// sub-model has its own head W^m in R^{V x D_m}), on the tensor cores:
+//
+//   warp 8   TMA producer: H_m and W_m k-blocks (128 bytes of K) into a
+//            4-stage shared-memory ring, 128B-swizzled
+//   warp 9   MMA issuer: tcgen05.mma 128x256xK into one of two TMEM
+//            accumulators (2 x 256 columns), tcgen05.commit to barriers
+//   warps 0-7 epilogue: tcgen05.ld, one thread per (token, half tile); these
+//            two warpgroups take the registers the third one gives up, since
+//            each thread keeps the teacher's 128 weights of a tile in registers
+//
+// The epilogue never writes a logit to memory:
+//   forward  (Eq. 2 and Eq. 3): single-pass online logsumexp of z (tau = 1)
+//            and of z / tau, the teacher weights q~ = exp((z_t - max_t)/tau)
+//            kept in registers for the tile, the teacher-weighted sums
+//            A_m = sum_v q~_v z_m[v] (rescaled when the teacher's running max
+//            moves), the target logit and a running argmax.  Each CTA writes
+//            one partial state per (token, half, model); a merge kernel
+//            combines the partials.
+//   backward recomputes the same tiles and forms dL/dz in registers:
+//            teacher  c_t (softmax(z_t) - e_y)                (stop-grad on q)
+//            student  c_m [(1-alpha)(softmax(z_m) - e_y) + (alpha/tau)(softmax(z_m/tau) - q)]
+//            with q = softmax(z_t / tau) from the forward's statistics, and
+//            stores it (bf16, fp32 for fp32 inputs) for the dH / dW GEMMs.
+#include "mls_device.cuh"
+#include "mls_kernels.h"
+
+namespace mls {
+namespace {
+
+constexpr int kModeFwd = 0;
+constexpr int kModeBwd = 1;
+constexpr int kStud = kMaxModels - 1;
+
+// Shared-memory map, offsets from the 1024-byte-aligned base.
+struct HeadSmem {
+  static constexpr uint32_t kA = 0;
+  static constexpr uint32_t kB = kHeadStages * kHeadABytes;
+  static constexpr uint32_t kBar = kB + kHeadStages * kHeadBBytes;
+  static __device__ __forceinline__ uint32_t full(uint32_t b, int s) { return b + kBar + 8u * s; }
+  static __device__ __forceinline__ uint32_t empty(uint32_t b, int s) {
+    return b + kBar + 8u * (kHeadStages + s);
+  }
+  static __device__ __forceinline__ uint32_t accf(uint32_t b, uint32_t a) {
+    return b + kBar + 8u * (2 * kHeadStages + a);
+  }
+  static __device__ __forceinline__ uint32_t acce(uint32_t b, uint32_t a) {
+    return b + kBar + 8u * (2 * kHeadStages + 2 + a);
+  }
+  static __device__ __forceinline__ uint32_t drain(uint32_t b) {
+    return b + kBar + 8u * (2 * kHeadStages + 4);
+  }
+  static constexpr uint32_t kTmemSlot = kBar + 8u * (2 * kHeadStages + 5);
+  static constexpr uint32_t kAbort = kTmemSlot + 4;
+  static constexpr uint32_t kEnd = kAbort + 4;
+};
+static_assert(HeadSmem::kEnd + 1024 <= kHeadSmem, "head shared memory map overflows");
+
+constexpr uint32_t kTmemCols = 512;             // two 256-column fp32 accumulators
+constexpr uint64_t kDrainNs = 100000000ull;     // bound for shutdown waits
+
+// ------------------------------------------------------------------ producer
+template <bool kTF32>
+__device__ __forceinline__ void head_producer(const HeadParams& p, uint32_t base, int tt, int split,
+                                              volatile int* abort_flag) {
+  constexpr int KE = kTF32 ? 32 : 64;  // elements in 128 bytes of K
+  int stage = 0;
+  uint32_t phase = 0, filled = 0, lastpar = 0;
+  bool ok = true;
+  for (int vt = p.vt_begin + split; ok && vt < p.vt_end; vt += p.S) {
+    for (int u = 0; ok && u < p.M; ++u) {
+      const int m = p.order[u];
+      for (int kb = 0; kb < p.nk[m]; ++kb) {
+        if (!mbar_wait(HeadSmem::empty(base, stage), phase ^ 1u, abort_flag, p.status)) {
+          ok = false;
+          break;
+        }
+        const uint32_t fb = HeadSmem::full(base, stage);
+        mbar_arrive_expect_tx(fb, kHeadABytes + kHeadBBytes);
+        tma_load_2d(base + HeadSmem::kA + stage * kHeadABytes, &p.mapH[m], fb, kb * KE,
+                    tt * kHeadBM);
+        tma_load_2d(base + HeadSmem::kB + stage * kHeadBBytes, &p.mapW[m], fb, kb * KE,
+                    vt * kHeadBN);
+        filled |= 1u << stage;
+        lastpar = (lastpar & ~(1u << stage)) | (phase << stage);
+        if (++stage == kHeadStages) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+    }
+  }
+  if (!ok) {
+    // Let every load already issued land before the CTA's shared memory goes away.
+    for (int s = 0; s < kHeadStages; ++s)
+      if ((filled >> s) & 1u) mbar_wait_drain(HeadSmem::full(base, s), (lastpar >> s) & 1u, kDrainNs);
+  }
+}
+
+// ------------------------------------------------------------------ MMA issuer
+template <bool kTF32>
+__device__ __forceinline__ void head_mma(const HeadParams& p, uint32_t base, uint32_t tmem,
+                                         int split, volatile int* abort_flag) {
+  constexpr uint32_t kIdesc = make_idesc(kHeadBM, kHeadBN, kTF32, false, false);
+  int stage = 0;
+  uint32_t phase = 0, acc = 0, acc_par = 0;
+  bool ok = true;
+  for (int vt = p.vt_begin + split; ok && vt < p.vt_end; vt += p.S) {
+    for (int u = 0; ok && u < p.M; ++u) {
+      const int m = p.order[u];
+      if (!mbar_wait(HeadSmem::acce(base, acc), acc_par ^ 1u, abort_flag, p.status)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t d = tmem + acc * kHeadBN;
+      for (int kb = 0; kb < p.nk[m]; ++kb) {
+        if (!mbar_wait(HeadSmem::full(base, stage), phase, abort_flag, p.status)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint64_t ad = make_sdesc(base + HeadSmem::kA + stage * kHeadABytes, 16);
+        const uint64_t bd = make_sdesc(base + HeadSmem::kB + stage * kHeadBBytes, 16);
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk)  // 4 x 32 bytes of K per stage
+          mma_issue<kTF32>(d, ad + 2u * kk, bd + 2u * kk, kIdesc, (kb | kk) != 0);
+        mma_commit(HeadSmem::empty(base, stage));
+        if (++stage == kHeadStages) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+      if (!ok) break;
+      mma_commit(HeadSmem::accf(base, acc));
+      acc ^= 1u;
+      if (acc == 0) acc_par ^= 1u;
+    }
+  }
+  // Every MMA this thread issued has finished before TMEM is released.
+  mma_commit(HeadSmem::drain(base));
+  mbar_wait_drain(HeadSmem::drain(base), 0, kDrainNs);
+}
+
+// Waits for accumulator `acc` to be full; warp-uniform result.
+__device__ __forceinline__ bool epi_acquire(const HeadParams& p, uint32_t base, uint32_t acc,
+                                            uint32_t acc_par, volatile int* abort_flag) {
+  const bool ok = mbar_wait(HeadSmem::accf(base, acc), acc_par, abort_flag, p.status);
+  const bool all = __all_sync(0xffffffffu, ok);
+  tc_fence_after();
+  return all;
+}
+
+__device__ __forceinline__ void epi_release(uint32_t base, uint32_t& acc, uint32_t& acc_par,
+                                            int lane) {
+  tc_fence_before();
+  __syncwarp();
+  if (lane == 0) mbar_arrive(HeadSmem::acce(base, acc));
+  acc ^= 1u;
+  if (acc == 0) acc_par ^= 1u;
+}
+
+// ------------------------------------------------------------------ forward epilogue
+// Teacher tile: two passes over the thread's 128 columns.  Pass 1 finds the
+// tile maximum (and argmax); the running statistics and every student's
+// teacher-weighted sum are rescaled to the new maximum; pass 2 accumulates
+// the exponentials and leaves q~_v = exp((z_t[v] - max_t) / tau) in q[].
+// The teacher's own weighted sum is kept relative to its running maximum,
+// acc = sum_v q~_v (z_t[v] - max_t) log2(e) / tau (every term <= 0), so that the
+// entropy H(q) = log S - acc / (S log2(e)) is formed without cancellation even
+// when q is sharply peaked.
+template <bool kMasked, bool kTauOne>
+__device__ __forceinline__ void fwd_teacher(uint32_t ta, int nvalid, int yl, long long col0,
+                                            float L1, float Lt, float& m, float& s1, float& st,
+                                            float& acc, float& zy, int& am, float (&q)[128],
+                                            float (&aS)[kStud]) {
+  float v[32];
+  float tmax = -INFINITY;
+  int targ = 0;
+#pragma unroll
+  for (int c = 0; c < 4; ++c) {
+    if (kMasked && c * 32 >= nvalid) break;
+    tmem_ld32(ta + c * 32, v);
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      const bool ok = !kMasked || (c * 32 + i < nvalid);
+      if (ok && v[i] > tmax) {
+        tmax = v[i];
+        targ = c * 32 + i;
+      }
+    }
+  }
+  if (tmax > m) am = static_cast<int>(col0 + targ);
+  const float mn = fmaxf(m, tmax);
+  const float sc1 = fast_exp2((m - mn) * L1);
+  const float sct = kTauOne ? sc1 : fast_exp2((m - mn) * Lt);
+  const float st_old = kTauOne ? s1 : st;
+  if (st_old > 0.f) acc = sct * (acc + (m - mn) * Lt * st_old);
+  s1 *= sc1;
+  if (!kTauOne) st *= sct;
+#pragma unroll
+  for (int j = 0; j < kStud; ++j) aS[j] *= sct;
+  m = mn;
+  const float b1 = -mn * L1, bt = -mn * Lt;
+#pragma unroll
+  for (int c = 0; c < 4; ++c) {
+    if (kMasked && c * 32 >= nvalid) {
+#pragma unroll
+      for (int i = 0; i < 32; ++i) q[c * 32 + i] = 0.f;
+      continue;
+    }
+    tmem_ld32(ta + c * 32, v);
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      const bool ok = !kMasked || (c * 32 + i < nvalid);
+      const float z = ok ? v[i] : -INFINITY;
+      const float x1 = fmaf(z, L1, b1);
+      const float xt = kTauOne ? x1 : fmaf(z, Lt, bt);
+      const float e1 = fast_exp2(x1);
+      const float et = kTauOne ? e1 : fast_exp2(xt);
+      s1 += e1;
+      if (!kTauOne) st += et;
+      acc = fmaf(et, ok ? xt : 0.f, acc);
+      q[c * 32 + i] = et;
+    }
+    const int r = yl - c * 32;
+    if (static_cast<unsigned>(r) < 32u) {
+#pragma unroll
+      for (int i = 0; i < 32; ++i)
+        if (i == r) zy = v[i];
+    }
+  }
+}
+
+// Student tile: one pass, online per 32-column chunk.  Its teacher-weighted
+// sum uses the q~ of the same vocabulary tile, relative to the teacher's
+// current running maximum.
+template <bool kMasked, bool kTauOne>
+__device__ __forceinline__ void fwd_student(uint32_t ta, int nvalid, int yl, long long col0,
+                                            float L1, float Lt, float& m, float& s1, float& st,
+                                            float& acc, float& zy, int& am, const float (&q)[128]) {
+  float v[32];
+#pragma unroll
+  for (int c = 0; c < 4; ++c) {
+    if (kMasked && c * 32 >= nvalid) break;
+    tmem_ld32(ta + c * 32, v);
+    float cmax = -INFINITY;
+    int carg = 0;
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      const bool ok = !kMasked || (c * 32 + i < nvalid);
+      if (ok && v[i] > cmax) {
+        cmax = v[i];
+        carg = i;
+      }
+    }
+    if (cmax > m) {
+      am = static_cast<int>(col0 + c * 32 + carg);
+      s1 *= fast_exp2((m - cmax) * L1);
+      if (!kTauOne) st *= fast_exp2((m - cmax) * Lt);
+      m = cmax;
+    }
+    const float b1 = -m * L1, bt = -m * Lt;
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      const bool ok = !kMasked || (c * 32 + i < nvalid);
+      const float z = ok ? v[i] : -INFINITY;
+      s1 += fast_exp2(fmaf(z, L1, b1));
+      if (!kTauOne) st += fast_exp2(fmaf(z, Lt, bt));
+      acc = fmaf(q[c * 32 + i], ok ? v[i] : 0.f, acc);
+    }
+    const int r = yl - c * 32;
+    if (static_cast<unsigned>(r) < 32u) {
+#pragma unroll
+      for (int i = 0; i < 32; ++i)
+        if (i == r) zy = v[i];
+    }
+  }
+}
+
+template <bool kTauOne>
+__device__ __forceinline__ void fwd_epilogue(const HeadParams& p, uint32_t base, uint32_t tmem,
+                                             int tt, int split, int warp, int lane,
+                                             volatile int* abort_flag) {
+  const int quad = warp & 3, half = warp >> 2;
+  const long long row = static_cast<long long>(tt) * kHeadBM + quad * 32 + lane;
+  const bool row_ok = row < p.T;
+  const int y = row_ok ? __ldg(p.y + row) : -1;
+  const uint32_t tl = tmem + (static_cast<uint32_t>(quad * 32) << 16) + static_cast<uint32_t>(half * 128);
+  const float L1 = p.L1, Lt = p.Ltau;
+  const int nst = p.M - 1;
+
+  float mT = -INFINITY, s1T = 0.f, stT = 0.f, aT = 0.f, zT = 0.f;
+  int amT = 0;
+  float mS[kStud], s1S[kStud], stS[kStud], aS[kStud], zS[kStud];
+  int amS[kStud];
+#pragma unroll
+  for (int j = 0; j < kStud; ++j) {
+    mS[j] = -INFINITY;
+    s1S[j] = stS[j] = aS[j] = zS[j] = 0.f;
+    amS[j] = 0;
+  }
+  float q[128];
+  uint32_t acc = 0, acc_par = 0;
+
+  for (int vt = p.vt_begin + split; vt < p.vt_end; vt += p.S) {
+    const long long col0 = static_cast<long long>(vt) * kHeadBN + half * 128;
+    const int nvalid = static_cast<int>(max(0LL, min(128LL, p.V - col0)));
+    const int yl = y >= 0 ? static_cast<int>(y - col0) : -1;
+
+    if (!epi_acquire(p, base, acc, acc_par, abort_flag)) return;
+    {
+      const uint32_t ta = tl + acc * kHeadBN;
+      if (nvalid == 128)
+        fwd_teacher<false, kTauOne>(ta, 128, yl, col0, L1, Lt, mT, s1T, stT, aT, zT, amT, q, aS);
+      else if (nvalid > 0)
+        fwd_teacher<true, kTauOne>(ta, nvalid, yl, col0, L1, Lt, mT, s1T, stT, aT, zT, amT, q, aS);
+      else {
+#pragma unroll
+        for (int i = 0; i < 128; ++i) q[i] = 0.f;
+      }
+    }
+    epi_release(base, acc, acc_par, lane);
+
+#pragma unroll
+    for (int j = 0; j < kStud; ++j) {
+      if (j < nst) {
+        if (!epi_acquire(p, base, acc, acc_par, abort_flag)) return;
+        const uint32_t ta = tl + acc * kHeadBN;
+        if (nvalid == 128)
+          fwd_student<false, kTauOne>(ta, 128, yl, col0, L1, Lt, mS[j], s1S[j], stS[j], aS[j],
+                                      zS[j], amS[j], q);
+        else if (nvalid > 0)
+          fwd_student<true, kTauOne>(ta, nvalid, yl, col0, L1, Lt, mS[j], s1S[j], stS[j], aS[j],
+                                     zS[j], amS[j], q);
+        epi_release(base, acc, acc_par, lane);
+      }
+    }
+  }
+
+  if (row_ok) {
+    const long long MT = static_cast<long long>(p.M) * p.T;
+    float* P = p.part + static_cast<long long>(split * 2 + half) * kPartFields * MT;
+    const int t = p.order[0];
+    float* Pt = P + static_cast<long long>(t) * p.T + row;
+    Pt[kPartMax * MT] = mT;
+    Pt[kPartSum1 * MT] = s1T;
+    Pt[kPartSumTau * MT] = kTauOne ? s1T : stT;
+    Pt[kPartAcc * MT] = aT;
+    Pt[kPartTarget * MT] = zT;
+    Pt[kPartArgmax * MT] = __int_as_float(amT);
+#pragma unroll
+    for (int j = 0; j < kStud; ++j) {
+      if (j < nst) {
+        float* Pm = P + static_cast<long long>(p.order[j + 1]) * p.T + row;
+        Pm[kPartMax * MT] = mS[j];
+        Pm[kPartSum1 * MT] = s1S[j];
+        Pm[kPartSumTau * MT] = kTauOne ? s1S[j] : stS[j];
+        Pm[kPartAcc * MT] = aS[j];
+        Pm[kPartTarget * MT] = zS[j];
+        Pm[kPartArgmax * MT] = __int_as_float(amS[j]);
+      }
+    }
+  }
+}
+
+// ------------------------------------------------------------------ backward epilogue
+template <bool kTF32>
+__device__ __forceinline__ void store_chunk(void* dst, const float (&g)[32]) {
+  if constexpr (kTF32) {
+    float4* d = reinterpret_cast<float4*>(dst);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) d[i] = make_float4(g[4 * i], g[4 * i + 1], g[4 * i + 2], g[4 * i + 3]);
+  } else {
+    uint4* d = reinterpret_cast<uint4*>(dst);
+    uint32_t w[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      __nv_bfloat162 h = __floats2bfloat162_rn(g[2 * i], g[2 * i + 1]);
+      w[i] = *reinterpret_cast<uint32_t*>(&h);
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) d[i] = make_uint4(w[4 * i], w[4 * i + 1], w[4 * i + 2], w[4 * i + 3]);
+  }
+}
+
+// Teacher: q = softmax(z_t / tau) (kept in q[] for the students) and
+// G_t = c_t (softmax(z_t) - e_y).
+template <bool kMasked, bool kTauOne, bool kTF32>
+__device__ __forceinline__ void bwd_teacher(uint32_t ta, int nvalid, int yl, float L1, float Lt,
+                                            float b1, float bt, float c, float (&q)[128],
+                                            char* gdst, bool store) {
+  constexpr int kElt = kTF32 ? 4 : 2;
+  float v[32], g[32];
+#pragma unroll
+  for (int ch = 0; ch < 4; ++ch) {
+    tmem_ld32(ta + ch * 32, v);
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      const bool ok = !kMasked || (ch * 32 + i < nvalid);
+      const float qv = fast_exp2(fmaf(v[i], Lt, bt));
+      const float pv = kTauOne ? qv : fast_exp2(fmaf(v[i], L1, b1));
+      q[ch * 32 + i] = ok ? qv : 0.f;
+      g[i] = ok ? c * pv : 0.f;
+    }
+    const int r = yl - ch * 32;
+    if (static_cast<unsigned>(r) < 32u) {
+#pragma unroll
+      for (int i = 0; i < 32; ++i)
+        if (i == r) g[i] -= c;
+    }
+    if (store) store_chunk<kTF32>(gdst + ch * 32 * kElt, g);
+  }
+}
+
+// Student: G_m = a1 (softmax(z_m) - e_y) + a2 (softmax(z_m / tau) - q),
+// a1 = c_m (1 - alpha), a2 = c_m alpha / tau.
+template <bool kMasked, bool kTauOne, bool kTF32>
+__device__ __forceinline__ void bwd_student(uint32_t ta, int nvalid, int yl, float L1, float Lt,
+                                            float b1, float bt, float a1, float a2,
+                                            const float (&q)[128], char* gdst, bool store) {
+  constexpr int kElt = kTF32 ? 4 : 2;
+  float v[32], g[32];
+  const float a12 = a1 + a2;
+#pragma unroll
+  for (int ch = 0; ch < 4; ++ch) {
+    tmem_ld32(ta + ch * 32, v);
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      const bool ok = !kMasked || (ch * 32 + i < nvalid);
+      const float pv = fast_exp2(fmaf(v[i], L1, b1));
+      float gv;
+      if (kTauOne) {
+        gv = fmaf(a12, pv, -a2 * q[ch * 32 + i]);
+      } else {
+        const float pt = fast_exp2(fmaf(v[i], Lt, bt));
+        gv = fmaf(a1, pv, a2 * (pt - q[ch * 32 + i]));
+      }
+      g[i] = ok ? gv : 0.f;
+    }
+    const int r = yl - ch * 32;
+    if (static_cast<unsigned>(r) < 32u) {
+#pragma unroll
+      for (int i = 0; i < 32; ++i)
+        if (i == r) g[i] -= a1;
+    }
+    if (store) store_chunk<kTF32>(gdst + ch * 32 * kElt, g);
+  }
+}
+
+template <bool kTauOne, bool kTF32>
+__device__ __forceinline__ void bwd_epilogue(const HeadParams& p, uint32_t base, uint32_t tmem,
+                                             int tt, int split, int warp, int lane,
+                                             volatile int* abort_flag) {
+  constexpr int kElt = kTF32 ? 4 : 2;
+  const int quad = warp & 3, half = warp >> 2;
+  const long long row = static_cast<long long>(tt) * kHeadBM + quad * 32 + lane;
+  const bool row_ok = row < p.T;
+  const int y = row_ok ? __ldg(p.y + row) : -1;
+  const bool valid = row_ok && y >= 0 && y < p.V;
+  const float inv_n = *p.inv_n;
+  const uint32_t tl = tmem + (static_cast<uint32_t>(quad * 32) << 16) + static_cast<uint32_t>(half * 128);
+  const float L1 = p.L1, Lt = p.Ltau;
+  const long long MT = static_cast<long long>(p.M) * p.T;
+  const int nst = p.M - 1;
+  const long long rr = row_ok ? row : 0;
+
+  const int t = p.order[0];
+  const float cT = valid ? p.coef[t] * inv_n : 0.f;
+  const float bT1 = -__ldg(p.stats + static_cast<long long>(t) * p.T + rr) * L1;
+  const float bTt = -__ldg(p.stats + MT + static_cast<long long>(t) * p.T + rr) * L1;
+  char* gT = static_cast<char*>(p.G) + (static_cast<long long>(t) * p.g_model_stride + rr * p.g_pitch) * kElt;
+
+  float a1[kStud], a2[kStud], b1[kStud], bt[kStud];
+  char* gS[kStud];
+#pragma unroll
+  for (int j = 0; j < kStud; ++j) {
+    const int m = j < nst ? p.order[j + 1] : t;
+    const float c = valid ? p.coef[m] * inv_n : 0.f;
+    a1[j] = c * p.one_minus_alpha;
+    a2[j] = c * p.alpha_over_tau;
+    b1[j] = -__ldg(p.stats + static_cast<long long>(m) * p.T + rr) * L1;
+    bt[j] = -__ldg(p.stats + MT + static_cast<long long>(m) * p.T + rr) * L1;
+    gS[j] = static_cast<char*>(p.G) + (static_cast<long long>(m) * p.g_model_stride + rr * p.g_pitch) * kElt;
+  }
+  float q[128];
+  uint32_t acc = 0, acc_par = 0;
+
+  for (int vt = p.vt_begin + split; vt < p.vt_end; vt += p.S) {
+    const long long col0 = static_cast<long long>(vt) * kHeadBN + half * 128;
+    const int nvalid = static_cast<int>(max(0LL, min(128LL, p.V - col0)));
+    const int yl = y >= 0 ? static_cast<int>(y - col0) : -1;
+    const long long goff = (col0 - p.g_col0) * kElt;
+
+    if (!epi_acquire(p, base, acc, acc_par, abort_flag)) return;
+    {
+      const uint32_t ta = tl + acc * kHeadBN;
+      if (nvalid == 128)
+        bwd_teacher<false, kTauOne, kTF32>(ta, 128, yl, L1, Lt, bT1, bTt, cT, q, gT + goff, row_ok);
+      else
+        bwd_teacher<true, kTauOne, kTF32>(ta, nvalid, yl, L1, Lt, bT1, bTt, cT, q, gT + goff, row_ok);
+    }
+    epi_release(base, acc, acc_par, lane);
+
+#pragma unroll
+    for (int j = 0; j < kStud; ++j) {
+      if (j < nst) {
+        if (!epi_acquire(p, base, acc, acc_par, abort_flag)) return;
+        const uint32_t ta = tl + acc * kHeadBN;
+        if (nvalid == 128)
+          bwd_student<false, kTauOne, kTF32>(ta, 128, yl, L1, Lt, b1[j], bt[j], a1[j], a2[j], q,
+                                             gS[j] + goff, row_ok);
+        else
+          bwd_student<true, kTauOne, kTF32>(ta, nvalid, yl, L1, Lt, b1[j], bt[j], a1[j], a2[j], q,
+                                            gS[j] + goff, row_ok);
+        epi_release(base, acc, acc_par, lane);
+      }
+    }
+  }
+}
+
+// ------------------------------------------------------------------ kernel
+template <int kMode, bool kTF32, bool kTauOne>
+__global__ void __launch_bounds__(kHeadThreads, 1) head_kernel(const __grid_constant__ HeadParams p) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* gbase = smem_raw + (base - raw);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(gbase + HeadSmem::kAbort);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + HeadSmem::kTmemSlot);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int tt = blockIdx.x % p.ntt;
+  const int split = blockIdx.x / p.ntt;
+
+  if (threadIdx.x == 0) {
+    *abort_flag = 0;
+    for (int s = 0; s < kHeadStages; ++s) {
+      mbar_init(HeadSmem::full(base, s), 1);
+      mbar_init(HeadSmem::empty(base, s), 1);
+    }
+    for (uint32_t a = 0; a < 2; ++a) {
+      mbar_init(HeadSmem::accf(base, a), 1);
+      mbar_init(HeadSmem::acce(base, a), kHeadEpiWarps);
+    }
+    mbar_init(HeadSmem::drain(base), 1);
+    fence_barrier_init();
+  }
+  if (warp == kHeadEpiWarps + 1) {
+    tmem_alloc(base + HeadSmem::kTmemSlot, kTmemCols);
+    tmem_relinquish();
+  }
+  if (warp == kHeadEpiWarps && lane == 0) {
+    for (int m = 0; m < p.M; ++m) {
+      tma_prefetch_desc(&p.mapH[m]);
+      tma_prefetch_desc(&p.mapW[m]);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp >= kHeadEpiWarps) {
+    regs_decrease<kHeadCtlRegs>();
+    if (warp == kHeadEpiWarps) {
+      if (lane == 0) head_producer<kTF32>(p, base, tt, split, abort_flag);
+    } else if (warp == kHeadEpiWarps + 1) {
+      if (lane == 0) head_mma<kTF32>(p, base, tmem, split, abort_flag);
+      __syncwarp();
+    }
+  } else {
+    regs_increase<kHeadEpiRegs>();
+    if constexpr (kMode == kModeFwd)
+      fwd_epilogue<kTauOne>(p, base, tmem, tt, split, warp, lane, abort_flag);
+    else
+      bwd_epilogue<kTauOne, kTF32>(p, base, tmem, tt, split, warp, lane, abort_flag);
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == kHeadEpiWarps + 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+template <int kMode>
+cudaError_t launch_head(const HeadParams& p, bool tf32, bool tau_one, cudaStream_t s) {
+  const int grid = p.ntt * p.S;
+  if (grid <= 0) return cudaSuccess;
+  const dim3 g(grid), b(kHeadThreads);
+  if (tf32) {
+    if (tau_one) head_kernel<kMode, true, true><<<g, b, kHeadSmem, s>>>(p);
+    else head_kernel<kMode, true, false><<<g, b, kHeadSmem, s>>>(p);
+  } else {
+    if (tau_one) head_kernel<kMode, false, true><<<g, b, kHeadSmem, s>>>(p);
+    else head_kernel<kMode, false, false><<<g, b, kHeadSmem, s>>>(p);
+  }
+  return cudaGetLastError();
+}
+
+template <int kMode>
+cudaError_t setup_mode() {
+  cudaError_t e;
+#define MLS_SET(TF, TO)                                                                      \
+  e = cudaFuncSetAttribute(head_kernel<kMode, TF, TO>, cudaFuncAttributeMaxDynamicSharedMemorySize, \
+                           kHeadSmem);                                                       \
+  if (e != cudaSuccess) return e;                                                            \
+  {                                                                                          \
+    cudaFuncAttributes fa;                                                                   \
+    e = cudaFuncGetAttributes(&fa, head_kernel<kMode, TF, TO>);                              \
+    if (e != cudaSuccess) return e;                                                          \
+    if (fa.maxThreadsPerBlock < kHeadThreads || fa.numRegs != kHeadLaunchRegs)               \
+      return cudaErrorLaunchOutOfResources;                                                  \
+  }
+  MLS_SET(true, true)
+  MLS_SET(true, false)
+  MLS_SET(false, true)
+  MLS_SET(false, false)
+#undef MLS_SET
+  return cudaSuccess;
+}
+
+}  // namespace
+
+cudaError_t launch_head_fwd(const HeadParams& p, bool tf32, bool tau_one, cudaStream_t s) {
+  return launch_head<kModeFwd>(p, tf32, tau_one, s);
+}
+cudaError_t launch_head_bwd(const HeadParams& p, bool tf32, bool tau_one, cudaStream_t s) {
+  return launch_head<kModeBwd>(p, tf32, tau_one, s);
+}
+cudaError_t setup_head_kernels() {
+  cudaError_t e = setup_mode<kModeFwd>();
+  if (e != cudaSuccess) return e;
+  return setup_mode<kModeBwd>();
+}
+
+}  // namespace mls

@@ -1,0 +1,140 @@
+// Internal interface between the host API (mls_api.cu) and the kernel
+// translation units.  Parameter blocks are passed by value as __grid_constant__
+// kernel arguments, so the tensor maps live in the kernel parameter space.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace mls {
+
+constexpr int kMaxModels = 4;
+
+// ------------------------------------------------------------------ head kernels
+// One CTA owns a tile of kHeadBM tokens and walks vocabulary tiles of kHeadBN
+// columns; for each vocabulary tile it computes the teacher's logit tile first
+// and then every student's, all into TMEM (double-buffered).
+constexpr int kHeadBM = 128;
+constexpr int kHeadBN = 256;
+constexpr int kHeadStages = 4;
+constexpr int kHeadEpiWarps = 8;                       // warpgroups 0 and 1
+constexpr int kHeadThreads = (kHeadEpiWarps + 4) * 32;  // + warpgroup 2: TMA, MMA, 2 idle
+// Registers: launched at 168 per thread (384 x 168 = 64512), then the control
+// warpgroup gives up registers and the epilogue warpgroups take them:
+// 2 x 128 x 232 + 128 x 40 = 64512.  Per SM sub-partition: 232 + 232 + 40 warps' worth.
+constexpr int kHeadLaunchRegs = 168;
+constexpr int kHeadEpiRegs = 232;
+constexpr int kHeadCtlRegs = 40;
+static_assert(2 * 128 * kHeadEpiRegs + 128 * kHeadCtlRegs == kHeadThreads * kHeadLaunchRegs,
+              "register reallocation must add up to the launch allocation");
+constexpr uint32_t kHeadABytes = kHeadBM * 128;
+constexpr uint32_t kHeadBBytes = kHeadBN * 128;
+constexpr uint32_t kHeadSmem = kHeadStages * (kHeadABytes + kHeadBBytes) + 1024 + 1024;
+
+// Partial row state written by the forward head kernel, per (partial, field, model, token).
+// kPartAcc holds, for a student, sum_v q~_v z_m[v] with q~ relative to the
+// teacher's running maximum of the same partial; for the teacher,
+// sum_v q~_v (z_t[v] - max_t) log2(e) / tau.
+enum PartField { kPartMax = 0, kPartSum1, kPartSumTau, kPartAcc, kPartTarget, kPartArgmax, kPartFields };
+
+struct HeadParams {
+  CUtensorMap mapH[kMaxModels];  // H_m [T, d_m], box {128 B of K, kHeadBM rows}
+  CUtensorMap mapW[kMaxModels];  // W_m [V, d_m], box {128 B of K, kHeadBN rows}
+  int M;
+  int order[kMaxModels];         // order[0] = teacher, then the students
+  int nk[kMaxModels];            // k-blocks (128 bytes of K each) of model m
+  int ntt;                       // token tiles
+  int vt_begin, vt_end;          // vocabulary tiles handled by this launch
+  int S;                         // CTAs per token tile (vocabulary splits)
+  long long T, V;
+  float L1;                      // log2(e)
+  float Ltau;                    // log2(e) / tau
+  const int* y;                  // targets [T]
+  int* status;
+  // forward
+  float* part;                   // [2*S][kPartFields][M][T]
+  // backward
+  const float* stats;            // [2][M][T]: logsumexp(z), logsumexp(z/tau)
+  const float* inv_n;            // device scalar 1/N (0 if N == 0)
+  float coef[kMaxModels];        // grad_scale * w_m
+  float one_minus_alpha;         // (1 - alpha)
+  float alpha_over_tau;          // alpha / tau
+  void* G;                       // [M][T][g_pitch] bf16 (fp32 for fp32 inputs)
+  long long g_model_stride;      // elements
+  long long g_pitch;             // elements per token row
+  long long g_col0;              // vocabulary column of the group's first column
+};
+
+// ------------------------------------------------------------------ GEMM kernels
+constexpr int kGemmBM = 128;
+constexpr int kGemmBN = 256;
+constexpr int kGemmStages = 4;
+constexpr int kGemmEpiWarps = 4;
+constexpr int kGemmThreads = (kGemmEpiWarps + 2) * 32;
+constexpr uint32_t kGemmABytes = kGemmBM * 128;
+constexpr uint32_t kGemmBBytes = kGemmBN * 128;
+// 32 KB of slack past the last stage keeps every operand read of an MN-major
+// descriptor inside the CTA's allocation.
+constexpr uint32_t kGemmSmem = kGemmStages * (kGemmABytes + kGemmBBytes) + 1024 + 1024 + 32768;
+
+struct GemmProblem {
+  int Mrows, Ncols, K;           // C is Mrows x Ncols, reduction length K
+  int a_map, b_map;              // index into mapA / mapB
+  int a_m0, a_k0, b_n0, b_k0;    // coordinate offsets into the tensors
+  float* C;                      // row-major fp32, leading dimension ldc
+  long long ldc;
+  int accumulate;                // C += A*B if 1, C = A*B if 0
+  int tiles_n;                   // ceil(Ncols / kGemmBN)
+  int tile_begin;                // first linear tile of this problem
+};
+
+struct GemmParams {
+  CUtensorMap mapA[kMaxModels];
+  CUtensorMap mapB[kMaxModels];
+  int nprob;
+  GemmProblem prob[kMaxModels];
+  int total_tiles;
+  int* status;
+};
+
+// ------------------------------------------------------------------ reductions
+struct MergeParams {
+  const float* part;             // [nparts][kPartFields][M][T]
+  int nparts;
+  int M, teacher;
+  long long T, V;
+  float L1, Ltau, tau, alpha;
+  float w[kMaxModels];
+  const int* y;
+  float* tok_loss;               // [M][T]
+  float* tok_diag;               // [3][M][T] or nullptr
+  int* argmax;                   // [M][T] or nullptr
+  float* stats;                  // [2][M][T]
+  double* block_sum;             // [gridDim.x]: sum over the block's tokens of sum_m w_m L_m
+  long long* block_cnt;          // [gridDim.x]: valid tokens in the block
+  int* status;
+};
+
+constexpr int kMergeThreads = 128;
+
+// Launchers (return the cudaError_t of the launch).
+cudaError_t launch_head_fwd(const HeadParams& p, bool tf32, bool tau_one, cudaStream_t s);
+cudaError_t launch_head_bwd(const HeadParams& p, bool tf32, bool tau_one, cudaStream_t s);
+cudaError_t launch_gemm_dw(const GemmParams& p, bool tf32, int grid, cudaStream_t s);
+cudaError_t launch_gemm_dh(const GemmParams& p, bool tf32, int grid, cudaStream_t s);
+// Both operands K-major (tf32 path: fp32 inputs with transposed copies).
+cudaError_t launch_gemm_kk(const GemmParams& p, bool tf32, int grid, cudaStream_t s);
+cudaError_t launch_transpose(const float* in, long long rows, long long cols, long long ld_in,
+                             float* out, long long ld_out, cudaStream_t s);
+cudaError_t launch_merge(const MergeParams& p, int blocks, cudaStream_t s);
+cudaError_t launch_final(const double* block_sum, const long long* block_cnt, int nblocks,
+                         float* loss, cudaStream_t s);
+cudaError_t launch_count(const int* y, long long T, long long V, float* inv_n, int* status,
+                         cudaStream_t s);
+
+// One-time per-device kernel attribute setup (dynamic shared memory limits).
+cudaError_t setup_head_kernels();
+cudaError_t setup_gemm_kernels();
+
+}  // namespace mls
