@@ -126,6 +126,36 @@ int mls_get_status(mls_stream_t stream);
 const char* mls_strerror(int code);
 
 /*
+ * Forward without a caller-provided workspace (the paper has no counterpart;
+ * this is an interface convenience).  Same operation, arguments and outputs as
+ * mls_head_loss_fwd minus ws/ws_bytes: the scratch it needs (per-CTA partial
+ * row states and per-block sums) lives in a fixed device array of
+ * MLS_NOALLOC_SCRATCH_BYTES that the library reserves on every GPU that loads
+ * it, for the life of the process.  It calls no cudaMalloc or cudaFree and no
+ * allocating library routine.  It is meant for callers that cannot allocate
+ * device memory at the point of the call: a host program or plugin that has no
+ * allocator to hand out a workspace, or a steady-state loop that must not call
+ * cudaMalloc, which can synchronise the device and carve memory out of a pool
+ * another allocator already owns.
+ *   - A problem whose forward needs more than MLS_NOALLOC_SCRATCH_BYTES of
+ *     scratch is rejected with MLS_ERR_WORKSPACE before anything is launched.
+ *     (The benchmark workloads need at most about 31 MiB; mls_workspace_size
+ *     reports the larger forward+backward requirement, not this one.)
+ *   - The first call on a device looks up the array's device address on that
+ *     device (cudaGetSymbolAddress); make that first call before any stream
+ *     capture.
+ *   - All calls on a device share the one array and it keeps the previous
+ *     call's contents.  Nothing in it needs to start at zero: each call writes
+ *     every word it later reads.  Calls whose kernels overlap on the GPU (other
+ *     streams, other host threads) race on the array and corrupt each other's
+ *     results; serialise them.
+ */
+#define MLS_NOALLOC_SCRATCH_BYTES (32u << 20)
+int mls_head_loss_fwd_noalloc(const mls_problem* p, const void* const* H, const void* const* W,
+                              const int32_t* targets, float* loss, float* tok_loss,
+                              float* tok_diag, int32_t* argmax, float* stats, mls_stream_t stream);
+
+/*
  * Kernel timing (a tracing aid; not part of the paper's method).  While
  * enabled, every kernel the library launches is bracketed by two CUDA events
  * recorded on the launch stream.  mls_profile_read synchronises on the last

@@ -75,6 +75,8 @@ def lib():
         L.mls_get_status.restype = ctypes.c_int
         L.mls_strerror.argtypes = [ctypes.c_int]
         L.mls_strerror.restype = ctypes.c_char_p
+        L.mls_head_loss_fwd_noalloc.argtypes = [P, vpp, vpp, vp, vp, vp, vp, vp, vp, vp]
+        L.mls_head_loss_fwd_noalloc.restype = ctypes.c_int
         L.mls_profile_enable.argtypes = [ctypes.c_int]
         L.mls_profile_enable.restype = ctypes.c_int
         L.mls_profile_read.argtypes = [ctypes.POINTER(mls_kernel_time), ctypes.c_int]
@@ -142,6 +144,19 @@ def mls_head_loss_bwd(prob: Problem, H, W, targets, stats, grad_scale: float, dH
                                  float(grad_scale), _ptrs(dH), _ptrs(dW), _ptr(ws), ws_bytes,
                                  _stream(stream))
     _check(rc, "mls_head_loss_bwd")
+
+
+def mls_head_loss_fwd_noalloc(prob: Problem, H, W, targets, loss, tok_loss, tok_diag, argmax,
+                              stats, stream=None) -> None:
+    """Forward with the library's built-in scratch instead of a workspace, for
+    callers that cannot allocate device memory when they call; allocates nothing."""
+    rc = lib().mls_head_loss_fwd_noalloc(prob.ref(), _ptrs(H), _ptrs(W), _ptr(targets), _ptr(loss),
+                                         _ptr(tok_loss), _ptr(tok_diag), _ptr(argmax), _ptr(stats),
+                                         _stream(stream))
+    _check(rc, "mls_head_loss_fwd_noalloc")
+
+
+MLS_NOALLOC_SCRATCH_BYTES = 32 << 20
 
 
 def mls_get_status(stream=None) -> int:

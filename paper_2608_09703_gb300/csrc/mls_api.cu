@@ -560,3 +560,94 @@ extern "C" int mls_profile_read(mls_kernel_time* out, int n) {
   for (int i = 0; i < k && i < n; ++i) out[i] = {names[i], launches[i], ms[i]};
   return k;
 }
+
+// ------------------------------------------------------------------ forward without allocation
+// Scratch for mls_head_loss_fwd_noalloc: a fixed device array that every GPU
+// loading this library holds until the process exits.  Host code must not use
+// the symbol's name as a device address; the address is looked up once per
+// device with cudaGetSymbolAddress (that device current) and passed to the kernels.
+static __device__ __align__(256) unsigned char g_noalloc_scratch[MLS_NOALLOC_SCRATCH_BYTES];
+
+namespace mls {
+namespace {
+void* g_noalloc_ptr[kMaxDevices] = {};
+
+int noalloc_scratch(void** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return fail(MLS_ERR_CUDA, "cudaGetDevice", e);
+  if (dev < 0 || dev >= kMaxDevices) return MLS_ERR_DEVICE;
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (!g_noalloc_ptr[dev]) {
+    void* ptr = nullptr;
+    e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);
+    if (e != cudaSuccess || !ptr) return fail(MLS_ERR_CUDA, "cudaGetSymbolAddress(scratch)", e);
+    g_noalloc_ptr[dev] = ptr;
+  }
+  *out = g_noalloc_ptr[dev];
+  return MLS_OK;
+}
+}  // namespace
+}  // namespace mls
+
+extern "C" int mls_head_loss_fwd_noalloc(const mls_problem* p, const void* const* H,
+                                         const void* const* W, const int32_t* targets, float* loss,
+                                         float* tok_loss, float* tok_diag, int32_t* argmax,
+                                         float* stats, mls_stream_t stream) {
+  int rc = validate(p);
+  if (rc) return rc;
+  if (!H || !W || !loss || (p->T > 0 && (!targets || !tok_loss || !stats))) return MLS_ERR_ARG;
+  for (int m = 0; m < p->M; ++m) {
+    if (!H[m] || !W[m]) return MLS_ERR_ARG;
+    if (!aligned16(H[m]) || !aligned16(W[m])) return MLS_ERR_ALIGN;
+  }
+  DeviceState* dev = nullptr;
+  if ((rc = device_state(&dev))) return rc;
+  const Plan pl = make_plan(p, dev->sms);
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (p->T == 0) return launch_ok(cudaMemsetAsync(loss, 0, sizeof(float), s));
+  if (pl.fwd_bytes > static_cast<size_t>(MLS_NOALLOC_SCRATCH_BYTES))
+    return fail(MLS_ERR_WORKSPACE, "forward needs more scratch than MLS_NOALLOC_SCRATCH_BYTES");
+  void* scratch = nullptr;
+  if ((rc = noalloc_scratch(&scratch))) return rc;
+  char* wsb = static_cast<char*>(scratch);
+  // Every word of scratch that the kernels read is written earlier in the same
+  // call (partials of valid rows, one sum per merge block), so nothing is cleared.
+
+  HeadParams hp;
+  std::memset(&hp, 0, sizeof hp);
+  fill_head_common(hp, p, pl, targets, dev->status);
+  if ((rc = encode_head_maps(hp, p, pl, H, W))) return rc;
+  hp.vt_begin = 0;
+  hp.vt_end = pl.nvt;
+  hp.S = pl.S;
+  hp.part = reinterpret_cast<float*>(wsb + pl.off_part);
+  if ((rc = timed("head_fwd", s, [&] { return launch_head_fwd(hp, pl.elt == 4, p->tau == 1.0f, s); })))
+    return rc;
+
+  MergeParams mp;
+  std::memset(&mp, 0, sizeof mp);
+  mp.part = hp.part;
+  mp.nparts = pl.nparts;
+  mp.M = p->M;
+  mp.teacher = p->teacher;
+  mp.T = p->T;
+  mp.V = p->V;
+  mp.L1 = hp.L1;
+  mp.Ltau = hp.Ltau;
+  mp.tau = p->tau;
+  mp.alpha = p->alpha;
+  for (int m = 0; m < p->M; ++m) mp.w[m] = p->w ? p->w[m] : 1.0f;
+  mp.y = targets;
+  mp.tok_loss = tok_loss;
+  mp.tok_diag = tok_diag;
+  mp.argmax = argmax;
+  mp.stats = stats;
+  mp.block_sum = reinterpret_cast<double*>(wsb + pl.off_bsum);
+  mp.block_cnt = reinterpret_cast<long long*>(wsb + pl.off_bcnt);
+  mp.status = dev->status;
+  if ((rc = timed("merge", s, [&] { return launch_merge(mp, pl.merge_blocks, s); }))) return rc;
+  return timed("final", s, [&] {
+    return launch_final(mp.block_sum, mp.block_cnt, pl.merge_blocks, loss, s);
+  });
+}
