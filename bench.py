@@ -207,7 +207,7 @@ def reference_arm(args, rank, world):
 
     if rank != 0:
         return
-    wl = synth.WORKLOADS[args.workload]
+    wl = workload(args)
     oracle.build()
     # size each step so that warmup + steps fit in about three minutes
     Hs, Ws, ys = oracle_sample(wl, 2)
@@ -240,6 +240,16 @@ def reference_arm(args, rank, world):
     print(json.dumps(line), flush=True)
 
 
+def workload(args):
+    from paper_2608_09703_gb300 import synth
+
+    wl = synth.WORKLOADS[args.workload]
+    if args.tokens or args.vocab:
+        T, V = args.tokens or wl.T, args.vocab or wl.V
+        wl = wl.with_(name=f"{wl.name}_T{T}_V{V}", T=T, V=V)
+    return wl
+
+
 def workload_config(wl, world):
     return {"workload": f"{wl.name}: 3-level Matryoshka suite head+CE+distillation, T={wl.T} tokens "
                         f"(4x2048), d={list(wl.d)}, V={wl.V}, bf16, tau={wl.tau}, alpha={wl.alpha}",
@@ -258,7 +268,7 @@ def gpu_arm(args, rank, world, local):
 
     dev = torch.device(f"cuda:{local}")
     torch.cuda.set_device(dev)
-    wl = synth.WORKLOADS[args.workload]
+    wl = workload(args)
     H, W, y = synth.make_inputs(wl, seed=1234 + rank, device=dev)
     op = B.HeadLoss(wl.d, wl.T, wl.V, teacher=wl.teacher_index, tau=wl.tau, alpha=wl.alpha,
                     w=wl.weights, dtype=torch.bfloat16, device=dev)
@@ -320,6 +330,38 @@ def gpu_arm(args, rank, world, local):
     gpu_launches = sum(v[0] for v in kern.values())
 
     # ---- end to end through the C ABI with host buffers (pinned), copies timed
+    e2e = None
+    if not args.no_e2e:
+        e2e = e2e_run(args, op, H, W, y, world, stream, wl)
+    if rank != 0:
+        return
+    cpu = None
+    if world == 1 and not args.no_cpu_baseline:
+        rate, ntok, secs = oracle_rate(wl, budget_s=15.0)
+        from oracle import oracle
+
+        cpu = {"value": rate, "unit": UNIT, "cores": oracle.threads(), "kind": "oracle",
+               "sample": f"first {ntok} of {wl.T} tokens of {wl.name} (full V and widths), "
+                         f"fp64 forward+backward, {secs:.1f} s"}
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded N(0,1) hidden states, "
+        "N(0,0.02^2) heads, uniform targets; FineWeb-Edu not available)",
+        "config": workload_config(wl, world),
+        "tensor_frac_step": step_flops / (ms_max / 1e3) / 1e12 / peak,
+        "roofline": roofline, "kernels": per_kernel, "gpu_launches": gpu_launches,
+        "clocks": clocks, "e2e": e2e, "cpu_baseline": cpu,
+    }
+    print(json.dumps(line), flush=True)
+
+
+def e2e_run(args, op, H, W, y, world, stream, wl):
+    import torch
+
+    from paper_2608_09703_gb300 import binding as B
+
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     Hh = [h.cpu().pin_memory() for h in H]
     Wh = [w.cpu().pin_memory() for w in W]
     yh = y.cpu().pin_memory()
@@ -354,28 +396,7 @@ def gpu_arm(args, rank, world, local):
     status = B.mls_get_status()
     if status:
         raise RuntimeError(f"device status: {B.mls_strerror(status)}")
-
-    if rank != 0:
-        return
-    cpu = None
-    if world == 1 and not args.no_cpu_baseline:
-        rate, ntok, secs = oracle_rate(wl, budget_s=15.0)
-        from oracle import oracle
-
-        cpu = {"value": rate, "unit": UNIT, "cores": oracle.threads(), "kind": "oracle",
-               "sample": f"first {ntok} of {wl.T} tokens of {wl.name} (full V and widths), "
-                         f"fp64 forward+backward, {secs:.1f} s"}
-    line = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded N(0,1) hidden states, "
-        "N(0,0.02^2) heads, uniform targets; FineWeb-Edu not available)",
-        "config": workload_config(wl, world),
-        "tensor_frac_step": step_flops / (ms_max / 1e3) / 1e12 / peak,
-        "roofline": roofline, "kernels": per_kernel, "gpu_launches": gpu_launches,
-        "clocks": clocks, "e2e": e2e, "cpu_baseline": cpu,
-    }
-    print(json.dumps(line), flush=True)
+    return e2e
 
 
 def main():
@@ -386,6 +407,9 @@ def main():
     ap.add_argument("--impl", default="mls", choices=["mls", "reference"])
     ap.add_argument("--workload", default=WORKLOAD)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--tokens", type=int, default=0, help="override T (profiling captures)")
+    ap.add_argument("--vocab", type=int, default=0, help="override V (profiling captures)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
