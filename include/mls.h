@@ -139,7 +139,7 @@ const char* mls_strerror(int code);
  * another allocator already owns.
  *   - A problem whose forward needs more than MLS_NOALLOC_SCRATCH_BYTES of
  *     scratch is rejected with MLS_ERR_WORKSPACE before anything is launched.
- *     (The benchmark workloads need at most about 31 MiB; mls_workspace_size
+ *     (The benchmark workloads need at most about 36 MiB; mls_workspace_size
  *     reports the larger forward+backward requirement, not this one.)
  *   - The first call on a device looks up the array's device address on that
  *     device (cudaGetSymbolAddress); make that first call before any stream
@@ -150,7 +150,7 @@ const char* mls_strerror(int code);
  *     streams, other host threads) race on the array and corrupt each other's
  *     results; serialise them.
  */
-#define MLS_NOALLOC_SCRATCH_BYTES (32u << 20)
+#define MLS_NOALLOC_SCRATCH_BYTES (64u << 20)
 int mls_head_loss_fwd_noalloc(const mls_problem* p, const void* const* H, const void* const* W,
                               const int32_t* targets, float* loss, float* tok_loss,
                               float* tok_diag, int32_t* argmax, float* stats, mls_stream_t stream);

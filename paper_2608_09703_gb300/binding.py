@@ -156,7 +156,7 @@ def mls_head_loss_fwd_noalloc(prob: Problem, H, W, targets, loss, tok_loss, tok_
     _check(rc, "mls_head_loss_fwd_noalloc")
 
 
-MLS_NOALLOC_SCRATCH_BYTES = 32 << 20
+MLS_NOALLOC_SCRATCH_BYTES = 64 << 20
 
 
 def mls_get_status(stream=None) -> int:

@@ -110,12 +110,26 @@ struct Plan {
   size_t total = 0;
 };
 
-// CTAs per token tile: about eight waves of one CTA per SM.
+// CTAs per token tile (vocabulary splits).  Each CTA of a head kernel walks
+// ceil(tiles / S) vocabulary tiles and one CTA fits per SM, so the kernel lasts
+// about waves * (tiles per CTA + a fixed per-CTA cost); S minimises that.
 int choose_splits(int ntt, long long tiles, int sms) {
-  long long s = std::llround(8.0 * sms / (ntt > 0 ? ntt : 1));
-  if (s < 1) s = 1;
-  if (s > tiles) s = tiles;
-  return static_cast<int>(s < 1 ? 1 : s);
+  if (ntt < 1) ntt = 1;
+  if (tiles < 1) return 1;
+  const double kCtaCost = 0.25;  // prologue + pipeline drain, in vocabulary tiles
+  long long best = 1;
+  double best_cost = 1e300;
+  for (long long S = 1; S <= tiles && S <= 512; ++S) {
+    const long long per = (tiles + S - 1) / S;
+    if (S > 1 && (per - 1) * S >= tiles) continue;  // same tiles per CTA with fewer CTAs
+    const long long waves = (ntt * S + sms - 1) / sms;
+    const double cost = waves * (per + kCtaCost);
+    if (cost < best_cost - 1e-9) {
+      best_cost = cost;
+      best = S;
+    }
+  }
+  return static_cast<int>(best);
 }
 
 int validate(const mls_problem* p) {
@@ -145,7 +159,7 @@ Plan make_plan(const mls_problem* p, int sms) {
   pl.ntt = static_cast<int>(ceil_div(T, kHeadBM));
   pl.nvt = static_cast<int>(ceil_div(V, kHeadBN));
   pl.S = choose_splits(pl.ntt, pl.nvt, sms);
-  pl.nparts = 2 * pl.S;
+  pl.nparts = pl.S;
   pl.merge_blocks = static_cast<int>(ceil_div(T, kMergeThreads));
   size_t o = 0;
   pl.off_part = o;
@@ -195,9 +209,11 @@ Plan make_plan(const mls_problem* p, int sms) {
 
 bool aligned16(const void* ptr) { return (reinterpret_cast<uintptr_t>(ptr) & 15u) == 0; }
 
-// 2-D row-major tensor [rows, cols] of `elt`-byte elements, 128-byte swizzle.
+// 2-D row-major tensor [rows, cols] of `elt`-byte elements (128-byte swizzle
+// unless told otherwise).
 int encode(CUtensorMap* map, const void* ptr, int elt, long long cols, long long rows,
-           long long pitch_elems, int box_cols, int box_rows) {
+           long long pitch_elems, int box_cols, int box_rows,
+           CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B) {
   const cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
   const cuuint64_t strides[1] = {static_cast<cuuint64_t>(pitch_elems) * elt};
   const cuuint32_t box[2] = {static_cast<cuuint32_t>(box_cols), static_cast<cuuint32_t>(box_rows)};
@@ -205,7 +221,7 @@ int encode(CUtensorMap* map, const void* ptr, int elt, long long cols, long long
   const CUresult r = g_encode(
       map, elt == 2 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2,
       const_cast<void*>(ptr), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-      CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+      swizzle, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
       CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) {
     char what[160];
@@ -408,6 +424,10 @@ extern "C" int mls_head_loss_bwd(const mls_problem* p, const void* const* H, con
   for (int m = 0; m < p->M; ++m) {
     const void* Gm = static_cast<const char*>(G) + static_cast<size_t>(pl.elt) * hp.g_model_stride * m;
     if (encode(&gh.mapA[m], Gm, pl.elt, pl.group, p->T, pl.group, KE, kGemmBM)) return MLS_ERR_CUDA;
+    // the backward head kernel's TMA stores of 32x32 dL/dz chunks (bf16 only)
+    if (!tf32 && encode(&hp.mapG[m], Gm, 2, pl.group, p->T, pl.group, 32, 32,
+                        CU_TENSOR_MAP_SWIZZLE_64B))
+      return MLS_ERR_CUDA;
     if (!tf32) {
       if (encode(&gw.mapA[m], Gm, pl.elt, pl.group, p->T, pl.group, KE, KE) ||
           encode(&gw.mapB[m], H[m], pl.elt, p->d[m], p->T, p->d[m], KE, KE) ||

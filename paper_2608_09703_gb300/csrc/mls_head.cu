@@ -18,9 +18,10 @@
 //            and of z / tau, the teacher weights q~ = exp((z_t - max_t)/tau)
 //            kept in registers for the tile, the teacher-weighted sums
 //            A_m = sum_v q~_v z_m[v] (rescaled when the teacher's running max
-//            moves), the target logit and a running argmax.  Each CTA writes
-//            one partial state per (token, half, model); a merge kernel
-//            combines the partials.
+//            moves), the target logit and a running argmax.  The two threads
+//            of a token (one per column half) combine their states through
+//            shared memory and each CTA writes one partial state per
+//            (token, model); a merge kernel combines the CTAs' partials.
 //   backward recomputes the same tiles and forms dL/dz in registers:
 //            teacher  c_t (softmax(z_t) - e_y)                (stop-grad on q)
 //            student  c_m [(1-alpha)(softmax(z_m) - e_y) + (alpha/tau)(softmax(z_m/tau) - q)]
@@ -40,7 +41,8 @@ constexpr int kStud = kMaxModels - 1;
 struct HeadSmem {
   static constexpr uint32_t kA = 0;
   static constexpr uint32_t kB = kHeadStages * kHeadABytes;
-  static constexpr uint32_t kBar = kB + kHeadStages * kHeadBBytes;
+  static constexpr uint32_t kStage = kB + kHeadStages * kHeadBBytes;  // dL/dz staging
+  static constexpr uint32_t kBar = kStage + kHeadStaging;
   static __device__ __forceinline__ uint32_t full(uint32_t b, int s) { return b + kBar + 8u * s; }
   static __device__ __forceinline__ uint32_t empty(uint32_t b, int s) {
     return b + kBar + 8u * (kHeadStages + s);
@@ -59,6 +61,8 @@ struct HeadSmem {
   static constexpr uint32_t kEnd = kAbort + 4;
 };
 static_assert(HeadSmem::kEnd + 1024 <= kHeadSmem, "head shared memory map overflows");
+static_assert(kPartFields * kMaxModels * kHeadBM * 4 <= kHeadStaging,
+              "forward half-merge exchange must fit in the staging area");
 
 constexpr uint32_t kTmemCols = 512;             // two 256-column fp32 accumulators
 constexpr uint64_t kDrainNs = 100000000ull;     // bound for shutdown waits
@@ -282,9 +286,27 @@ __device__ __forceinline__ void fwd_student(uint32_t ta, int nvalid, int yl, lon
   }
 }
 
+// Combines the row state of the other column half (b) into this one (a):
+// both are rescaled to the larger running maximum.
+struct RowState {
+  float m, s1, st, acc, zy;
+  int am;
+};
+
+__device__ __forceinline__ float scale_from(float from, float to, float L) {
+  return from == -INFINITY ? 0.f : fast_exp2((from - to) * L);
+}
+
+// Argmax of two halves: the larger maximum, the lower index on a tie.
+__device__ __forceinline__ int merged_argmax(float ma, int aa, float mb, int ab) {
+  if (mb > ma) return ab;
+  if (ma > mb) return aa;
+  return aa < ab ? aa : ab;
+}
+
 template <bool kTauOne>
 __device__ __forceinline__ void fwd_epilogue(const HeadParams& p, uint32_t base, uint32_t tmem,
-                                             int tt, int split, int warp, int lane,
+                                             float* xchg, int tt, int split, int warp, int lane,
                                              volatile int* abort_flag) {
   const int quad = warp & 3, half = warp >> 2;
   const long long row = static_cast<long long>(tt) * kHeadBM + quad * 32 + lane;
@@ -307,12 +329,13 @@ __device__ __forceinline__ void fwd_epilogue(const HeadParams& p, uint32_t base,
   float q[128];
   uint32_t acc = 0, acc_par = 0;
 
-  for (int vt = p.vt_begin + split; vt < p.vt_end; vt += p.S) {
+  bool aborted = false;
+  for (int vt = p.vt_begin + split; !aborted && vt < p.vt_end; vt += p.S) {
     const long long col0 = static_cast<long long>(vt) * kHeadBN + half * 128;
     const int nvalid = static_cast<int>(max(0LL, min(128LL, p.V - col0)));
     const int yl = y >= 0 ? static_cast<int>(y - col0) : -1;
 
-    if (!epi_acquire(p, base, acc, acc_par, abort_flag)) return;
+    if (!epi_acquire(p, base, acc, acc_par, abort_flag)) break;
     {
       const uint32_t ta = tl + acc * kHeadBN;
       if (nvalid == 128)
@@ -328,8 +351,11 @@ __device__ __forceinline__ void fwd_epilogue(const HeadParams& p, uint32_t base,
 
 #pragma unroll
     for (int j = 0; j < kStud; ++j) {
-      if (j < nst) {
-        if (!epi_acquire(p, base, acc, acc_par, abort_flag)) return;
+      if (j < nst && !aborted) {
+        if (!epi_acquire(p, base, acc, acc_par, abort_flag)) {
+          aborted = true;
+          break;
+        }
         const uint32_t ta = tl + acc * kHeadBN;
         if (nvalid == 128)
           fwd_student<false, kTauOne>(ta, 128, yl, col0, L1, Lt, mS[j], s1S[j], stS[j], aS[j],
@@ -341,29 +367,61 @@ __device__ __forceinline__ void fwd_epilogue(const HeadParams& p, uint32_t base,
       }
     }
   }
+  if (kTauOne) {
+    stT = s1T;
+#pragma unroll
+    for (int j = 0; j < kStud; ++j) stS[j] = s1S[j];
+  }
 
-  if (row_ok) {
-    const long long MT = static_cast<long long>(p.M) * p.T;
-    float* P = p.part + static_cast<long long>(split * 2 + half) * kPartFields * MT;
-    const int t = p.order[0];
-    float* Pt = P + static_cast<long long>(t) * p.T + row;
-    Pt[kPartMax * MT] = mT;
-    Pt[kPartSum1 * MT] = s1T;
-    Pt[kPartSumTau * MT] = kTauOne ? s1T : stT;
-    Pt[kPartAcc * MT] = aT;
-    Pt[kPartTarget * MT] = zT;
-    Pt[kPartArgmax * MT] = __int_as_float(amT);
+  // The two threads of a token (warps w and w + 4) hold the states of the two
+  // column halves; the second hands its state over through shared memory
+  // (xchg[field][slot][128 rows]) and the first writes the CTA's partial.
+  const int r = quad * 32 + lane;
+  auto X = [&](int f, int slot) -> float& { return xchg[(f * kMaxModels + slot) * kHeadBM + r]; };
+  if (half == 1) {
+    X(kPartMax, 0) = mT; X(kPartSum1, 0) = s1T; X(kPartSumTau, 0) = stT;
+    X(kPartAcc, 0) = aT; X(kPartTarget, 0) = zT; X(kPartArgmax, 0) = __int_as_float(amT);
 #pragma unroll
     for (int j = 0; j < kStud; ++j) {
-      if (j < nst) {
-        float* Pm = P + static_cast<long long>(p.order[j + 1]) * p.T + row;
-        Pm[kPartMax * MT] = mS[j];
-        Pm[kPartSum1 * MT] = s1S[j];
-        Pm[kPartSumTau * MT] = kTauOne ? s1S[j] : stS[j];
-        Pm[kPartAcc * MT] = aS[j];
-        Pm[kPartTarget * MT] = zS[j];
-        Pm[kPartArgmax * MT] = __int_as_float(amS[j]);
-      }
+      X(kPartMax, j + 1) = mS[j]; X(kPartSum1, j + 1) = s1S[j]; X(kPartSumTau, j + 1) = stS[j];
+      X(kPartAcc, j + 1) = aS[j]; X(kPartTarget, j + 1) = zS[j];
+      X(kPartArgmax, j + 1) = __int_as_float(amS[j]);
+    }
+  }
+  named_bar_sync(1, kHeadEpiWarps * 32);
+  if (half == 1 || !row_ok) return;
+
+  // teacher (its weighted sum is relative to its own maximum)
+  const float mT1 = X(kPartMax, 0), s1T1 = X(kPartSum1, 0), stT1 = X(kPartSumTau, 0);
+  const float mTm = fmaxf(mT, mT1);
+  const float fa1 = scale_from(mT, mTm, L1), fb1 = scale_from(mT1, mTm, L1);
+  const float fat = scale_from(mT, mTm, Lt), fbt = scale_from(mT1, mTm, Lt);
+  const float accT = (mT == -INFINITY ? 0.f : fat * (aT + (mT - mTm) * Lt * stT)) +
+                     (mT1 == -INFINITY ? 0.f : fbt * (X(kPartAcc, 0) + (mT1 - mTm) * Lt * stT1));
+  const long long MT = static_cast<long long>(p.M) * p.T;
+  float* P = p.part + static_cast<long long>(split) * kPartFields * MT;
+  {
+    float* Pt = P + static_cast<long long>(p.order[0]) * p.T + row;
+    Pt[kPartMax * MT] = mTm;
+    Pt[kPartSum1 * MT] = s1T * fa1 + s1T1 * fb1;
+    Pt[kPartSumTau * MT] = stT * fat + stT1 * fbt;
+    Pt[kPartAcc * MT] = accT;
+    Pt[kPartTarget * MT] = zT + X(kPartTarget, 0);
+    Pt[kPartArgmax * MT] = __int_as_float(merged_argmax(mT, amT, mT1, __float_as_int(X(kPartArgmax, 0))));
+  }
+#pragma unroll
+  for (int j = 0; j < kStud; ++j) {
+    if (j < nst) {
+      const float m1 = X(kPartMax, j + 1);
+      const float mm = fmaxf(mS[j], m1);
+      float* Pm = P + static_cast<long long>(p.order[j + 1]) * p.T + row;
+      Pm[kPartMax * MT] = mm;
+      Pm[kPartSum1 * MT] = s1S[j] * scale_from(mS[j], mm, L1) + X(kPartSum1, j + 1) * scale_from(m1, mm, L1);
+      Pm[kPartSumTau * MT] = stS[j] * scale_from(mS[j], mm, Lt) + X(kPartSumTau, j + 1) * scale_from(m1, mm, Lt);
+      // a student's teacher-weighted sum follows the teacher's maximum of its half
+      Pm[kPartAcc * MT] = aS[j] * fat + X(kPartAcc, j + 1) * fbt;
+      Pm[kPartTarget * MT] = zS[j] + X(kPartTarget, j + 1);
+      Pm[kPartArgmax * MT] = __int_as_float(merged_argmax(mS[j], amS[j], m1, __float_as_int(X(kPartArgmax, j + 1))));
     }
   }
 }
@@ -388,13 +446,54 @@ __device__ __forceinline__ void store_chunk(void* dst, const float (&g)[32]) {
   }
 }
 
+// Where one warp's 32x32 chunk of dL/dz goes.  bf16: staged in this warp's
+// shared-memory buffers (64B swizzle: 16-byte piece j of row r sits at piece
+// j ^ ((r >> 1) & 3)) and written by a TMA store; fp32: direct global stores.
+struct GOut {
+  const CUtensorMap* map;  // bf16 TMA store map of this sub-model
+  uint32_t stage;          // this warp's two staging buffers
+  uint32_t* count;         // chunks issued by this warp (buffer parity)
+  int row0;                // first token row of the warp
+  char* gdst;              // fp32: this thread's row pointer at the unit's first column
+  bool row_ok;
+};
+
+template <bool kTF32>
+__device__ __forceinline__ void put_chunk(const GOut& o, int gcol, int ch, const float (&g)[32],
+                                          int lane) {
+  if constexpr (kTF32) {
+    if (o.row_ok) store_chunk<true>(o.gdst + ch * 32 * 4, g);
+  } else {
+    const uint32_t buf = o.stage + ((*o.count) & 1u) * kHeadStageChunk;
+    if (lane == 0) bulk_wait_read<1>();  // the store that last used this buffer has read it
+    __syncwarp();
+    uint32_t w[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      __nv_bfloat162 h = __floats2bfloat162_rn(g[2 * i], g[2 * i + 1]);
+      w[i] = *reinterpret_cast<uint32_t*>(&h);
+    }
+    const uint32_t rowaddr = buf + lane * 64;
+    const uint32_t sw = (lane >> 1) & 3;
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      st_shared_v4(rowaddr + ((j ^ sw) << 4), w[4 * j], w[4 * j + 1], w[4 * j + 2], w[4 * j + 3]);
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      tma_store_2d(o.map, buf, gcol + ch * 32, o.row0);
+      bulk_commit();
+    }
+    *o.count += 1;
+  }
+}
+
 // Teacher: q = softmax(z_t / tau) (kept in q[] for the students) and
 // G_t = c_t (softmax(z_t) - e_y).
 template <bool kMasked, bool kTauOne, bool kTF32>
 __device__ __forceinline__ void bwd_teacher(uint32_t ta, int nvalid, int yl, float L1, float Lt,
                                             float b1, float bt, float c, float (&q)[128],
-                                            char* gdst, bool store) {
-  constexpr int kElt = kTF32 ? 4 : 2;
+                                            const GOut& o, int gcol, int lane) {
   float v[32], g[32];
 #pragma unroll
   for (int ch = 0; ch < 4; ++ch) {
@@ -413,7 +512,7 @@ __device__ __forceinline__ void bwd_teacher(uint32_t ta, int nvalid, int yl, flo
       for (int i = 0; i < 32; ++i)
         if (i == r) g[i] -= c;
     }
-    if (store) store_chunk<kTF32>(gdst + ch * 32 * kElt, g);
+    put_chunk<kTF32>(o, gcol, ch, g, lane);
   }
 }
 
@@ -422,8 +521,8 @@ __device__ __forceinline__ void bwd_teacher(uint32_t ta, int nvalid, int yl, flo
 template <bool kMasked, bool kTauOne, bool kTF32>
 __device__ __forceinline__ void bwd_student(uint32_t ta, int nvalid, int yl, float L1, float Lt,
                                             float b1, float bt, float a1, float a2,
-                                            const float (&q)[128], char* gdst, bool store) {
-  constexpr int kElt = kTF32 ? 4 : 2;
+                                            const float (&q)[128], const GOut& o, int gcol,
+                                            int lane) {
   float v[32], g[32];
   const float a12 = a1 + a2;
 #pragma unroll
@@ -448,7 +547,7 @@ __device__ __forceinline__ void bwd_student(uint32_t ta, int nvalid, int yl, flo
       for (int i = 0; i < 32; ++i)
         if (i == r) g[i] -= a1;
     }
-    if (store) store_chunk<kTF32>(gdst + ch * 32 * kElt, g);
+    put_chunk<kTF32>(o, gcol, ch, g, lane);
   }
 }
 
@@ -473,19 +572,24 @@ __device__ __forceinline__ void bwd_epilogue(const HeadParams& p, uint32_t base,
   const float cT = valid ? p.coef[t] * inv_n : 0.f;
   const float bT1 = -__ldg(p.stats + static_cast<long long>(t) * p.T + rr) * L1;
   const float bTt = -__ldg(p.stats + MT + static_cast<long long>(t) * p.T + rr) * L1;
-  char* gT = static_cast<char*>(p.G) + (static_cast<long long>(t) * p.g_model_stride + rr * p.g_pitch) * kElt;
+  uint32_t nchunks = 0;
+  const uint32_t stage = base + HeadSmem::kStage + static_cast<uint32_t>(warp) * 2 * kHeadStageChunk;
+  const int row0 = tt * kHeadBM + quad * 32;
+  const GOut oT{&p.mapG[t], stage, &nchunks, row0,
+                static_cast<char*>(p.G) + (static_cast<long long>(t) * p.g_model_stride + rr * p.g_pitch) * kElt,
+                row_ok};
 
   float a1[kStud], a2[kStud], b1[kStud], bt[kStud];
-  char* gS[kStud];
+  int ms[kStud];
 #pragma unroll
   for (int j = 0; j < kStud; ++j) {
     const int m = j < nst ? p.order[j + 1] : t;
+    ms[j] = m;
     const float c = valid ? p.coef[m] * inv_n : 0.f;
     a1[j] = c * p.one_minus_alpha;
     a2[j] = c * p.alpha_over_tau;
     b1[j] = -__ldg(p.stats + static_cast<long long>(m) * p.T + rr) * L1;
     bt[j] = -__ldg(p.stats + MT + static_cast<long long>(m) * p.T + rr) * L1;
-    gS[j] = static_cast<char*>(p.G) + (static_cast<long long>(m) * p.g_model_stride + rr * p.g_pitch) * kElt;
   }
   float q[128];
   uint32_t acc = 0, acc_par = 0;
@@ -494,33 +598,47 @@ __device__ __forceinline__ void bwd_epilogue(const HeadParams& p, uint32_t base,
     const long long col0 = static_cast<long long>(vt) * kHeadBN + half * 128;
     const int nvalid = static_cast<int>(max(0LL, min(128LL, p.V - col0)));
     const int yl = y >= 0 ? static_cast<int>(y - col0) : -1;
-    const long long goff = (col0 - p.g_col0) * kElt;
+    const int gcol = static_cast<int>(col0 - p.g_col0);  // column within the group buffer
 
-    if (!epi_acquire(p, base, acc, acc_par, abort_flag)) return;
+    if (!epi_acquire(p, base, acc, acc_par, abort_flag)) break;
     {
       const uint32_t ta = tl + acc * kHeadBN;
+      GOut o = oT;
+      o.gdst += static_cast<long long>(gcol) * kElt;
       if (nvalid == 128)
-        bwd_teacher<false, kTauOne, kTF32>(ta, 128, yl, L1, Lt, bT1, bTt, cT, q, gT + goff, row_ok);
+        bwd_teacher<false, kTauOne, kTF32>(ta, 128, yl, L1, Lt, bT1, bTt, cT, q, o, gcol, lane);
       else
-        bwd_teacher<true, kTauOne, kTF32>(ta, nvalid, yl, L1, Lt, bT1, bTt, cT, q, gT + goff, row_ok);
+        bwd_teacher<true, kTauOne, kTF32>(ta, nvalid, yl, L1, Lt, bT1, bTt, cT, q, o, gcol, lane);
     }
     epi_release(base, acc, acc_par, lane);
 
+    bool aborted = false;
 #pragma unroll
     for (int j = 0; j < kStud; ++j) {
-      if (j < nst) {
-        if (!epi_acquire(p, base, acc, acc_par, abort_flag)) return;
+      if (j < nst && !aborted) {
+        if (!epi_acquire(p, base, acc, acc_par, abort_flag)) {
+          aborted = true;
+          break;
+        }
         const uint32_t ta = tl + acc * kHeadBN;
+        const GOut o{&p.mapG[ms[j]], stage, &nchunks, row0,
+                     static_cast<char*>(p.G) +
+                         (static_cast<long long>(ms[j]) * p.g_model_stride + rr * p.g_pitch + gcol) * kElt,
+                     row_ok};
         if (nvalid == 128)
           bwd_student<false, kTauOne, kTF32>(ta, 128, yl, L1, Lt, b1[j], bt[j], a1[j], a2[j], q,
-                                             gS[j] + goff, row_ok);
+                                             o, gcol, lane);
         else
           bwd_student<true, kTauOne, kTF32>(ta, nvalid, yl, L1, Lt, b1[j], bt[j], a1[j], a2[j], q,
-                                            gS[j] + goff, row_ok);
+                                            o, gcol, lane);
         epi_release(base, acc, acc_par, lane);
       }
     }
+    if (aborted) break;
   }
+  // Every staged store has finished before the CTA's shared memory goes away.
+  if (!kTF32 && lane == 0) bulk_wait_all();
+  __syncwarp();
 }
 
 // ------------------------------------------------------------------ kernel
@@ -576,7 +694,8 @@ __global__ void __launch_bounds__(kHeadThreads, 1) head_kernel(const __grid_cons
   } else {
     regs_increase<kHeadEpiRegs>();
     if constexpr (kMode == kModeFwd)
-      fwd_epilogue<kTauOne>(p, base, tmem, tt, split, warp, lane, abort_flag);
+      fwd_epilogue<kTauOne>(p, base, tmem, reinterpret_cast<float*>(gbase + HeadSmem::kStage), tt,
+                            split, warp, lane, abort_flag);
     else
       bwd_epilogue<kTauOne, kTF32>(p, base, tmem, tt, split, warp, lane, abort_flag);
   }

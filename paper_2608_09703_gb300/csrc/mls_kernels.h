@@ -30,7 +30,11 @@ static_assert(2 * 128 * kHeadEpiRegs + 128 * kHeadCtlRegs == kHeadThreads * kHea
               "register reallocation must add up to the launch allocation");
 constexpr uint32_t kHeadABytes = kHeadBM * 128;
 constexpr uint32_t kHeadBBytes = kHeadBN * 128;
-constexpr uint32_t kHeadSmem = kHeadStages * (kHeadABytes + kHeadBBytes) + 1024 + 1024;
+// Backward: each epilogue warp stages its dL/dz chunks (32 tokens x 32 bf16
+// columns, 2 KB, 64B-swizzled) in two buffers and writes them with TMA stores.
+constexpr uint32_t kHeadStageChunk = 32 * 64;
+constexpr uint32_t kHeadStaging = kHeadEpiWarps * 2 * kHeadStageChunk;
+constexpr uint32_t kHeadSmem = kHeadStages * (kHeadABytes + kHeadBBytes) + kHeadStaging + 1024 + 1024;
 
 // Partial row state written by the forward head kernel, per (partial, field, model, token).
 // kPartAcc holds, for a student, sum_v q~_v z_m[v] with q~ relative to the
@@ -53,13 +57,14 @@ struct HeadParams {
   const int* y;                  // targets [T]
   int* status;
   // forward
-  float* part;                   // [2*S][kPartFields][M][T]
+  float* part;                   // [S][kPartFields][M][T]
   // backward
   const float* stats;            // [2][M][T]: logsumexp(z), logsumexp(z/tau)
   const float* inv_n;            // device scalar 1/N (0 if N == 0)
   float coef[kMaxModels];        // grad_scale * w_m
   float one_minus_alpha;         // (1 - alpha)
   float alpha_over_tau;          // alpha / tau
+  CUtensorMap mapG[kMaxModels];  // G_m [T, g_pitch] bf16, box {32, 32}, 64B swizzle (TMA store)
   void* G;                       // [M][T][g_pitch] bf16 (fp32 for fp32 inputs)
   long long g_model_stride;      // elements
   long long g_pitch;             // elements per token row

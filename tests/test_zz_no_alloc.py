@@ -60,8 +60,9 @@ def test_noalloc_forward_matches_workspace_forward_on_two_calls():
 
 def test_noalloc_rejects_problems_beyond_the_scratch():
     dev = torch.device("cuda")
-    # 4 sub-models x 200000 tokens: the partial row states alone exceed 32 MiB
-    d, T, V = (64, 64, 64, 64), 200000, 1000
+    # 4 sub-models x 10^6 tokens: the partial row states alone (6 floats per
+    # token and sub-model) exceed the 64 MiB scratch
+    d, T, V = (64, 64, 64, 64), 1000000, 1000
     H = [torch.zeros(T, x, dtype=torch.bfloat16, device=dev) for x in d]
     W = [torch.zeros(V, x, dtype=torch.bfloat16, device=dev) for x in d]
     y = torch.zeros(T, dtype=torch.int32, device=dev)
