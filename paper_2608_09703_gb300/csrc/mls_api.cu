@@ -25,6 +25,8 @@ struct DeviceState {
   bool ready = false;
   int err = 0;
   int sms = 0;
+  int gemm_pairs = 0;  // co-resident CTA pairs of the GEMM kernel
+  int head_pairs = 0;  // co-resident CTA pairs of the head kernels
   int* status = nullptr;
 };
 
@@ -64,6 +66,10 @@ int device_state(DeviceState** out) {
       s.err = fail(MLS_ERR_CUDA, "head kernel attributes", e);
     } else if ((e = setup_gemm_kernels()) != cudaSuccess) {
       s.err = fail(MLS_ERR_CUDA, "gemm kernel attributes", e);
+    } else if ((s.gemm_pairs = gemm_max_active_pairs()) <= 0) {
+      s.err = fail(MLS_ERR_CUDA, "gemm cluster occupancy");
+    } else if ((s.head_pairs = head_max_active_pairs()) <= 0) {
+      s.err = fail(MLS_ERR_CUDA, "head cluster occupancy");
     } else if (!g_encode) {
       void* fn = nullptr;
       cudaDriverEntryPointQueryResult q;
@@ -80,13 +86,13 @@ int device_state(DeviceState** out) {
   return s.err;
 }
 
-int current_sms() {
-  int dev = 0, sms = 0;
-  if (cudaGetDevice(&dev) == cudaSuccess &&
-      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && sms > 0)
-    return sms;
+// Co-resident head-kernel CTA pairs on the current device, for sizing a plan
+// without launching (76 on a GB300 when no device can be queried).
+int current_head_pairs() {
+  DeviceState* dev = nullptr;
+  if (device_state(&dev) == MLS_OK && dev->head_pairs > 0) return dev->head_pairs;
   cudaGetLastError();
-  return 152;  // GB300
+  return 76;
 }
 
 // ------------------------------------------------------------------ planning
@@ -110,10 +116,11 @@ struct Plan {
   size_t total = 0;
 };
 
-// CTAs per token tile (vocabulary splits).  Each CTA of a head kernel walks
-// ceil(tiles / S) vocabulary tiles and one CTA fits per SM, so the kernel lasts
-// about waves * (tiles per CTA + a fixed per-CTA cost); S minimises that.
-int choose_splits(int ntt, long long tiles, int sms) {
+// CTA pairs per token tile (vocabulary splits).  Each pair of a head kernel
+// walks ceil(tiles / S) vocabulary tiles and `pairs` pairs are resident at a
+// time, so the kernel lasts about waves * (tiles per pair + a fixed per-pair
+// cost); S minimises that.
+int choose_splits(int ntt, long long tiles, int pairs) {
   if (ntt < 1) ntt = 1;
   if (tiles < 1) return 1;
   const double kCtaCost = 0.25;  // prologue + pipeline drain, in vocabulary tiles
@@ -122,7 +129,7 @@ int choose_splits(int ntt, long long tiles, int sms) {
   for (long long S = 1; S <= tiles && S <= 512; ++S) {
     const long long per = (tiles + S - 1) / S;
     if (S > 1 && (per - 1) * S >= tiles) continue;  // same tiles per CTA with fewer CTAs
-    const long long waves = (ntt * S + sms - 1) / sms;
+    const long long waves = (ntt * S + pairs - 1) / pairs;
     const double cost = waves * (per + kCtaCost);
     if (cost < best_cost - 1e-9) {
       best_cost = cost;
@@ -152,13 +159,13 @@ int validate(const mls_problem* p) {
   return MLS_OK;
 }
 
-Plan make_plan(const mls_problem* p, int sms) {
+Plan make_plan(const mls_problem* p, int pairs) {
   Plan pl;
   pl.elt = p->in_dtype == MLS_BF16 ? 2 : 4;
   const long long T = p->T, V = p->V, M = p->M;
-  pl.ntt = static_cast<int>(ceil_div(T, kHeadBM));
+  pl.ntt = static_cast<int>(ceil_div(T, 2 * kHeadBM));  // token tiles of a CTA pair
   pl.nvt = static_cast<int>(ceil_div(V, kHeadBN));
-  pl.S = choose_splits(pl.ntt, pl.nvt, sms);
+  pl.S = choose_splits(pl.ntt, pl.nvt, pairs);
   pl.nparts = pl.S;
   pl.merge_blocks = static_cast<int>(ceil_div(T, kMergeThreads));
   size_t o = 0;
@@ -254,7 +261,7 @@ int encode_head_maps(HeadParams& hp, const mls_problem* p, const Plan& pl, const
   const int KE = 128 / pl.elt;
   for (int m = 0; m < p->M; ++m) {
     if (encode(&hp.mapH[m], H[m], pl.elt, p->d[m], p->T, p->d[m], KE, kHeadBM) ||
-        encode(&hp.mapW[m], W[m], pl.elt, p->d[m], p->V, p->d[m], KE, kHeadBN))
+        encode(&hp.mapW[m], W[m], pl.elt, p->d[m], p->V, p->d[m], KE, kHeadBHalf))
       return MLS_ERR_CUDA;
   }
   return MLS_OK;
@@ -312,7 +319,7 @@ using namespace mls;
 
 extern "C" size_t mls_workspace_size(const mls_problem* p) {
   if (validate(p) != MLS_OK) return 0;
-  return make_plan(p, current_sms()).total;
+  return make_plan(p, current_head_pairs()).total;
 }
 
 extern "C" int mls_head_loss_fwd(const mls_problem* p, const void* const* H, const void* const* W,
@@ -328,7 +335,7 @@ extern "C" int mls_head_loss_fwd(const mls_problem* p, const void* const* H, con
   }
   DeviceState* dev = nullptr;
   if ((rc = device_state(&dev))) return rc;
-  const Plan pl = make_plan(p, dev->sms);
+  const Plan pl = make_plan(p, dev->head_pairs);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (p->T == 0) return launch_ok(cudaMemsetAsync(loss, 0, sizeof(float), s));
   if ((rc = check_ws(pl, ws, ws_bytes, pl.total))) return rc;
@@ -384,7 +391,7 @@ extern "C" int mls_head_loss_bwd(const mls_problem* p, const void* const* H, con
   }
   DeviceState* dev = nullptr;
   if ((rc = device_state(&dev))) return rc;
-  const Plan pl = make_plan(p, dev->sms);
+  const Plan pl = make_plan(p, dev->head_pairs);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (p->T == 0) {
     for (int m = 0; m < p->M; ++m)
@@ -443,8 +450,8 @@ extern "C" int mls_head_loss_bwd(const mls_problem* p, const void* const* H, con
         return rc;
       if (encode(&gw.mapA[m], GT + static_cast<size_t>(m) * pl.group * pl.t_pitch, 4, p->T,
                  pl.group, pl.t_pitch, KE, kGemmBM) ||
-          encode(&gw.mapB[m], HT, 4, p->T, p->d[m], pl.t_pitch, KE, kGemmBN) ||
-          encode(&gh.mapB[m], WT, 4, p->V, p->d[m], pl.v_pitch, KE, kGemmBN))
+          encode(&gw.mapB[m], HT, 4, p->T, p->d[m], pl.t_pitch, KE, kGemmBHalf) ||
+          encode(&gh.mapB[m], WT, 4, p->V, p->d[m], pl.v_pitch, KE, kGemmBHalf))
         return MLS_ERR_CUDA;
     }
   }
@@ -457,7 +464,7 @@ extern "C" int mls_head_loss_bwd(const mls_problem* p, const void* const* H, con
     const long long gc = (p->V - c0 < pl.group) ? p->V - c0 : pl.group;  // columns of this group
     hp.vt_begin = static_cast<int>(g * tiles_per_group);
     hp.vt_end = static_cast<int>(ceil_div(c0 + gc, kHeadBN));
-    hp.S = choose_splits(pl.ntt, hp.vt_end - hp.vt_begin, dev->sms);
+    hp.S = choose_splits(pl.ntt, hp.vt_end - hp.vt_begin, dev->head_pairs);
     hp.g_col0 = c0;
     if ((rc = timed("head_bwd", s, [&] { return launch_head_bwd(hp, tf32, p->tau == 1.0f, s); }))) return rc;
     if (tf32)
@@ -480,7 +487,7 @@ extern "C" int mls_head_loss_bwd(const mls_problem* p, const void* const* H, con
       a.accumulate = 0;
       a.tiles_n = static_cast<int>(ceil_div(p->d[m], kGemmBN));
       a.tile_begin = tw;
-      tw += static_cast<int>(ceil_div(gc, kGemmBM)) * a.tiles_n;
+      tw += static_cast<int>(ceil_div(gc, 2 * kGemmBM)) * a.tiles_n;
 
       GemmProblem& b = gh.prob[m];
       b.Mrows = static_cast<int>(p->T);
@@ -493,11 +500,13 @@ extern "C" int mls_head_loss_bwd(const mls_problem* p, const void* const* H, con
       b.accumulate = g > 0 ? 1 : 0;
       b.tiles_n = static_cast<int>(ceil_div(p->d[m], kGemmBN));
       b.tile_begin = th;
-      th += static_cast<int>(ceil_div(p->T, kGemmBM)) * b.tiles_n;
+      th += static_cast<int>(ceil_div(p->T, 2 * kGemmBM)) * b.tiles_n;
     }
     gw.total_tiles = tw;
     gh.total_tiles = th;
-    const int grid_w = tw < dev->sms ? tw : dev->sms, grid_h = th < dev->sms ? th : dev->sms;
+    // persistent: one CTA pair per resident pair slot, never more pairs than tiles
+    const int pairs = dev->gemm_pairs;
+    const int grid_w = 2 * (tw < pairs ? tw : pairs), grid_h = 2 * (th < pairs ? th : pairs);
     if (tf32) {
       if ((rc = timed("gemm_dw", s, [&] { return launch_gemm_kk(gw, true, grid_w, s); }))) return rc;
       if ((rc = timed("gemm_dh", s, [&] { return launch_gemm_kk(gh, true, grid_h, s); }))) return rc;
@@ -623,7 +632,7 @@ extern "C" int mls_head_loss_fwd_noalloc(const mls_problem* p, const void* const
   }
   DeviceState* dev = nullptr;
   if ((rc = device_state(&dev))) return rc;
-  const Plan pl = make_plan(p, dev->sms);
+  const Plan pl = make_plan(p, dev->head_pairs);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (p->T == 0) return launch_ok(cudaMemsetAsync(loss, 0, sizeof(float), s));
   if (pl.fwd_bytes > static_cast<size_t>(MLS_NOALLOC_SCRATCH_BYTES))

@@ -8,10 +8,15 @@
 // only used with K-major operands here, so fp32 inputs go through transposed
 // copies (G^T, H^T, W^T) instead.
 //
-// Persistent CTAs walk a list of 128x256 output tiles over up to four
-// problems (one per sub-model): warp 4 streams A/B k-blocks with TMA, warp 5
-// issues the MMAs into one of two TMEM accumulators, warps 0-3 drain the other
-// accumulator to global memory (optionally adding to what is there).
+// CTA pairs (clusters of 2) own 256x256 output tiles: each CTA loads the 128
+// rows of A and the 128 rows of B that are its half, the even CTA issues
+// 256x256xK pair MMAs (cta_group::2) and each CTA drains its 128 accumulator
+// rows.  Persistent pairs walk a list of tiles over up to four problems (one
+// per sub-model):
+//   warp 4    TMA producer (each CTA its own halves; both CTAs' loads complete
+//             on the even CTA's barrier, which expects the bytes of both)
+//   warp 5    MMA issuer (even CTA)
+//   warps 0-3 epilogue (each CTA its 128 rows)
 #include "mls_device.cuh"
 #include "mls_kernels.h"
 
@@ -22,6 +27,8 @@ struct GemmSmem {
   static constexpr uint32_t kA = 0;
   static constexpr uint32_t kB = kGemmStages * kGemmABytes;
   static constexpr uint32_t kBar = kB + kGemmStages * kGemmBBytes;
+  // full (even CTA): both CTAs' loads landed; empty: the pair's MMAs are done
+  // with the stage; accf/acce: accumulator full/empty.
   static __device__ __forceinline__ uint32_t full(uint32_t b, int s) { return b + kBar + 8u * s; }
   static __device__ __forceinline__ uint32_t empty(uint32_t b, int s) {
     return b + kBar + 8u * (kGemmStages + s);
@@ -43,6 +50,7 @@ static_assert(GemmSmem::kEnd + 1024 <= kGemmSmem, "gemm shared memory map overfl
 
 constexpr uint32_t kTmemCols = 512;
 constexpr uint64_t kDrainNs = 100000000ull;
+constexpr int kPairM = 2 * kGemmBM;  // output rows of a pair tile
 
 struct TileCoord {
   int prob, tm, tn;
@@ -55,43 +63,46 @@ __device__ __forceinline__ TileCoord decode_tile(const GemmParams& p, int t) {
   return {i, local / p.prob[i].tiles_n, local % p.prob[i].tiles_n};
 }
 
+// This CTA's loads: its 128 rows of A and its 128 rows of B for every k-block.
 template <bool kTF32, bool kAMN, bool kBMN>
-__device__ __forceinline__ void gemm_producer(const GemmParams& p, uint32_t base,
+__device__ __forceinline__ void gemm_producer(const GemmParams& p, uint32_t base, uint32_t rank,
                                               volatile int* abort_flag) {
-  constexpr int KE = kTF32 ? 32 : 64;           // elements per 128-byte row
-  constexpr uint32_t kBox = KE * 128;           // bytes of one MN-major box {KE, KE}
+  constexpr int KE = kTF32 ? 32 : 64;  // elements per 128-byte row
+  constexpr uint32_t kBox = KE * 128;  // bytes of one MN-major box {KE, KE}
+  const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
   int stage = 0;
   uint32_t phase = 0, filled = 0, lastpar = 0;
   bool ok = true;
-  for (int t = blockIdx.x; ok && t < p.total_tiles; t += gridDim.x) {
+  for (int t = pair; ok && t < p.total_tiles; t += npairs) {
     const TileCoord tc = decode_tile(p, t);
     const GemmProblem& pr = p.prob[tc.prob];
     const CUtensorMap* ma = &p.mapA[pr.a_map];
     const CUtensorMap* mb = &p.mapB[pr.b_map];
     const int nkb = (pr.K + KE - 1) / KE;
-    const int m0 = pr.a_m0 + tc.tm * kGemmBM;
-    const int n0 = pr.b_n0 + tc.tn * kGemmBN;
+    const int m0 = pr.a_m0 + tc.tm * kPairM + static_cast<int>(rank) * kGemmBM;
+    const int n0 = pr.b_n0 + tc.tn * kGemmBN + static_cast<int>(rank) * kGemmBHalf;
     for (int kb = 0; kb < nkb; ++kb) {
       if (!mbar_wait(GemmSmem::empty(base, stage), phase ^ 1u, abort_flag, p.status)) {
         ok = false;
         break;
       }
-      const uint32_t fb = GemmSmem::full(base, stage);
-      mbar_arrive_expect_tx(fb, kGemmABytes + kGemmBBytes);
+      const uint32_t fb = map_to_rank(GemmSmem::full(base, stage), 0);
+      if (rank == 0) mbar_arrive_expect_tx(GemmSmem::full(base, stage), 2 * (kGemmABytes + kGemmBBytes));
       const uint32_t sa = base + GemmSmem::kA + stage * kGemmABytes;
       const uint32_t sb = base + GemmSmem::kB + stage * kGemmBBytes;
       const int ka = pr.a_k0 + kb * KE, kbb = pr.b_k0 + kb * KE;
       if (kAMN) {
 #pragma unroll
-        for (int j = 0; j < kGemmBM / KE; ++j) tma_load_2d(sa + j * kBox, ma, fb, m0 + j * KE, ka);
+        for (int j = 0; j < kGemmBM / KE; ++j) tma_load_2d_pair(sa + j * kBox, ma, fb, m0 + j * KE, ka);
       } else {
-        tma_load_2d(sa, ma, fb, ka, m0);
+        tma_load_2d_pair(sa, ma, fb, ka, m0);
       }
       if (kBMN) {
 #pragma unroll
-        for (int j = 0; j < kGemmBN / KE; ++j) tma_load_2d(sb + j * kBox, mb, fb, n0 + j * KE, kbb);
+        for (int j = 0; j < kGemmBHalf / KE; ++j)
+          tma_load_2d_pair(sb + j * kBox, mb, fb, n0 + j * KE, kbb);
       } else {
-        tma_load_2d(sb, mb, fb, kbb, n0);
+        tma_load_2d_pair(sb, mb, fb, kbb, n0);
       }
       filled |= 1u << stage;
       lastpar = (lastpar & ~(1u << stage)) | (phase << stage);
@@ -101,9 +112,16 @@ __device__ __forceinline__ void gemm_producer(const GemmParams& p, uint32_t base
       }
     }
   }
-  if (!ok) {
-    for (int s = 0; s < kGemmStages; ++s)
-      if ((filled >> s) & 1u) mbar_wait_drain(GemmSmem::full(base, s), (lastpar >> s) & 1u, kDrainNs);
+  if (!ok && filled) {
+    // Loads already issued must land before this CTA's shared memory goes away.
+    // The even CTA can watch its barriers; the odd CTA's loads are counted on
+    // the even CTA's barriers, so it waits out a bound no TMA load approaches.
+    if (rank == 0) {
+      for (int s = 0; s < kGemmStages; ++s)
+        if ((filled >> s) & 1u) mbar_wait_drain(GemmSmem::full(base, s), (lastpar >> s) & 1u, kDrainNs);
+    } else {
+      spin_ns(kDrainNs);
+    }
   }
 }
 
@@ -111,16 +129,18 @@ template <bool kTF32, bool kAMN, bool kBMN>
 __device__ __forceinline__ void gemm_mma(const GemmParams& p, uint32_t base, uint32_t tmem,
                                          volatile int* abort_flag) {
   constexpr int KE = kTF32 ? 32 : 64;
-  constexpr uint32_t kIdesc = make_idesc(kGemmBM, kGemmBN, kTF32, kAMN, kBMN);
+  constexpr uint32_t kIdesc = make_idesc(kPairM, kGemmBN, kTF32, kAMN, kBMN);
   constexpr uint32_t kBox = KE * 128;
   // Advance per MMA (32 bytes of K): along a 128-byte row for K-major
   // operands, by (32 / element size) rows of 128 bytes for MN-major ones.
   constexpr uint32_t kStepK = 32u >> 4;
   constexpr uint32_t kStepMN = ((32u / (kTF32 ? 4u : 2u)) * 128u) >> 4;
+  constexpr uint16_t kBoth = 0x3;
+  const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
   int stage = 0;
   uint32_t phase = 0, acc = 0, acc_par = 0;
   bool ok = true;
-  for (int t = blockIdx.x; ok && t < p.total_tiles; t += gridDim.x) {
+  for (int t = pair; ok && t < p.total_tiles; t += npairs) {
     const TileCoord tc = decode_tile(p, t);
     const int nkb = (p.prob[tc.prob].K + KE - 1) / KE;
     if (!mbar_wait(GemmSmem::acce(base, acc), acc_par ^ 1u, abort_flag, p.status)) {
@@ -139,34 +159,36 @@ __device__ __forceinline__ void gemm_mma(const GemmParams& p, uint32_t base, uin
       const uint64_t bd = make_sdesc(base + GemmSmem::kB + stage * kGemmBBytes, kBMN ? kBox : 16u);
 #pragma unroll
       for (int kk = 0; kk < 4; ++kk)
-        mma_issue<kTF32>(d, ad + kk * (kAMN ? kStepMN : kStepK), bd + kk * (kBMN ? kStepMN : kStepK),
-                         kIdesc, (kb | kk) != 0);
-      mma_commit(GemmSmem::empty(base, stage));
+        mma_issue_pair<kTF32>(d, ad + kk * (kAMN ? kStepMN : kStepK),
+                              bd + kk * (kBMN ? kStepMN : kStepK), kIdesc, (kb | kk) != 0);
+      mma_commit_pair(GemmSmem::empty(base, stage), kBoth);
       if (++stage == kGemmStages) {
         stage = 0;
         phase ^= 1u;
       }
     }
     if (!ok) break;
-    mma_commit(GemmSmem::accf(base, acc));
+    mma_commit_pair(GemmSmem::accf(base, acc), kBoth);
     acc ^= 1u;
     if (acc == 0) acc_par ^= 1u;
   }
-  mma_commit(GemmSmem::drain(base));
+  mma_commit_pair(GemmSmem::drain(base), 0x1);
   mbar_wait_drain(GemmSmem::drain(base), 0, kDrainNs);
 }
 
 __device__ __forceinline__ void gemm_epilogue(const GemmParams& p, uint32_t base, uint32_t tmem,
-                                              int warp, int lane, volatile int* abort_flag) {
+                                              uint32_t rank, int warp, int lane,
+                                              volatile int* abort_flag) {
+  const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
   uint32_t acc = 0, acc_par = 0;
   const uint32_t tl = tmem + (static_cast<uint32_t>(warp * 32) << 16);
-  for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x) {
+  for (int t = pair; t < p.total_tiles; t += npairs) {
     const TileCoord tc = decode_tile(p, t);
     const GemmProblem& pr = p.prob[tc.prob];
     const bool ok = mbar_wait(GemmSmem::accf(base, acc), acc_par, abort_flag, p.status);
     if (!__all_sync(0xffffffffu, ok)) return;
     tc_fence_after();
-    const long long row = static_cast<long long>(tc.tm) * kGemmBM + warp * 32 + lane;
+    const long long row = static_cast<long long>(tc.tm) * kPairM + rank * kGemmBM + warp * 32 + lane;
     const bool row_ok = row < pr.Mrows;
     float* crow = pr.C + (row_ok ? row : 0) * pr.ldc;
     float v[32];
@@ -174,38 +196,40 @@ __device__ __forceinline__ void gemm_epilogue(const GemmParams& p, uint32_t base
     for (int c = 0; c < kGemmBN / 32; ++c) {
       tmem_ld32(tl + acc * kGemmBN + c * 32, v);
       const int col = tc.tn * kGemmBN + c * 32;
-      if (!row_ok || col >= pr.Ncols) continue;
-      float* dst = crow + col;
-      if (col + 32 <= pr.Ncols) {
-        float4* d4 = reinterpret_cast<float4*>(dst);
+      if (row_ok && col < pr.Ncols) {
+        float* dst = crow + col;
+        if (col + 32 <= pr.Ncols) {
+          float4* d4 = reinterpret_cast<float4*>(dst);
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          float4 o = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
-          if (pr.accumulate) {
-            const float4 c4 = d4[i];
-            o.x += c4.x;
-            o.y += c4.y;
-            o.z += c4.z;
-            o.w += c4.w;
+          for (int i = 0; i < 8; ++i) {
+            float4 o = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+            if (pr.accumulate) {
+              const float4 c4 = d4[i];
+              o.x += c4.x;
+              o.y += c4.y;
+              o.z += c4.z;
+              o.w += c4.w;
+            }
+            d4[i] = o;
           }
-          d4[i] = o;
-        }
-      } else {
+        } else {
 #pragma unroll
-        for (int i = 0; i < 32; ++i)
-          if (col + i < pr.Ncols) dst[i] = pr.accumulate ? dst[i] + v[i] : v[i];
+          for (int i = 0; i < 32; ++i)
+            if (col + i < pr.Ncols) dst[i] = pr.accumulate ? dst[i] + v[i] : v[i];
+        }
       }
     }
     tc_fence_before();
     __syncwarp();
-    if (lane == 0) mbar_arrive(GemmSmem::acce(base, acc));
+    if (lane == 0) mbar_arrive_remote(map_to_rank(GemmSmem::acce(base, acc), 0));
     acc ^= 1u;
     if (acc == 0) acc_par ^= 1u;
   }
 }
 
 template <bool kTF32, bool kAMN, bool kBMN>
-__global__ void __launch_bounds__(kGemmThreads, 1) gemm_kernel(const __grid_constant__ GemmParams p) {
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
+    gemm_kernel(const __grid_constant__ GemmParams p) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -213,6 +237,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_kernel(const __grid_cons
   volatile int* abort_flag = reinterpret_cast<volatile int*>(gbase + GemmSmem::kAbort);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + GemmSmem::kTmemSlot);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
 
   if (threadIdx.x == 0) {
     *abort_flag = 0;
@@ -222,14 +247,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_kernel(const __grid_cons
     }
     for (uint32_t a = 0; a < 2; ++a) {
       mbar_init(GemmSmem::accf(base, a), 1);
-      mbar_init(GemmSmem::acce(base, a), kGemmEpiWarps);
+      mbar_init(GemmSmem::acce(base, a), 2 * kGemmEpiWarps);
     }
     mbar_init(GemmSmem::drain(base), 1);
     fence_barrier_init();
   }
   if (warp == kGemmEpiWarps + 1) {
-    tmem_alloc(base + GemmSmem::kTmemSlot, kTmemCols);
-    tmem_relinquish();
+    tmem_alloc_pair(base + GemmSmem::kTmemSlot, kTmemCols);
+    tmem_relinquish_pair();
   }
   if (warp == kGemmEpiWarps && lane == 0) {
     for (int i = 0; i < p.nprob; ++i) {
@@ -238,24 +263,24 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_kernel(const __grid_cons
     }
   }
   tc_fence_before();
-  __syncthreads();
+  cluster_sync();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
   if (warp == kGemmEpiWarps) {
-    if (lane == 0) gemm_producer<kTF32, kAMN, kBMN>(p, base, abort_flag);
+    if (lane == 0) gemm_producer<kTF32, kAMN, kBMN>(p, base, rank, abort_flag);
   } else if (warp == kGemmEpiWarps + 1) {
-    if (lane == 0) gemm_mma<kTF32, kAMN, kBMN>(p, base, tmem, abort_flag);
+    if (lane == 0 && rank == 0) gemm_mma<kTF32, kAMN, kBMN>(p, base, tmem, abort_flag);
     __syncwarp();
   } else {
-    gemm_epilogue(p, base, tmem, warp, lane, abort_flag);
+    gemm_epilogue(p, base, tmem, rank, warp, lane, abort_flag);
   }
 
   tc_fence_before();
-  __syncthreads();
+  cluster_sync();
   if (warp == kGemmEpiWarps + 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, kTmemCols);
+    tmem_dealloc_pair(tmem, kTmemCols);
   }
 }
 
@@ -279,6 +304,21 @@ cudaError_t launch_gemm_dh(const GemmParams& p, bool tf32, int grid, cudaStream_
 }
 cudaError_t launch_gemm_kk(const GemmParams& p, bool tf32, int grid, cudaStream_t s) {
   return launch<false, false>(p, tf32, grid, s);
+}
+
+// How many CTA pairs of the GEMM kernel can be resident at once (GPCs with an
+// odd number of free SMs host one CTA fewer than a pair needs).
+int gemm_max_active_pairs() {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2 * 1024);
+  cfg.blockDim = dim3(kGemmThreads);
+  cfg.dynamicSmemBytes = kGemmSmem;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, gemm_kernel<false, true, true>, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  return n;
 }
 
 cudaError_t setup_gemm_kernels() {

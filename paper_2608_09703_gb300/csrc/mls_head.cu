@@ -1,14 +1,17 @@
 // Fused LM-head kernels of the Matryoshka-suite output stage.
 //
-// One CTA owns kHeadBM = 128 tokens and a strided set of 256-column vocabulary
-// tiles.  For every vocabulary tile it computes the teacher's logit tile
-// z_t = H_t W_t^T first and then each student's z_m = H_m W_m^T (Sec. 2: each
-// sub-model has its own head W^m in R^{V x D_m}), on the tensor cores:
+// A CTA pair (cluster of 2) owns 256 tokens and a strided set of 256-column
+// vocabulary tiles.  For every vocabulary tile it computes the teacher's logit
+// tile z_t = H_t W_t^T first and then each student's z_m = H_m W_m^T (Sec. 2:
+// each sub-model has its own head W^m in R^{V x D_m}), on the tensor cores:
 //
-//   warp 8   TMA producer: H_m and W_m k-blocks (128 bytes of K) into a
-//            4-stage shared-memory ring, 128B-swizzled
-//   warp 9   MMA issuer: tcgen05.mma 128x256xK into one of two TMEM
-//            accumulators (2 x 256 columns), tcgen05.commit to barriers
+//   warp 8   TMA producer (each CTA): its 128 token rows of H_m and its 128
+//            vocabulary rows of W_m, k-blocks of 128 bytes, into a 6-stage
+//            128B-swizzled ring; both CTAs' loads complete on the even CTA's
+//            barrier
+//   warp 9   MMA issuer (even CTA): pair tcgen05.mma 256x256xK (cta_group::2)
+//            into one of two TMEM accumulators (2 x 256 columns in each CTA),
+//            commits multicast to both CTAs
 //   warps 0-7 epilogue: tcgen05.ld, one thread per (token, half tile); these
 //            two warpgroups take the registers the third one gives up, since
 //            each thread keeps the teacher's 128 weights of a tile in registers
@@ -69,8 +72,8 @@ constexpr uint64_t kDrainNs = 100000000ull;     // bound for shutdown waits
 
 // ------------------------------------------------------------------ producer
 template <bool kTF32>
-__device__ __forceinline__ void head_producer(const HeadParams& p, uint32_t base, int tt, int split,
-                                              volatile int* abort_flag) {
+__device__ __forceinline__ void head_producer(const HeadParams& p, uint32_t base, int row0,
+                                              uint32_t rank, int split, volatile int* abort_flag) {
   constexpr int KE = kTF32 ? 32 : 64;  // elements in 128 bytes of K
   int stage = 0;
   uint32_t phase = 0, filled = 0, lastpar = 0;
@@ -83,12 +86,12 @@ __device__ __forceinline__ void head_producer(const HeadParams& p, uint32_t base
           ok = false;
           break;
         }
-        const uint32_t fb = HeadSmem::full(base, stage);
-        mbar_arrive_expect_tx(fb, kHeadABytes + kHeadBBytes);
-        tma_load_2d(base + HeadSmem::kA + stage * kHeadABytes, &p.mapH[m], fb, kb * KE,
-                    tt * kHeadBM);
-        tma_load_2d(base + HeadSmem::kB + stage * kHeadBBytes, &p.mapW[m], fb, kb * KE,
-                    vt * kHeadBN);
+        // both CTAs' halves are counted on the even CTA's barrier
+        if (rank == 0) mbar_arrive_expect_tx(HeadSmem::full(base, stage), 2 * (kHeadABytes + kHeadBBytes));
+        const uint32_t fb = map_to_rank(HeadSmem::full(base, stage), 0);
+        tma_load_2d_pair(base + HeadSmem::kA + stage * kHeadABytes, &p.mapH[m], fb, kb * KE, row0);
+        tma_load_2d_pair(base + HeadSmem::kB + stage * kHeadBBytes, &p.mapW[m], fb, kb * KE,
+                         vt * kHeadBN + static_cast<int>(rank) * kHeadBHalf);
         filled |= 1u << stage;
         lastpar = (lastpar & ~(1u << stage)) | (phase << stage);
         if (++stage == kHeadStages) {
@@ -98,10 +101,16 @@ __device__ __forceinline__ void head_producer(const HeadParams& p, uint32_t base
       }
     }
   }
-  if (!ok) {
-    // Let every load already issued land before the CTA's shared memory goes away.
-    for (int s = 0; s < kHeadStages; ++s)
-      if ((filled >> s) & 1u) mbar_wait_drain(HeadSmem::full(base, s), (lastpar >> s) & 1u, kDrainNs);
+  if (!ok && filled) {
+    // Loads already issued must land before this CTA's shared memory goes away.
+    // The even CTA can watch its barriers; the odd CTA's loads are counted on
+    // the even CTA's barriers, so it waits out a bound no TMA load approaches.
+    if (rank == 0) {
+      for (int s = 0; s < kHeadStages; ++s)
+        if ((filled >> s) & 1u) mbar_wait_drain(HeadSmem::full(base, s), (lastpar >> s) & 1u, kDrainNs);
+    } else {
+      spin_ns(kDrainNs);
+    }
   }
 }
 
@@ -109,7 +118,8 @@ __device__ __forceinline__ void head_producer(const HeadParams& p, uint32_t base
 template <bool kTF32>
 __device__ __forceinline__ void head_mma(const HeadParams& p, uint32_t base, uint32_t tmem,
                                          int split, volatile int* abort_flag) {
-  constexpr uint32_t kIdesc = make_idesc(kHeadBM, kHeadBN, kTF32, false, false);
+  constexpr uint32_t kIdesc = make_idesc(2 * kHeadBM, kHeadBN, kTF32, false, false);
+  constexpr uint16_t kBoth = 0x3;
   int stage = 0;
   uint32_t phase = 0, acc = 0, acc_par = 0;
   bool ok = true;
@@ -132,21 +142,21 @@ __device__ __forceinline__ void head_mma(const HeadParams& p, uint32_t base, uin
         const uint64_t bd = make_sdesc(base + HeadSmem::kB + stage * kHeadBBytes, 16);
 #pragma unroll
         for (int kk = 0; kk < 4; ++kk)  // 4 x 32 bytes of K per stage
-          mma_issue<kTF32>(d, ad + 2u * kk, bd + 2u * kk, kIdesc, (kb | kk) != 0);
-        mma_commit(HeadSmem::empty(base, stage));
+          mma_issue_pair<kTF32>(d, ad + 2u * kk, bd + 2u * kk, kIdesc, (kb | kk) != 0);
+        mma_commit_pair(HeadSmem::empty(base, stage), kBoth);
         if (++stage == kHeadStages) {
           stage = 0;
           phase ^= 1u;
         }
       }
       if (!ok) break;
-      mma_commit(HeadSmem::accf(base, acc));
+      mma_commit_pair(HeadSmem::accf(base, acc), kBoth);
       acc ^= 1u;
       if (acc == 0) acc_par ^= 1u;
     }
   }
   // Every MMA this thread issued has finished before TMEM is released.
-  mma_commit(HeadSmem::drain(base));
+  mma_commit_pair(HeadSmem::drain(base), 0x1);
   mbar_wait_drain(HeadSmem::drain(base), 0, kDrainNs);
 }
 
@@ -163,7 +173,7 @@ __device__ __forceinline__ void epi_release(uint32_t base, uint32_t& acc, uint32
                                             int lane) {
   tc_fence_before();
   __syncwarp();
-  if (lane == 0) mbar_arrive(HeadSmem::acce(base, acc));
+  if (lane == 0) mbar_arrive_remote(map_to_rank(HeadSmem::acce(base, acc), 0));
   acc ^= 1u;
   if (acc == 0) acc_par ^= 1u;
 }
@@ -306,10 +316,10 @@ __device__ __forceinline__ int merged_argmax(float ma, int aa, float mb, int ab)
 
 template <bool kTauOne>
 __device__ __forceinline__ void fwd_epilogue(const HeadParams& p, uint32_t base, uint32_t tmem,
-                                             float* xchg, int tt, int split, int warp, int lane,
-                                             volatile int* abort_flag) {
+                                             float* xchg, int row_base, int split, int warp,
+                                             int lane, volatile int* abort_flag) {
   const int quad = warp & 3, half = warp >> 2;
-  const long long row = static_cast<long long>(tt) * kHeadBM + quad * 32 + lane;
+  const long long row = static_cast<long long>(row_base) + quad * 32 + lane;
   const bool row_ok = row < p.T;
   const int y = row_ok ? __ldg(p.y + row) : -1;
   const uint32_t tl = tmem + (static_cast<uint32_t>(quad * 32) << 16) + static_cast<uint32_t>(half * 128);
@@ -553,11 +563,11 @@ __device__ __forceinline__ void bwd_student(uint32_t ta, int nvalid, int yl, flo
 
 template <bool kTauOne, bool kTF32>
 __device__ __forceinline__ void bwd_epilogue(const HeadParams& p, uint32_t base, uint32_t tmem,
-                                             int tt, int split, int warp, int lane,
+                                             int row_base, int split, int warp, int lane,
                                              volatile int* abort_flag) {
   constexpr int kElt = kTF32 ? 4 : 2;
   const int quad = warp & 3, half = warp >> 2;
-  const long long row = static_cast<long long>(tt) * kHeadBM + quad * 32 + lane;
+  const long long row = static_cast<long long>(row_base) + quad * 32 + lane;
   const bool row_ok = row < p.T;
   const int y = row_ok ? __ldg(p.y + row) : -1;
   const bool valid = row_ok && y >= 0 && y < p.V;
@@ -574,7 +584,7 @@ __device__ __forceinline__ void bwd_epilogue(const HeadParams& p, uint32_t base,
   const float bTt = -__ldg(p.stats + MT + static_cast<long long>(t) * p.T + rr) * L1;
   uint32_t nchunks = 0;
   const uint32_t stage = base + HeadSmem::kStage + static_cast<uint32_t>(warp) * 2 * kHeadStageChunk;
-  const int row0 = tt * kHeadBM + quad * 32;
+  const int row0 = row_base + quad * 32;
   const GOut oT{&p.mapG[t], stage, &nchunks, row0,
                 static_cast<char*>(p.G) + (static_cast<long long>(t) * p.g_model_stride + rr * p.g_pitch) * kElt,
                 row_ok};
@@ -643,7 +653,8 @@ __device__ __forceinline__ void bwd_epilogue(const HeadParams& p, uint32_t base,
 
 // ------------------------------------------------------------------ kernel
 template <int kMode, bool kTF32, bool kTauOne>
-__global__ void __launch_bounds__(kHeadThreads, 1) head_kernel(const __grid_constant__ HeadParams p) {
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kHeadThreads, 1)
+    head_kernel(const __grid_constant__ HeadParams p) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -652,8 +663,11 @@ __global__ void __launch_bounds__(kHeadThreads, 1) head_kernel(const __grid_cons
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + HeadSmem::kTmemSlot);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int tt = blockIdx.x % p.ntt;
-  const int split = blockIdx.x / p.ntt;
+  const uint32_t rank = cluster_ctarank();
+  const int pair = blockIdx.x >> 1;
+  const int tt = pair % p.ntt;
+  const int split = pair / p.ntt;
+  const int row_base = tt * 2 * kHeadBM + static_cast<int>(rank) * kHeadBM;  // this CTA's tokens
 
   if (threadIdx.x == 0) {
     *abort_flag = 0;
@@ -663,14 +677,14 @@ __global__ void __launch_bounds__(kHeadThreads, 1) head_kernel(const __grid_cons
     }
     for (uint32_t a = 0; a < 2; ++a) {
       mbar_init(HeadSmem::accf(base, a), 1);
-      mbar_init(HeadSmem::acce(base, a), kHeadEpiWarps);
+      mbar_init(HeadSmem::acce(base, a), 2 * kHeadEpiWarps);
     }
     mbar_init(HeadSmem::drain(base), 1);
     fence_barrier_init();
   }
   if (warp == kHeadEpiWarps + 1) {
-    tmem_alloc(base + HeadSmem::kTmemSlot, kTmemCols);
-    tmem_relinquish();
+    tmem_alloc_pair(base + HeadSmem::kTmemSlot, kTmemCols);
+    tmem_relinquish_pair();
   }
   if (warp == kHeadEpiWarps && lane == 0) {
     for (int m = 0; m < p.M; ++m) {
@@ -679,38 +693,38 @@ __global__ void __launch_bounds__(kHeadThreads, 1) head_kernel(const __grid_cons
     }
   }
   tc_fence_before();
-  __syncthreads();
+  cluster_sync();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
   if (warp >= kHeadEpiWarps) {
     regs_decrease<kHeadCtlRegs>();
     if (warp == kHeadEpiWarps) {
-      if (lane == 0) head_producer<kTF32>(p, base, tt, split, abort_flag);
+      if (lane == 0) head_producer<kTF32>(p, base, row_base, rank, split, abort_flag);
     } else if (warp == kHeadEpiWarps + 1) {
-      if (lane == 0) head_mma<kTF32>(p, base, tmem, split, abort_flag);
+      if (lane == 0 && rank == 0) head_mma<kTF32>(p, base, tmem, split, abort_flag);
       __syncwarp();
     }
   } else {
     regs_increase<kHeadEpiRegs>();
     if constexpr (kMode == kModeFwd)
-      fwd_epilogue<kTauOne>(p, base, tmem, reinterpret_cast<float*>(gbase + HeadSmem::kStage), tt,
-                            split, warp, lane, abort_flag);
+      fwd_epilogue<kTauOne>(p, base, tmem, reinterpret_cast<float*>(gbase + HeadSmem::kStage),
+                            row_base, split, warp, lane, abort_flag);
     else
-      bwd_epilogue<kTauOne, kTF32>(p, base, tmem, tt, split, warp, lane, abort_flag);
+      bwd_epilogue<kTauOne, kTF32>(p, base, tmem, row_base, split, warp, lane, abort_flag);
   }
 
   tc_fence_before();
-  __syncthreads();
+  cluster_sync();
   if (warp == kHeadEpiWarps + 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, kTmemCols);
+    tmem_dealloc_pair(tmem, kTmemCols);
   }
 }
 
 template <int kMode>
 cudaError_t launch_head(const HeadParams& p, bool tf32, bool tau_one, cudaStream_t s) {
-  const int grid = p.ntt * p.S;
+  const int grid = 2 * p.ntt * p.S;  // CTA pairs
   if (grid <= 0) return cudaSuccess;
   const dim3 g(grid), b(kHeadThreads);
   if (tf32) {
@@ -746,6 +760,19 @@ cudaError_t setup_mode() {
 }
 
 }  // namespace
+
+int head_max_active_pairs() {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2 * 1024);
+  cfg.blockDim = dim3(kHeadThreads);
+  cfg.dynamicSmemBytes = kHeadSmem;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, head_kernel<kModeFwd, false, true>, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  return n;
+}
 
 cudaError_t launch_head_fwd(const HeadParams& p, bool tf32, bool tau_one, cudaStream_t s) {
   return launch_head<kModeFwd>(p, tf32, tau_one, s);

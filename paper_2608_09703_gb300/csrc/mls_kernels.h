@@ -12,12 +12,14 @@ namespace mls {
 constexpr int kMaxModels = 4;
 
 // ------------------------------------------------------------------ head kernels
-// One CTA owns a tile of kHeadBM tokens and walks vocabulary tiles of kHeadBN
+// A CTA pair owns 2 x kHeadBM tokens and walks vocabulary tiles of kHeadBN
 // columns; for each vocabulary tile it computes the teacher's logit tile first
-// and then every student's, all into TMEM (double-buffered).
+// and then every student's, all into TMEM (double-buffered).  Each CTA holds
+// its kHeadBM token rows and kHeadBHalf vocabulary rows per stage.
 constexpr int kHeadBM = 128;
 constexpr int kHeadBN = 256;
-constexpr int kHeadStages = 4;
+constexpr int kHeadBHalf = 128;
+constexpr int kHeadStages = 6;
 constexpr int kHeadEpiWarps = 8;                       // warpgroups 0 and 1
 constexpr int kHeadThreads = (kHeadEpiWarps + 4) * 32;  // + warpgroup 2: TMA, MMA, 2 idle
 // Registers: launched at 168 per thread (384 x 168 = 64512), then the control
@@ -29,7 +31,7 @@ constexpr int kHeadCtlRegs = 40;
 static_assert(2 * 128 * kHeadEpiRegs + 128 * kHeadCtlRegs == kHeadThreads * kHeadLaunchRegs,
               "register reallocation must add up to the launch allocation");
 constexpr uint32_t kHeadABytes = kHeadBM * 128;
-constexpr uint32_t kHeadBBytes = kHeadBN * 128;
+constexpr uint32_t kHeadBBytes = kHeadBHalf * 128;
 // Backward: each epilogue warp stages its dL/dz chunks (32 tokens x 32 bf16
 // columns, 2 KB, 64B-swizzled) in two buffers and writes them with TMA stores.
 constexpr uint32_t kHeadStageChunk = 32 * 64;
@@ -48,7 +50,7 @@ struct HeadParams {
   int M;
   int order[kMaxModels];         // order[0] = teacher, then the students
   int nk[kMaxModels];            // k-blocks (128 bytes of K each) of model m
-  int ntt;                       // token tiles
+  int ntt;                       // token tiles of 2 * kHeadBM (one per CTA pair)
   int vt_begin, vt_end;          // vocabulary tiles handled by this launch
   int S;                         // CTAs per token tile (vocabulary splits)
   long long T, V;
@@ -72,15 +74,18 @@ struct HeadParams {
 };
 
 // ------------------------------------------------------------------ GEMM kernels
-constexpr int kGemmBM = 128;
-constexpr int kGemmBN = 256;
-constexpr int kGemmStages = 4;
+// CTA pairs: a pair owns a 256 x kGemmBN output tile; each CTA of the pair
+// holds 128 rows of A and kGemmBHalf rows of B per stage.
+constexpr int kGemmBM = 128;       // rows of A (and of C) per CTA
+constexpr int kGemmBN = 256;       // columns of C per pair tile
+constexpr int kGemmBHalf = 128;    // rows of B per CTA
+constexpr int kGemmStages = 6;
 constexpr int kGemmEpiWarps = 4;
 constexpr int kGemmThreads = (kGemmEpiWarps + 2) * 32;
 constexpr uint32_t kGemmABytes = kGemmBM * 128;
-constexpr uint32_t kGemmBBytes = kGemmBN * 128;
-// 32 KB of slack past the last stage keeps every operand read of an MN-major
-// descriptor inside the CTA's allocation.
+constexpr uint32_t kGemmBBytes = kGemmBHalf * 128;
+// 32 KB of slack past the last stage keeps every operand read of a descriptor
+// inside the CTA's allocation.
 constexpr uint32_t kGemmSmem = kGemmStages * (kGemmABytes + kGemmBBytes) + 1024 + 1024 + 32768;
 
 struct GemmProblem {
@@ -91,7 +96,7 @@ struct GemmProblem {
   long long ldc;
   int accumulate;                // C += A*B if 1, C = A*B if 0
   int tiles_n;                   // ceil(Ncols / kGemmBN)
-  int tile_begin;                // first linear tile of this problem
+  int tile_begin;                // first linear pair tile (256 x kGemmBN) of this problem
 };
 
 struct GemmParams {
@@ -141,5 +146,7 @@ cudaError_t launch_count(const int* y, long long T, long long V, float* inv_n, i
 // One-time per-device kernel attribute setup (dynamic shared memory limits).
 cudaError_t setup_head_kernels();
 cudaError_t setup_gemm_kernels();
+int gemm_max_active_pairs();  // 0 if the query failed
+int head_max_active_pairs();
 
 }  // namespace mls
