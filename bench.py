@@ -271,7 +271,7 @@ def gpu_arm(args, rank, world, local):
     wl = workload(args)
     H, W, y = synth.make_inputs(wl, seed=1234 + rank, device=dev)
     op = B.HeadLoss(wl.d, wl.T, wl.V, teacher=wl.teacher_index, tau=wl.tau, alpha=wl.alpha,
-                    w=wl.weights, dtype=torch.bfloat16, device=dev)
+                    w=wl.weights, dtype=torch.bfloat16, device=dev, vocab_group=args.vocab_group)
 
     def step():
         op.forward(H, W, y)
@@ -319,12 +319,15 @@ def gpu_arm(args, rank, world, local):
     launches, total_ms = kern[dom]
     flops_launch = (step_flops / 4) / (launches / args.steps)
     achieved = flops_launch / (total_ms / launches / 1e3) / 1e12
-    peak = float(pk["bf16_tflops"])
+    # The kernels are timed inside a loop of back-to-back steps, the regime in
+    # which the clock settles under the power cap: the sustained bf16 figure
+    # is the denominator; the burst figure is reported beside it.
+    peak = float(pk["bf16_tflops_sustained"])
+    burst = float(pk["bf16_tflops"])
     roofline = {"bound": "tensor", "kernel": dom, "achieved": achieved, "peak": peak,
-                "unit": "TFLOP/s", "frac": achieved / peak,
-                "frac_of_sustained": achieved / float(pk["bf16_tflops_sustained"]),
-                "peak_source": f"{pk_src} bf16 dense burst (MEASURED_PEAKS.json)" if pk_src == "measured"
-                else "fallback 1.9 PFLOP/s bf16",
+                "unit": "TFLOP/s", "frac": achieved / peak, "frac_of_burst": achieved / burst,
+                "peak_source": (f"{pk_src} bf16 dense sustained (MEASURED_PEAKS.json; burst {burst})"
+                                if pk_src == "measured" else "fallback 1.7 PFLOP/s bf16 sustained"),
                 "flops_per_launch": flops_launch,
                 "traffic": traffic_for(dom)}
     gpu_launches = sum(v[0] for v in kern.values())
@@ -349,7 +352,8 @@ def gpu_arm(args, rank, world, local):
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded N(0,1) hidden states, "
         "N(0,0.02^2) heads, uniform targets; FineWeb-Edu not available)",
         "config": workload_config(wl, world),
-        "tensor_frac_step": step_flops / (ms_max / 1e3) / 1e12 / peak,
+        "tensor_frac_step": step_flops / (ms_max / 1e3) / 1e12 / burst,
+        "tensor_frac_step_sustained": step_flops / (ms_max / 1e3) / 1e12 / peak,
         "roofline": roofline, "kernels": per_kernel, "gpu_launches": gpu_launches,
         "clocks": clocks, "e2e": e2e, "cpu_baseline": cpu,
     }
@@ -357,42 +361,74 @@ def gpu_arm(args, rank, world, local):
 
 
 def e2e_run(args, op, H, W, y, world, stream, wl):
+    """The same metric through the C ABI with the inputs in pinned host memory.
+
+    Every step copies its own H, W and targets host->device and reads its loss
+    back device->host inside the timed region.  The copies run on a second
+    stream into the other of two device buffers while the previous step
+    computes (a data pipeline's prefetch), so a step waits only for its own
+    inputs."""
     import torch
 
     from paper_2608_09703_gb300 import binding as B
 
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    dev = H[0].device
     Hh = [h.cpu().pin_memory() for h in H]
     Wh = [w.cpu().pin_memory() for w in W]
     yh = y.cpu().pin_memory()
-    loss_h = torch.empty(1, dtype=torch.float32).pin_memory()
-    Hd = [torch.empty_like(h) for h in H]
-    Wd = [torch.empty_like(w) for w in W]
-    yd = torch.empty_like(y)
-    h2d = sum(t.numel() * t.element_size() for t in Hh + Wh) + yh.numel() * yh.element_size()
-    d2h = loss_h.numel() * loss_h.element_size()
+    srcs = Hh + Wh + [yh]
+    bufs = [[torch.empty_like(t, device=dev) for t in srcs] for _ in range(2)]
+    n_e2e = max(3, min(args.steps, 10))
+    loss_h = torch.empty(n_e2e + 1, dtype=torch.float32).pin_memory()
+    h2d = sum(t.numel() * t.element_size() for t in srcs)
+    d2h = 4
+    copy_stream = torch.cuda.Stream(device=dev)
+    done = [torch.cuda.Event() for _ in range(2)]      # compute finished with buffer b
+    landed = [torch.cuda.Event() for _ in range(2)]    # inputs of buffer b copied
+    M = wl.M
 
-    def e2e_step():
-        for src, dst in zip(Hh + Wh + [yh], Hd + Wd + [yd]):
-            dst.copy_(src, non_blocking=True)
+    def copy_into(b):
+        with torch.cuda.stream(copy_stream):
+            copy_stream.wait_event(done[b])
+            for src, dst in zip(srcs, bufs[b]):
+                dst.copy_(src, non_blocking=True)
+            landed[b].record(copy_stream)
+
+    def compute(i, b):
+        stream.wait_event(landed[b])
+        Hd, Wd, yd = bufs[b][:M], bufs[b][M:2 * M], bufs[b][2 * M]
         op.forward(Hd, Wd, yd)
         op.backward(Hd, Wd, yd)
-        loss_h.copy_(op.loss, non_blocking=True)
+        loss_h[i].copy_(op.loss[0], non_blocking=True)
+        done[b].record(stream)
 
-    n_e2e = max(3, min(args.steps, 10))
-    e2e_step()
+    for b in range(2):
+        done[b].record(stream)
+    torch.cuda.synchronize()
+    # warm-up step (not timed)
+    copy_into(0)
+    compute(n_e2e, 0)
     torch.cuda.synchronize()
     barrier(world)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     t0 = time.perf_counter()
     e0.record(stream)
-    for _ in range(n_e2e):
-        e2e_step()
+    copy_stream.wait_event(e0)
+    copy_into(0)
+    for i in range(n_e2e):
+        if i + 1 < n_e2e:
+            copy_into((i + 1) % 2)
+        compute(i, i % 2)
     e1.record(stream)
     torch.cuda.synchronize()
-    e2e_ms = max(e0.elapsed_time(e1), (time.perf_counter() - t0) * 1e3) / n_e2e
+    host_ms = (time.perf_counter() - t0) * 1e3
+    e2e_ms = max(e0.elapsed_time(e1), host_ms) / n_e2e
     e2e_ms = max_over_ranks(e2e_ms, world)
+    assert torch.isfinite(loss_h).all()
     e2e = {"value": world * wl.T / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
-           "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms}
+           "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms,
+           "note": "inputs copied from pinned host memory every step, prefetched one step ahead "
+                   "on a copy stream; loss read back every step"}
     status = B.mls_get_status()
     if status:
         raise RuntimeError(f"device status: {B.mls_strerror(status)}")
@@ -410,6 +446,8 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--tokens", type=int, default=0, help="override T (profiling captures)")
     ap.add_argument("--vocab", type=int, default=0, help="override V (profiling captures)")
+    ap.add_argument("--vocab-group", type=int, default=0,
+                    help="backward vocabulary group in columns (0 = the library's choice)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

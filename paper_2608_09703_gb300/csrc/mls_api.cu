@@ -178,12 +178,12 @@ Plan make_plan(const mls_problem* p, int pairs) {
   pl.fwd_bytes = o;
 
   // Backward vocabulary groups: the bf16 (fp32) gradient of the logits of one
-  // group of columns for every sub-model stays within ~2 GiB unless the caller
+  // group of columns for every sub-model stays within ~4 GiB unless the caller
   // chose the group width.
   const long long vpad = static_cast<long long>(pl.nvt) * kHeadBN;
   long long gmax = p->vocab_group;
   if (gmax == 0) {
-    const long long budget = 2LL << 30;
+    const long long budget = 4LL << 30;
     const long long per_col = M * (T > 0 ? T : 1) * pl.elt;
     gmax = budget / per_col / kHeadBN * kHeadBN;
     if (gmax < 2048) gmax = 2048;
