@@ -157,9 +157,17 @@ def max_over_ranks(x: float, world: int) -> float:
     import torch
     import torch.distributed as dist
 
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def aggregate(ms_local: float, tokens_per_rank: int, world: int):
+    """Whole-job throughput: every rank processed its own batch; the job took
+    as long as the slowest rank.  Returns (ms of the slowest rank, tokens/s)."""
+    ms_max = max_over_ranks(ms_local, world)
+    return ms_max, world * tokens_per_rank / (ms_max / 1e3)
 
 
 # ------------------------------------------------------------------------- oracle timing
@@ -303,8 +311,7 @@ def gpu_arm(args, rank, world, local):
     clocks = sampler.stop()
     barrier(world)
     ms = e0.elapsed_time(e1) / args.steps
-    ms_max = max_over_ranks(ms, world)
-    value = world * wl.T / (ms_max / 1e3)
+    ms_max, value = aggregate(ms, wl.T, world)
 
     pk, pk_src = peaks()
     step_flops = wl.flops_fwd_bwd()
