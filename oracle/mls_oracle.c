@@ -428,3 +428,54 @@ int mls_oracle_threads(void) {
   return 1;
 #endif
 }
+
+/*
+ * Evaluation metrics between sub-models (Sec. 3.2.2: pairwise KL divergence
+ * and top-1 next-token agreement across the suite's sub-models; App. A plots
+ * KL(p_student || p_teacher)).  For every token and every ordered pair (i, j),
+ * with p = softmax(z) at temperature 1:
+ *   kl[(i*M + j)*T + t] = KL(p_i || p_j) = sum_v p_i[v] (log p_i[v] - log p_j[v])
+ *   agree[(i*M + j)*T + t] = 1 if argmax z_i == argmax z_j (lowest index on ties)
+ * The diagonal is 0 (kl) and 1 (agree).  tau, alpha, w and the teacher index
+ * of the problem are not used.
+ */
+int mls_oracle_pairwise(const mls_oracle_problem* p, const void* const* H, const void* const* W,
+                        double* kl, int* agree) {
+  if (check_problem(p) || !H || !W || !kl) return 1;
+  const int M = p->M;
+  const long long T = p->T, V = p->V;
+  int err = 0;
+#pragma omp parallel
+  {
+    double* buf = (double*)malloc(sizeof(double) * 2 * (size_t)M * (size_t)V);
+    if (!buf) {
+#pragma omp atomic write
+      err = 4;
+    }
+#pragma omp for schedule(dynamic, 1)
+    for (long long t = 0; t < T; ++t) {
+      if (!buf) continue;
+      double* logp[ORACLE_MAX_M];
+      int am[ORACLE_MAX_M];
+      for (int m = 0; m < M; ++m) {
+        double* z = buf + (size_t)m * V;
+        logits_row(p, H[m], W[m], p->d[m], t, z);
+        am[m] = argmax_lowest(z, V);
+        const double lse = logsumexp_scaled(z, V, 1.0);
+        logp[m] = buf + (size_t)(M + m) * V;
+        for (long long v = 0; v < V; ++v) logp[m][v] = z[v] - lse;
+      }
+      for (int i = 0; i < M; ++i) {
+        for (int j = 0; j < M; ++j) {
+          double k = 0.0;
+          if (i != j)
+            for (long long v = 0; v < V; ++v) k += exp(logp[i][v]) * (logp[i][v] - logp[j][v]);
+          kl[((long long)i * M + j) * T + t] = k;
+          if (agree) agree[((long long)i * M + j) * T + t] = am[i] == am[j];
+        }
+      }
+    }
+    free(buf);
+  }
+  return err;
+}

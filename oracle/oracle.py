@@ -69,6 +69,8 @@ def _load():
                                         ctypes.c_int, ctypes.c_longlong, ctypes.c_double,
                                         dp, dp, ip, dp, dpp]
         lib.mls_oracle_rows.restype = ctypes.c_int
+        lib.mls_oracle_pairwise.argtypes = [P, vpp, vpp, dp, ip]
+        lib.mls_oracle_pairwise.restype = ctypes.c_int
         lib.mls_oracle_threads.argtypes = []
         lib.mls_oracle_threads.restype = ctypes.c_int
         _lib = lib
@@ -185,3 +187,16 @@ def rows(H, W, y, rows_idx, teacher=None, tau=1.0, alpha=0.5, w=None, grad_scale
     if with_dh:
         out["dH"] = dH
     return out
+
+
+def pairwise(H, W) -> dict:
+    """Per-token KL(p_i || p_j) [M, M, T] and top-1 agreement [M, M, T] (fp64)."""
+    T = H[0].shape[0]
+    a = _Args(H, W, np.zeros(T, np.int32), len(H) - 1, 1.0, 0.0, None)
+    M = a.M
+    kl = np.zeros((M, M, T), np.float64)
+    agree = np.zeros((M, M, T), np.int32)
+    rc = _load().mls_oracle_pairwise(ctypes.byref(a.prob), a.Hp, a.Wp, _dp(kl),
+                                     agree.ctypes.data_as(ctypes.POINTER(ctypes.c_int)))
+    _check(rc, "mls_oracle_pairwise")
+    return {"kl": kl, "agree": agree}

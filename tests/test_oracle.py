@@ -357,3 +357,39 @@ def test_golden_regression_fixture():
     for m in range(3):
         np.testing.assert_allclose(dH[m], np.asarray(fx["dH"][m]), rtol=1e-11, atol=1e-15)
         np.testing.assert_allclose(dW[m], np.asarray(fx["dW"][m]), rtol=1e-11, atol=1e-15)
+
+
+# ---------------------------------------------------------------- evaluation metrics
+def test_pairwise_kl_pins():
+    """Pairwise KL(p_i || p_j) and top-1 agreement (Sec. 3.2.2): library KL on the
+    same logits, zero on the diagonal and for identical sub-models, >= 0, and a
+    two-token case by hand."""
+    T, d, V = 9, (8, 16, 12), 23
+    H, W, y = problem(T, d, V, seed=13, ws=0.5)
+    H = H + [H[1].copy()]
+    W = W + [W[1].copy()]            # sub-model 3 duplicates sub-model 1
+    out = orc.pairwise(H, W)
+    zs = logits(H, W)
+    lp = [torch.log_softmax(z, -1) for z in zs]
+    for i in range(4):
+        for j in range(4):
+            want = F.kl_div(lp[j], lp[i], reduction="none", log_target=True).sum(-1).numpy()
+            np.testing.assert_allclose(out["kl"][i, j], want, rtol=1e-11, atol=1e-14)
+            am_i, am_j = np.argmax(zs[i].numpy(), -1), np.argmax(zs[j].numpy(), -1)
+            np.testing.assert_array_equal(out["agree"][i, j], (am_i == am_j).astype(np.int32))
+    assert (out["kl"] >= -1e-14).all()
+    np.testing.assert_allclose(out["kl"][1, 3], 0.0, atol=1e-13)
+    np.testing.assert_array_equal(out["agree"][1, 3], 1)
+    for i in range(4):
+        assert (out["kl"][i, i] == 0).all()
+    # by hand: z_0 = (1, 0), z_1 = (0, 0): KL(p0||p1) = log 2 - H(sigmoid(1))
+    H2 = [np.array([[1.0]]), np.array([[1.0]])]
+    W2 = [np.array([[1.0], [0.0]]), np.array([[0.0], [0.0]])]
+    o2 = orc.pairwise(H2, W2)
+    s1 = sig(1.0)
+    h = -(s1 * math.log(s1) + (1 - s1) * math.log(1 - s1))
+    assert o2["kl"][0, 1, 0] == pytest.approx(math.log(2.0) - h, abs=1e-14)
+    # KL(p1||p0) = sum 0.5 (log 0.5 - log p0) = -log 2 - 0.5 (log s1 + log(1 - s1))
+    assert o2["kl"][1, 0, 0] == pytest.approx(-math.log(2.0) - 0.5 * (math.log(s1) + math.log(1 - s1)),
+                                              abs=1e-14)
+    assert o2["agree"][0, 1, 0] == 1  # argmax (1, 0) is 0; argmax (0, 0) is 0 (lowest index)
