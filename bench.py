@@ -339,6 +339,30 @@ def gpu_arm(args, rank, world, local):
                 "traffic": traffic_for(dom)}
     gpu_launches = sum(v[0] for v in kern.values())
 
+    # ---- evaluation metrics between sub-models (forward only), same inputs
+    pairwise = None
+    if not args.no_pairwise:
+        for _ in range(2):
+            op.pairwise(H, W, y)
+        torch.cuda.synchronize()
+        B.mls_profile_enable(True)
+        e0.record(stream)
+        n_pw = max(3, args.steps // 2)
+        for _ in range(n_pw):
+            op.pairwise(H, W, y)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        kp = B.mls_profile_read()
+        B.mls_profile_enable(False)
+        pw_ms = e0.elapsed_time(e1) / n_pw
+        k_launches, k_ms = kp["pairwise"]
+        k_tflops = (step_flops / 4) / (k_ms / k_launches / 1e3) / 1e12
+        pairwise = {"ms_per_call": pw_ms, "tokens_per_s": wl.T / (pw_ms / 1e3),
+                    "kernel_tflops": k_tflops, "kernel_frac_of_sustained": k_tflops / peak,
+                    "flops_per_call": step_flops / 4,
+                    "what": "per-token KL(p_i||p_j) for all ordered sub-model pairs, means and "
+                            "top-1 agreement (forward only)"}
+
     # ---- end to end through the C ABI with host buffers (pinned), copies timed
     e2e = None
     if not args.no_e2e:
@@ -362,7 +386,7 @@ def gpu_arm(args, rank, world, local):
         "tensor_frac_step": step_flops / (ms_max / 1e3) / 1e12 / burst,
         "tensor_frac_step_sustained": step_flops / (ms_max / 1e3) / 1e12 / peak,
         "roofline": roofline, "kernels": per_kernel, "gpu_launches": gpu_launches,
-        "clocks": clocks, "e2e": e2e, "cpu_baseline": cpu,
+        "clocks": clocks, "e2e": e2e, "cpu_baseline": cpu, "pairwise_eval": pairwise,
     }
     print(json.dumps(line), flush=True)
 
@@ -451,6 +475,7 @@ def main():
     ap.add_argument("--workload", default=WORKLOAD)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-pairwise", action="store_true")
     ap.add_argument("--tokens", type=int, default=0, help="override T (profiling captures)")
     ap.add_argument("--vocab", type=int, default=0, help="override V (profiling captures)")
     ap.add_argument("--vocab-group", type=int, default=0,

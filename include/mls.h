@@ -77,8 +77,8 @@ typedef struct {
 } mls_problem;
 
 /*
- * Bytes of device workspace that mls_head_loss_fwd and mls_head_loss_bwd need
- * for this problem (the larger of the two).  Returns 0 if the problem is
+ * Bytes of device workspace that mls_head_loss_fwd, mls_head_loss_bwd and
+ * mls_head_pairwise need for this problem (the largest of the three).  Returns 0 if the problem is
  * invalid.  The backward keeps the gradient of the logits for one vocabulary
  * group, bf16 [M, T, group] (fp32 for MLS_FP32 inputs), in this workspace.
  */
@@ -114,6 +114,23 @@ int mls_head_loss_bwd(const mls_problem* p, const void* const* H, const void* co
                       const int32_t* targets, const float* stats, float grad_scale,
                       float* const* dH, float* const* dW, void* ws, size_t ws_bytes,
                       mls_stream_t stream);
+
+/*
+ * Evaluation metrics between sub-models (Sec. 3.2.2: pairwise KL divergence
+ * and top-1 next-token agreement across the suite; App. A plots
+ * KL(p_student || p_teacher)).  Forward only, softmax at temperature 1; tau,
+ * alpha, w and the teacher index of `p` are not used.
+ *   targets    device, int32 [T] or NULL: tokens with a target outside [0, V)
+ *              are left out of the means (NULL: every token counts)
+ *   tok_kl     device, fp32 [M, M, T]: KL(p_i || p_j) per token (diagonal 0)
+ *   argmax     device, int32 [M, T] or NULL
+ *   pair_stats device, fp32 [2, M, M]: mean KL(p_i || p_j) and the fraction of
+ *              tokens on which argmax z_i == argmax z_j
+ *   ws         device workspace, ws_bytes >= mls_workspace_size(p)
+ */
+int mls_head_pairwise(const mls_problem* p, const void* const* H, const void* const* W,
+                      const int32_t* targets, float* tok_kl, int32_t* argmax, float* pair_stats,
+                      void* ws, size_t ws_bytes, mls_stream_t stream);
 
 /*
  * Synchronises `stream`, then returns the status bits (MLS_STATUS_*) recorded by

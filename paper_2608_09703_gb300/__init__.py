@@ -12,6 +12,7 @@ from .binding import (  # noqa: F401
     mls_get_status,
     mls_head_loss_bwd,
     mls_head_loss_fwd,
+    mls_head_pairwise,
     mls_strerror,
     mls_workspace_size,
 )

@@ -75,6 +75,8 @@ def lib():
         L.mls_get_status.restype = ctypes.c_int
         L.mls_strerror.argtypes = [ctypes.c_int]
         L.mls_strerror.restype = ctypes.c_char_p
+        L.mls_head_pairwise.argtypes = [P, vpp, vpp, vp, vp, vp, vp, vp, ctypes.c_size_t, vp]
+        L.mls_head_pairwise.restype = ctypes.c_int
         L.mls_head_loss_fwd_noalloc.argtypes = [P, vpp, vpp, vp, vp, vp, vp, vp, vp, vp]
         L.mls_head_loss_fwd_noalloc.restype = ctypes.c_int
         L.mls_profile_enable.argtypes = [ctypes.c_int]
@@ -144,6 +146,15 @@ def mls_head_loss_bwd(prob: Problem, H, W, targets, stats, grad_scale: float, dH
                                  float(grad_scale), _ptrs(dH), _ptrs(dW), _ptr(ws), ws_bytes,
                                  _stream(stream))
     _check(rc, "mls_head_loss_bwd")
+
+
+def mls_head_pairwise(prob: Problem, H, W, targets, tok_kl, argmax, pair_stats, ws,
+                      stream=None) -> None:
+    """Per-token KL(p_i || p_j) between sub-models, their means and top-1 agreement."""
+    ws_bytes = 0 if ws is None else ws.numel() * ws.element_size()
+    rc = lib().mls_head_pairwise(prob.ref(), _ptrs(H), _ptrs(W), _ptr(targets), _ptr(tok_kl),
+                                 _ptr(argmax), _ptr(pair_stats), _ptr(ws), ws_bytes, _stream(stream))
+    _check(rc, "mls_head_pairwise")
 
 
 def mls_head_loss_fwd_noalloc(prob: Problem, H, W, targets, loss, tok_loss, tok_diag, argmax,
@@ -216,6 +227,18 @@ class HeadLoss:
         mls_head_loss_fwd(self.prob, H, W, targets, self.loss, self.tok_loss, self.tok_diag,
                           self.argmax, self.stats, self.ws, stream)
         return self.loss
+
+    def pairwise(self, H, W, targets=None, stream=None):
+        """Evaluation metrics between sub-models; returns (tok_kl [M,M,T],
+        argmax [M,T], pair_stats [2,M,M])."""
+        dev = self.loss.device
+        if not hasattr(self, "tok_kl"):
+            self.tok_kl = torch.empty(self.M, self.M, self.T, dtype=torch.float32, device=dev)
+            self.pair_stats = torch.empty(2, self.M, self.M, dtype=torch.float32, device=dev)
+            self.eval_argmax = torch.empty(self.M, self.T, dtype=torch.int32, device=dev)
+        mls_head_pairwise(self.prob, H, W, targets, self.tok_kl, self.eval_argmax, self.pair_stats,
+                          self.ws, stream)
+        return self.tok_kl, self.eval_argmax, self.pair_stats
 
     def backward(self, H, W, targets, grad_scale=1.0, stream=None):
         mls_head_loss_bwd(self.prob, H, W, targets, self.stats, grad_scale, self.dH, self.dW,

@@ -66,6 +66,8 @@ int device_state(DeviceState** out) {
       s.err = fail(MLS_ERR_CUDA, "head kernel attributes", e);
     } else if ((e = setup_gemm_kernels()) != cudaSuccess) {
       s.err = fail(MLS_ERR_CUDA, "gemm kernel attributes", e);
+    } else if ((e = setup_eval_kernels()) != cudaSuccess) {
+      s.err = fail(MLS_ERR_CUDA, "eval kernel attributes", e);
     } else if ((s.gemm_pairs = gemm_max_active_pairs()) <= 0) {
       s.err = fail(MLS_ERR_CUDA, "gemm cluster occupancy");
     } else if ((s.head_pairs = head_max_active_pairs()) <= 0) {
@@ -113,6 +115,9 @@ struct Plan {
   // W_m^T [d_m][v_pitch] for the tf32 GEMMs
   long long t_pitch = 0, v_pitch = 0;
   size_t off_GT = 0, off_HT[kMaxModels] = {}, off_WT[kMaxModels] = {};
+  // pairwise evaluation
+  int eval_nvt = 0, eval_S = 1;
+  size_t off_epart = 0, off_eacc = 0, off_ecnt = 0, eval_bytes = 0;
   size_t total = 0;
 };
 
@@ -210,7 +215,20 @@ Plan make_plan(const mls_problem* p, int pairs) {
     }
   }
   pl.bwd_bytes = o;
+
+  pl.eval_nvt = static_cast<int>(ceil_div(V, kEvalBN));
+  pl.eval_S = choose_splits(pl.ntt, pl.eval_nvt, pairs);
+  o = 0;
+  pl.off_epart = o;
+  o = align_up(o + sizeof(float) * static_cast<size_t>(pl.eval_S) * kEvalFields * T);
+  pl.off_eacc = o;
+  o = align_up(o + sizeof(double) * 2 * kMaxModels * kMaxModels * static_cast<size_t>(pl.merge_blocks + 1));
+  pl.off_ecnt = o;
+  o = align_up(o + sizeof(long long) * static_cast<size_t>(pl.merge_blocks + 1));
+  pl.eval_bytes = o;
+
   pl.total = pl.fwd_bytes > pl.bwd_bytes ? pl.fwd_bytes : pl.bwd_bytes;
+  if (pl.eval_bytes > pl.total) pl.total = pl.eval_bytes;
   return pl;
 }
 
@@ -678,5 +696,64 @@ extern "C" int mls_head_loss_fwd_noalloc(const mls_problem* p, const void* const
   if ((rc = timed("merge", s, [&] { return launch_merge(mp, pl.merge_blocks, s); }))) return rc;
   return timed("final", s, [&] {
     return launch_final(mp.block_sum, mp.block_cnt, pl.merge_blocks, loss, s);
+  });
+}
+
+extern "C" int mls_head_pairwise(const mls_problem* p, const void* const* H, const void* const* W,
+                                 const int32_t* targets, float* tok_kl, int32_t* argmax,
+                                 float* pair_stats, void* ws, size_t ws_bytes, mls_stream_t stream) {
+  int rc = validate(p);
+  if (rc) return rc;
+  if (!H || !W || !pair_stats || (p->T > 0 && !tok_kl)) return MLS_ERR_ARG;
+  for (int m = 0; m < p->M; ++m) {
+    if (!H[m] || !W[m]) return MLS_ERR_ARG;
+    if (!aligned16(H[m]) || !aligned16(W[m])) return MLS_ERR_ALIGN;
+  }
+  DeviceState* dev = nullptr;
+  if ((rc = device_state(&dev))) return rc;
+  const Plan pl = make_plan(p, dev->head_pairs);
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (p->T == 0)
+    return launch_ok(cudaMemsetAsync(pair_stats, 0, sizeof(float) * 2 * p->M * p->M, s));
+  if ((rc = check_ws(pl, ws, ws_bytes, pl.total))) return rc;
+  char* wsb = static_cast<char*>(ws);
+
+  EvalParams ep;
+  std::memset(&ep, 0, sizeof ep);
+  const int KE = 128 / pl.elt;
+  for (int m = 0; m < p->M; ++m) {
+    if (encode(&ep.mapH[m], H[m], pl.elt, p->d[m], p->T, p->d[m], KE, kHeadBM) ||
+        encode(&ep.mapW[m], W[m], pl.elt, p->d[m], p->V, p->d[m], KE, kEvalBHalf))
+      return MLS_ERR_CUDA;
+    ep.nk[m] = static_cast<int>(ceil_div(p->d[m], KE));
+  }
+  ep.M = p->M;
+  ep.ntt = pl.ntt;
+  ep.nvt = pl.eval_nvt;
+  ep.S = pl.eval_S;
+  ep.T = p->T;
+  ep.V = p->V;
+  ep.L1 = 1.4426950408889634f;
+  ep.status = dev->status;
+  ep.part = reinterpret_cast<float*>(wsb + pl.off_epart);
+  if ((rc = timed("pairwise", s, [&] { return launch_eval(ep, pl.elt == 4, s); }))) return rc;
+
+  EvalMergeParams mp;
+  std::memset(&mp, 0, sizeof mp);
+  mp.part = ep.part;
+  mp.nparts = ep.S;
+  mp.M = p->M;
+  mp.T = p->T;
+  mp.V = p->V;
+  mp.y = targets;
+  mp.tok_kl = tok_kl;
+  mp.argmax = argmax;
+  mp.block_acc = reinterpret_cast<double*>(wsb + pl.off_eacc);
+  mp.block_cnt = reinterpret_cast<long long*>(wsb + pl.off_ecnt);
+  mp.status = dev->status;
+  if ((rc = timed("pairwise_merge", s, [&] { return launch_eval_merge(mp, pl.merge_blocks, s); })))
+    return rc;
+  return timed("pairwise_final", s, [&] {
+    return launch_eval_final(mp.block_acc, mp.block_cnt, pl.merge_blocks, p->M, pair_stats, s);
   });
 }

@@ -108,6 +108,47 @@ struct GemmParams {
   int* status;
 };
 
+// ------------------------------------------------------------------ pairwise evaluation
+// Forward-only evaluation metrics between sub-models.  A CTA pair owns 256
+// tokens; for every 128-column vocabulary tile it computes the logit tiles of
+// all M <= 4 sub-models into TMEM at once (M x 128 columns) and accumulates,
+// for every ordered pair (s, j), D_sj = sum_v exp(z_s[v] - max_s) (z_s[v] - z_j[v]).
+constexpr int kEvalBN = 128;     // vocabulary columns per tile
+constexpr int kEvalBHalf = 64;   // rows of W per CTA
+constexpr int kEvalStages = 8;
+constexpr uint32_t kEvalABytes = kHeadBM * 128;
+constexpr uint32_t kEvalBBytes = kEvalBHalf * 128;
+// per token and split: max_s (4), sum_s (4), argmax_s (4), D_sj for j != s (4 x 3)
+constexpr int kEvalFields = 24;
+constexpr uint32_t kEvalXchg = kEvalFields * kHeadBM * 4;
+constexpr uint32_t kEvalSmem = kEvalStages * (kEvalABytes + kEvalBBytes) + kEvalXchg + 1024 + 1024;
+
+struct EvalParams {
+  CUtensorMap mapH[kMaxModels];  // H_m [T, d_m], box {128 B of K, kHeadBM rows}
+  CUtensorMap mapW[kMaxModels];  // W_m [V, d_m], box {128 B of K, kEvalBHalf rows}
+  int M;
+  int nk[kMaxModels];
+  int ntt;                       // token tiles of 256 (one per CTA pair)
+  int nvt;                       // vocabulary tiles of kEvalBN
+  int S;                         // CTA pairs per token tile
+  long long T, V;
+  float L1;
+  int* status;
+  float* part;                   // [S][kEvalFields][T]
+};
+
+struct EvalMergeParams {
+  const float* part;
+  int nparts, M;
+  long long T, V;
+  const int* y;                  // may be null: every token counts
+  float* tok_kl;                 // [M][M][T]
+  int* argmax;                   // [M][T] or null
+  double* block_acc;             // [blocks][2][M*M]: sums of KL and of agreement
+  long long* block_cnt;          // [blocks]
+  int* status;
+};
+
 // ------------------------------------------------------------------ reductions
 struct MergeParams {
   const float* part;             // [nparts][kPartFields][M][T]
@@ -142,6 +183,12 @@ cudaError_t launch_final(const double* block_sum, const long long* block_cnt, in
                          float* loss, cudaStream_t s);
 cudaError_t launch_count(const int* y, long long T, long long V, float* inv_n, int* status,
                          cudaStream_t s);
+
+cudaError_t launch_eval(const EvalParams& p, bool tf32, cudaStream_t s);
+cudaError_t launch_eval_merge(const EvalMergeParams& p, int blocks, cudaStream_t s);
+cudaError_t launch_eval_final(const double* block_acc, const long long* block_cnt, int nblocks,
+                              int M, float* pair_stats, cudaStream_t s);
+cudaError_t setup_eval_kernels();
 
 // One-time per-device kernel attribute setup (dynamic shared memory limits).
 cudaError_t setup_head_kernels();
