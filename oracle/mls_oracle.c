@@ -479,3 +479,72 @@ int mls_oracle_pairwise(const mls_oracle_problem* p, const void* const* H, const
   }
   return err;
 }
+
+/*
+ * Inter-model junction (Eq. 1).  Per token t, with o = o^m[t] (D_m values) the
+ * output of sub-model m and e = e^{m+1}[t] (D_{m+1} - D_m values) the fresh
+ * embedding of sub-model m+1:
+ *   o~ = o * ||e||_2 / ||o||_2          (o~ = 0 when ||o|| = 0)
+ *   x  = concat(o~, e)                  embed_first = 0: the first D_m channels
+ *                                       carry sub-model m (the reading of the prose)
+ *   x  = concat(e, o~)                  embed_first = 1: Eq. 1's written order
+ * Storage types as for the heads (in_dtype 0 bf16 bits, 1 fp32, 2 fp64); the
+ * output x is double.  The backward takes g = dL/dx and returns
+ *   dL/do = s (g_o - o (g_o . o) / ||o||^2),  dL/de = g_e + s (g_o . o) e / ||e||^2,
+ * with s = ||e|| / ||o|| (both 0 when ||o|| = 0; the e term is 0 when ||e|| = 0),
+ * written out from the chain rule of o~ = o ||e|| / ||o||.
+ */
+static double row_norm(const void* a, int dtype, long long t, int n) {
+  double s = 0.0;
+  for (int k = 0; k < n; ++k) {
+    const double v = elem(a, dtype, t * n + k);
+    s += v * v;
+  }
+  return sqrt(s);
+}
+
+int mls_oracle_junction_fwd(long long T, int d_prev, int d_next, int dtype, int embed_first,
+                            const void* o, const void* e, double* x) {
+  const int de = d_next - d_prev;
+  if (T < 0 || d_prev < 1 || de < 1 || dtype < 0 || dtype > 2 || !o || !e || !x) return 1;
+#pragma omp parallel for schedule(static)
+  for (long long t = 0; t < T; ++t) {
+    const double no = row_norm(o, dtype, t, d_prev), ne = row_norm(e, dtype, t, de);
+    const double s = no > 0.0 ? ne / no : 0.0;
+    double* xr = x + t * d_next;
+    const int oo = embed_first ? de : 0, eo = embed_first ? 0 : d_prev;
+    for (int k = 0; k < d_prev; ++k) xr[oo + k] = elem(o, dtype, t * d_prev + k) * s;
+    for (int k = 0; k < de; ++k) xr[eo + k] = elem(e, dtype, t * de + k);
+  }
+  return 0;
+}
+
+int mls_oracle_junction_bwd(long long T, int d_prev, int d_next, int dtype, int embed_first,
+                            const void* o, const void* e, const void* g, double* d_o, double* d_e) {
+  const int de = d_next - d_prev;
+  if (T < 0 || d_prev < 1 || de < 1 || dtype < 0 || dtype > 2 || !o || !e || !g || !d_o || !d_e)
+    return 1;
+#pragma omp parallel for schedule(static)
+  for (long long t = 0; t < T; ++t) {
+    const double no = row_norm(o, dtype, t, d_prev), ne = row_norm(e, dtype, t, de);
+    const int oo = embed_first ? de : 0, eo = embed_first ? 0 : d_prev;
+    double go_dot_o = 0.0;
+    for (int k = 0; k < d_prev; ++k)
+      go_dot_o += elem(g, dtype, t * d_next + oo + k) * elem(o, dtype, t * d_prev + k);
+    if (no > 0.0) {
+      const double s = ne / no;
+      for (int k = 0; k < d_prev; ++k)
+        d_o[t * d_prev + k] = s * (elem(g, dtype, t * d_next + oo + k) -
+                                   elem(o, dtype, t * d_prev + k) * go_dot_o / (no * no));
+      for (int k = 0; k < de; ++k) {
+        const double ge = elem(g, dtype, t * d_next + eo + k);
+        const double ek = elem(e, dtype, t * de + k);
+        d_e[t * de + k] = ge + (ne > 0.0 ? s * go_dot_o * ek / (ne * ne) : 0.0);
+      }
+    } else {
+      for (int k = 0; k < d_prev; ++k) d_o[t * d_prev + k] = 0.0;
+      for (int k = 0; k < de; ++k) d_e[t * de + k] = elem(g, dtype, t * d_next + eo + k);
+    }
+  }
+  return 0;
+}

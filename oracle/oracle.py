@@ -71,6 +71,14 @@ def _load():
         lib.mls_oracle_rows.restype = ctypes.c_int
         lib.mls_oracle_pairwise.argtypes = [P, vpp, vpp, dp, ip]
         lib.mls_oracle_pairwise.restype = ctypes.c_int
+        lib.mls_oracle_junction_fwd.argtypes = [ctypes.c_longlong, ctypes.c_int, ctypes.c_int,
+                                                ctypes.c_int, ctypes.c_int, ctypes.c_void_p,
+                                                ctypes.c_void_p, dp]
+        lib.mls_oracle_junction_fwd.restype = ctypes.c_int
+        lib.mls_oracle_junction_bwd.argtypes = [ctypes.c_longlong, ctypes.c_int, ctypes.c_int,
+                                                ctypes.c_int, ctypes.c_int, ctypes.c_void_p,
+                                                ctypes.c_void_p, ctypes.c_void_p, dp, dp]
+        lib.mls_oracle_junction_bwd.restype = ctypes.c_int
         lib.mls_oracle_threads.argtypes = []
         lib.mls_oracle_threads.restype = ctypes.c_int
         _lib = lib
@@ -200,3 +208,31 @@ def pairwise(H, W) -> dict:
                                      agree.ctypes.data_as(ctypes.POINTER(ctypes.c_int)))
     _check(rc, "mls_oracle_pairwise")
     return {"kl": kl, "agree": agree}
+
+
+def junction_fwd(o, e, embed_first=False):
+    """Eq. 1: x = concat(o * ||e|| / ||o||, e) per row (or concat(e, ...) with
+    embed_first); o [T, D_m], e [T, D_{m+1} - D_m] -> x [T, D_{m+1}] fp64."""
+    (o, dt), (e, dt2) = _as_input(o), _as_input(e)
+    assert dt == dt2
+    T, dp_ = o.shape
+    de = e.shape[1]
+    x = np.zeros((T, dp_ + de), np.float64)
+    rc = _load().mls_oracle_junction_fwd(T, dp_, dp_ + de, dt, int(embed_first), o.ctypes.data,
+                                         e.ctypes.data, _dp(x))
+    _check(rc, "mls_oracle_junction_fwd")
+    return x
+
+
+def junction_bwd(o, e, g, embed_first=False):
+    """Gradients (dL/do, dL/de) of the junction for upstream g = dL/dx (fp64)."""
+    (o, dt), (e, _), (g, dt3) = _as_input(o), _as_input(e), _as_input(g)
+    assert dt == dt3
+    T, dp_ = o.shape
+    de = e.shape[1]
+    d_o = np.zeros((T, dp_), np.float64)
+    d_e = np.zeros((T, de), np.float64)
+    rc = _load().mls_oracle_junction_bwd(T, dp_, dp_ + de, dt, int(embed_first), o.ctypes.data,
+                                         e.ctypes.data, g.ctypes.data, _dp(d_o), _dp(d_e))
+    _check(rc, "mls_oracle_junction_bwd")
+    return d_o, d_e

@@ -393,3 +393,52 @@ def test_pairwise_kl_pins():
     assert o2["kl"][1, 0, 0] == pytest.approx(-math.log(2.0) - 0.5 * (math.log(s1) + math.log(1 - s1)),
                                               abs=1e-14)
     assert o2["agree"][0, 1, 0] == 1  # argmax (1, 0) is 0; argmax (0, 0) is 0 (lowest index)
+
+
+# ---------------------------------------------------------------- junction (Eq. 1)
+@pytest.mark.parametrize("embed_first", [False, True])
+def test_junction_pins(embed_first):
+    """The rescaled part has the fresh embedding's norm and o's direction, the
+    embedding is copied unchanged, a hand-worked row, and central finite
+    differences of a random linear functional of x."""
+    rng = np.random.default_rng(14)
+    T, dp_, de = 6, 5, 3
+    o = rng.standard_normal((T, dp_)) * 3.0
+    e = rng.standard_normal((T, de)) * 0.1
+    o[4] = 0.0  # zero row: o~ = 0
+    x = orc.junction_fwd(o, e, embed_first)
+    ot = x[:, de:] if embed_first else x[:, :dp_]
+    ee = x[:, :de] if embed_first else x[:, dp_:]
+    np.testing.assert_array_equal(ee, e)
+    nrm = np.linalg.norm(ot, axis=1)
+    for t in range(T):
+        if t == 4:
+            assert np.abs(ot[t]).max() == 0.0
+            continue
+        assert nrm[t] == pytest.approx(np.linalg.norm(e[t]), rel=1e-13)
+        np.testing.assert_allclose(ot[t] / nrm[t], o[t] / np.linalg.norm(o[t]), rtol=1e-12)
+    # by hand: o = (3, 4) (norm 5), e = (0, 6) (norm 6): o~ = (3.6, 4.8)
+    xh = orc.junction_fwd(np.array([[3.0, 4.0]]), np.array([[0.0, 6.0]]), embed_first)
+    want = [0.0, 6.0, 3.6, 4.8] if embed_first else [3.6, 4.8, 0.0, 6.0]
+    np.testing.assert_allclose(xh[0], want, rtol=1e-15)
+    # finite differences of f(o, e) = sum(c * x)
+    c = rng.standard_normal((T, dp_ + de))
+    d_o, d_e = orc.junction_bwd(o, e, c, embed_first)
+    eps = 1e-6
+    for arr, grad in ((o, d_o), (e, d_e)):
+        fd = np.zeros_like(arr)
+        for idx in np.ndindex(*arr.shape):
+            if arr is o and idx[0] == 4:
+                continue  # the zero row sits on the kink of ||o||
+            vals = []
+            for sgn in (1, -1):
+                a2 = arr.copy()
+                a2[idx] += sgn * eps
+                xo = orc.junction_fwd(a2, e, embed_first) if arr is o else \
+                    orc.junction_fwd(o, a2, embed_first)
+                vals.append((c * xo).sum())
+            fd[idx] = (vals[0] - vals[1]) / (2 * eps)
+        mask = np.ones(arr.shape[0], bool)
+        if arr is o:
+            mask[4] = False
+        np.testing.assert_allclose(grad[mask], fd[mask], rtol=1e-6, atol=1e-8)
