@@ -197,10 +197,12 @@ def oracle_rate(wl, budget_s: float, seed: int = 1234):
     from oracle import oracle
 
     oracle.build()
-    Hs, Ws, ys = oracle_sample(wl, 2, seed)
+    # the oracle runs one token per thread: calibrate with one token per thread
+    ncal = max(2, oracle.threads())
+    Hs, Ws, ys = oracle_sample(wl, ncal, seed)
     t0 = time.perf_counter()
     oracle_step(wl, Hs, Ws, ys)
-    per_tok = (time.perf_counter() - t0) / 2
+    per_tok = (time.perf_counter() - t0) / ncal
     ntok = int(max(2, min(wl.T, budget_s / max(per_tok, 1e-6))))
     Hs, Ws, ys = oracle_sample(wl, ntok, seed)
     t0 = time.perf_counter()
@@ -218,10 +220,11 @@ def reference_arm(args, rank, world):
     wl = workload(args)
     oracle.build()
     # size each step so that warmup + steps fit in about three minutes
-    Hs, Ws, ys = oracle_sample(wl, 2)
+    ncal = max(2, oracle.threads())
+    Hs, Ws, ys = oracle_sample(wl, ncal)
     t0 = time.perf_counter()
     oracle_step(wl, Hs, Ws, ys)
-    per_tok = (time.perf_counter() - t0) / 2
+    per_tok = (time.perf_counter() - t0) / ncal
     per_step_budget = max(1.0, 180.0 / (args.steps + args.warmup))
     ntok = int(max(1, min(wl.T, per_step_budget / max(per_tok, 1e-6))))
     Hs, Ws, ys = oracle_sample(wl, ntok)
@@ -363,6 +366,11 @@ def gpu_arm(args, rank, world, local):
                     "what": "per-token KL(p_i||p_j) for all ordered sub-model pairs, means and "
                             "top-1 agreement (forward only)"}
 
+    # ---- inter-model junctions (Eq. 1) of the suite, forward + backward
+    junction = None
+    if not args.no_junction:
+        junction = junction_run(args, wl, dev, float(pk["hbm_gbs"]))
+
     # ---- end to end through the C ABI with host buffers (pinned), copies timed
     e2e = None
     if not args.no_e2e:
@@ -387,8 +395,57 @@ def gpu_arm(args, rank, world, local):
         "tensor_frac_step_sustained": step_flops / (ms_max / 1e3) / 1e12 / peak,
         "roofline": roofline, "kernels": per_kernel, "gpu_launches": gpu_launches,
         "clocks": clocks, "e2e": e2e, "cpu_baseline": cpu, "pairwise_eval": pairwise,
+        "junction": junction,
     }
     print(json.dumps(line), flush=True)
+
+
+def junction_run(args, wl, dev, hbm_gbs):
+    """Forward + backward of every junction m -> m+1 of the suite on T tokens,
+    bf16, timed with CUDA events.  Algorithmic bytes per junction: forward
+    reads o and e and writes x (2 * T * D_{m+1} elements), backward reads g, o,
+    e and writes dL/do, dL/de (3 * T * D_{m+1} elements)."""
+    import torch
+
+    from paper_2608_09703_gb300 import binding as B
+
+    g = torch.Generator(device=dev)
+    g.manual_seed(99)
+    bufs = []
+    nbytes = 0
+    for m in range(wl.M - 1):
+        dp, dn = wl.d[m], wl.d[m + 1]
+        mk = lambda *sh: torch.randn(*sh, generator=g, device=dev).to(torch.bfloat16)
+        o, e, gr = mk(wl.T, dp), mk(wl.T, dn - dp), mk(wl.T, dn)
+        x, d_o, d_e = torch.empty_like(gr), torch.empty_like(o), torch.empty_like(e)
+        bufs.append((o, e, gr, x, d_o, d_e))
+        nbytes += 5 * wl.T * dn * 2
+
+    def run():
+        for o, e, gr, x, d_o, d_e in bufs:
+            B.mls_junction_fwd(o, e, x)
+            B.mls_junction_bwd(o, e, gr, d_o, d_e)
+
+    for _ in range(3):
+        run()
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    n = max(5, args.steps)
+    B.mls_profile_enable(True)
+    e0.record(stream)
+    for _ in range(n):
+        run()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    kp = B.mls_profile_read()
+    B.mls_profile_enable(False)
+    ms = e0.elapsed_time(e1) / n
+    kern_ms = sum(v[1] for k, v in kp.items() if k.startswith("junction")) / n
+    gbs = nbytes / (kern_ms / 1e3) / 1e9
+    return {"junctions": wl.M - 1, "ms_per_fwd_bwd": ms, "kernel_ms": kern_ms,
+            "bytes": nbytes, "achieved_gbs": gbs, "peak_gbs": hbm_gbs, "frac": gbs / hbm_gbs,
+            "bound": "hbm"}
 
 
 def e2e_run(args, op, H, W, y, world, stream, wl):
@@ -476,6 +533,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-pairwise", action="store_true")
+    ap.add_argument("--no-junction", action="store_true")
     ap.add_argument("--tokens", type=int, default=0, help="override T (profiling captures)")
     ap.add_argument("--vocab", type=int, default=0, help="override V (profiling captures)")
     ap.add_argument("--vocab-group", type=int, default=0,

@@ -133,6 +133,29 @@ int mls_head_pairwise(const mls_problem* p, const void* const* H, const void* co
                       void* ws, size_t ws_bytes, mls_stream_t stream);
 
 /*
+ * Inter-model junction (Eq. 1) between sub-model m (width D_m = d_prev) and
+ * sub-model m+1 (width D_{m+1} = d_next), per token:
+ *   o~ = o * ||e||_2 / ||o||_2   (o~ = 0 when ||o|| = 0)
+ *   x  = concat(o~, e)  if embed_first == 0  (the prose: the first D_m channels
+ *                                             carry sub-model m)
+ *   x  = concat(e, o~)  if embed_first != 0  (Eq. 1's written order)
+ *   o  device [T, d_prev], e device [T, d_next - d_prev], x device [T, d_next],
+ *   all row-major in in_dtype (MLS_BF16 or MLS_FP32), 16-byte aligned, rows a
+ *   multiple of 16 bytes; sums are fp32.
+ * Backward: g = dL/dx [T, d_next]; d_o [T, d_prev] and d_e [T, d_next - d_prev]
+ * are overwritten (same storage type) with
+ *   dL/do = s (g_o - o (g_o . o) / ||o||^2),  dL/de = g_e + s (g_o . o) e / ||e||^2,
+ *   s = ||e|| / ||o||  (both terms 0 when ||o|| = 0).
+ * Asynchronous on `stream`; returns 0 or a negative MLS_ERR_* code.
+ */
+int mls_junction_fwd(int64_t T, int32_t d_prev, int32_t d_next, int32_t in_dtype,
+                     int32_t embed_first, const void* o, const void* e, void* x,
+                     mls_stream_t stream);
+int mls_junction_bwd(int64_t T, int32_t d_prev, int32_t d_next, int32_t in_dtype,
+                     int32_t embed_first, const void* o, const void* e, const void* g,
+                     void* d_o, void* d_e, mls_stream_t stream);
+
+/*
  * Synchronises `stream`, then returns the status bits (MLS_STATUS_*) recorded by
  * the device on the current device since the last call and clears them; returns
  * a negative MLS_ERR_CUDA if the synchronisation or the read failed.

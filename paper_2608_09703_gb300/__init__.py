@@ -13,6 +13,8 @@ from .binding import (  # noqa: F401
     mls_head_loss_bwd,
     mls_head_loss_fwd,
     mls_head_pairwise,
+    mls_junction_bwd,
+    mls_junction_fwd,
     mls_strerror,
     mls_workspace_size,
 )

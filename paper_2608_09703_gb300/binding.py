@@ -77,6 +77,11 @@ def lib():
         L.mls_strerror.restype = ctypes.c_char_p
         L.mls_head_pairwise.argtypes = [P, vpp, vpp, vp, vp, vp, vp, vp, ctypes.c_size_t, vp]
         L.mls_head_pairwise.restype = ctypes.c_int
+        i64, i32 = ctypes.c_int64, ctypes.c_int32
+        L.mls_junction_fwd.argtypes = [i64, i32, i32, i32, i32, vp, vp, vp, vp]
+        L.mls_junction_fwd.restype = ctypes.c_int
+        L.mls_junction_bwd.argtypes = [i64, i32, i32, i32, i32, vp, vp, vp, vp, vp, vp]
+        L.mls_junction_bwd.restype = ctypes.c_int
         L.mls_head_loss_fwd_noalloc.argtypes = [P, vpp, vpp, vp, vp, vp, vp, vp, vp, vp]
         L.mls_head_loss_fwd_noalloc.restype = ctypes.c_int
         L.mls_profile_enable.argtypes = [ctypes.c_int]
@@ -155,6 +160,29 @@ def mls_head_pairwise(prob: Problem, H, W, targets, tok_kl, argmax, pair_stats, 
     rc = lib().mls_head_pairwise(prob.ref(), _ptrs(H), _ptrs(W), _ptr(targets), _ptr(tok_kl),
                                  _ptr(argmax), _ptr(pair_stats), _ptr(ws), ws_bytes, _stream(stream))
     _check(rc, "mls_head_pairwise")
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return MLS_BF16
+    if t.dtype == torch.float32:
+        return MLS_FP32
+    raise TypeError(t.dtype)
+
+
+def mls_junction_fwd(o, e, x, embed_first=False, stream=None) -> None:
+    """Eq. 1: x = concat(o * ||e|| / ||o||, e) per row (concat(e, ...) if embed_first)."""
+    T, dp = o.shape
+    rc = lib().mls_junction_fwd(T, dp, dp + e.shape[1], _dtype_code(o), int(bool(embed_first)),
+                                _ptr(o), _ptr(e), _ptr(x), _stream(stream))
+    _check(rc, "mls_junction_fwd")
+
+
+def mls_junction_bwd(o, e, g, d_o, d_e, embed_first=False, stream=None) -> None:
+    T, dp = o.shape
+    rc = lib().mls_junction_bwd(T, dp, dp + e.shape[1], _dtype_code(o), int(bool(embed_first)),
+                                _ptr(o), _ptr(e), _ptr(g), _ptr(d_o), _ptr(d_e), _stream(stream))
+    _check(rc, "mls_junction_bwd")
 
 
 def mls_head_loss_fwd_noalloc(prob: Problem, H, W, targets, loss, tok_loss, tok_diag, argmax,

@@ -19,7 +19,8 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libmls.so")
-SOURCES = ["mls_api.cu", "mls_head.cu", "mls_gemm.cu", "mls_reduce.cu", "mls_eval.cu"]
+SOURCES = ["mls_api.cu", "mls_head.cu", "mls_gemm.cu", "mls_reduce.cu", "mls_eval.cu",
+           "mls_junction.cu"]
 HEADERS = ["mls_device.cuh", "mls_kernels.h"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

@@ -757,3 +757,44 @@ extern "C" int mls_head_pairwise(const mls_problem* p, const void* const* H, con
     return launch_eval_final(mp.block_acc, mp.block_cnt, pl.merge_blocks, p->M, pair_stats, s);
   });
 }
+
+namespace {
+int junction_check(long long T, int d_prev, int d_next, int dtype, const void* const* ptrs, int n) {
+  if (T < 0 || T > INT_MAX || d_prev < 1 || d_next <= d_prev) return MLS_ERR_ARG;
+  if (dtype != MLS_BF16 && dtype != MLS_FP32) return MLS_ERR_ARG;
+  const int elt = dtype == MLS_BF16 ? 2 : 4;
+  if ((static_cast<long long>(d_prev) * elt) % 16 || (static_cast<long long>(d_next) * elt) % 16)
+    return MLS_ERR_UNSUPPORTED;
+  for (int i = 0; i < n; ++i) {
+    if (T > 0 && !ptrs[i]) return MLS_ERR_ARG;
+    if (!aligned16(ptrs[i])) return MLS_ERR_ALIGN;
+  }
+  return MLS_OK;
+}
+}  // namespace
+
+extern "C" int mls_junction_fwd(int64_t T, int32_t d_prev, int32_t d_next, int32_t in_dtype,
+                                int32_t embed_first, const void* o, const void* e, void* x,
+                                mls_stream_t stream) {
+  const void* ptrs[3] = {o, e, x};
+  int rc = junction_check(T, d_prev, d_next, in_dtype, ptrs, 3);
+  if (rc) return rc;
+  DeviceState* dev = nullptr;
+  if ((rc = device_state(&dev))) return rc;
+  JunctionParams jp{T, d_prev, d_next, embed_first ? 1 : 0, o, e, x, nullptr, nullptr, nullptr};
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  return timed("junction_fwd", s, [&] { return launch_junction_fwd(jp, in_dtype == MLS_FP32, s); });
+}
+
+extern "C" int mls_junction_bwd(int64_t T, int32_t d_prev, int32_t d_next, int32_t in_dtype,
+                                int32_t embed_first, const void* o, const void* e, const void* g,
+                                void* d_o, void* d_e, mls_stream_t stream) {
+  const void* ptrs[5] = {o, e, g, d_o, d_e};
+  int rc = junction_check(T, d_prev, d_next, in_dtype, ptrs, 5);
+  if (rc) return rc;
+  DeviceState* dev = nullptr;
+  if ((rc = device_state(&dev))) return rc;
+  JunctionParams jp{T, d_prev, d_next, embed_first ? 1 : 0, o, e, nullptr, g, d_o, d_e};
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  return timed("junction_bwd", s, [&] { return launch_junction_bwd(jp, in_dtype == MLS_FP32, s); });
+}

@@ -149,6 +149,21 @@ struct EvalMergeParams {
   int* status;
 };
 
+// ------------------------------------------------------------------ junction (Eq. 1)
+struct JunctionParams {
+  long long T;
+  int d_prev, d_next;            // D_m and D_{m+1}
+  int embed_first;               // 0: x = [o~, e]; 1: x = [e, o~]
+  const void* o;                 // [T, D_m]
+  const void* e;                 // [T, D_{m+1} - D_m]
+  void* x;                       // [T, D_{m+1}] (forward)
+  const void* g;                 // [T, D_{m+1}] (backward)
+  void* d_o;                     // [T, D_m] (backward)
+  void* d_e;                     // [T, D_{m+1} - D_m] (backward)
+};
+cudaError_t launch_junction_fwd(const JunctionParams& p, bool fp32, cudaStream_t s);
+cudaError_t launch_junction_bwd(const JunctionParams& p, bool fp32, cudaStream_t s);
+
 // ------------------------------------------------------------------ reductions
 struct MergeParams {
   const float* part;             // [nparts][kPartFields][M][T]
