@@ -272,6 +272,10 @@ void fill_head_common(HeadParams& hp, const mls_problem* p, const Plan& pl, cons
   hp.Ltau = static_cast<float>(1.4426950408889634 / static_cast<double>(p->tau));
   hp.y = y;
   hp.status = status;
+  // Failure-detection test hook: with MLS_TEST_STALL_FIRST_STAGE set, the first
+  // CTA pair of a head kernel skips its first stage so that a bounded pipeline
+  // wait runs out and the call reports MLS_STATUS_TIMEOUT.
+  hp.test_stall = std::getenv("MLS_TEST_STALL_FIRST_STAGE") != nullptr ? 1 : 0;
 }
 
 int encode_head_maps(HeadParams& hp, const mls_problem* p, const Plan& pl, const void* const* H,

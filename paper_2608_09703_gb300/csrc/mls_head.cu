@@ -78,6 +78,9 @@ __device__ __forceinline__ void head_producer(const HeadParams& p, uint32_t base
   int stage = 0;
   uint32_t phase = 0, filled = 0, lastpar = 0;
   bool ok = true;
+  // Test hook (off unless the host sets it): the first pair issues nothing for
+  // its first stage, so the MMA issuer's wait on that stage must run out.
+  bool stall = p.test_stall && (blockIdx.x >> 1) == 0;
   for (int vt = p.vt_begin + split; ok && vt < p.vt_end; vt += p.S) {
     for (int u = 0; ok && u < p.M; ++u) {
       const int m = p.order[u];
@@ -85,6 +88,14 @@ __device__ __forceinline__ void head_producer(const HeadParams& p, uint32_t base
         if (!mbar_wait(HeadSmem::empty(base, stage), phase ^ 1u, abort_flag, p.status)) {
           ok = false;
           break;
+        }
+        if (stall) {
+          stall = false;
+          if (++stage == kHeadStages) {
+            stage = 0;
+            phase ^= 1u;
+          }
+          continue;
         }
         // both CTAs' halves are counted on the even CTA's barrier
         if (rank == 0) mbar_arrive_expect_tx(HeadSmem::full(base, stage), 2 * (kHeadABytes + kHeadBBytes));

@@ -58,6 +58,7 @@ struct HeadParams {
   float Ltau;                    // log2(e) / tau
   const int* y;                  // targets [T]
   int* status;
+  int test_stall;                // test hook: see head_producer (0 in normal use)
   // forward
   float* part;                   // [S][kPartFields][M][T]
   // backward
