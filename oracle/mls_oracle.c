@@ -548,3 +548,136 @@ int mls_oracle_junction_bwd(long long T, int d_prev, int d_next, int dtype, int 
   }
   return 0;
 }
+
+/*
+ * Speculative-decoding verify step for a nested draft / verifier pair
+ * (Sec. 2 "Speculative Decoding", Sec. 3.2.3: greedy and nucleus p = 0.9,
+ * temperature 0.4), written from the standard speculative sampling rule.
+ * Sequence b has gamma drafted tokens x_i, draft logits zd_i (i < gamma) and
+ * verifier logits zv_i (i <= gamma), both materialised from hidden states and
+ * heads.  For sampling, a distribution is nucleus(softmax(z / temperature)):
+ * tokens sorted by probability (descending, then by index) are kept up to and
+ * including the first one at which the cumulative probability reaches top_p,
+ * then renormalised.  With q_i (draft) and p_i (verifier):
+ *   x_i is accepted iff q_i(x_i) > 0 and u[b,i,0] * q_i(x_i) < p_i(x_i);
+ *   at the first rejection k: next = sample(norm(max(0, p_k - q_k)), u[b,k,1])
+ *     (sample(p_k, u[b,k,1]) if that is all zero);
+ *   if all gamma are accepted: next = sample(p_gamma, u[b,gamma,1]);
+ *   sample(r, u) = the smallest index v with sum_{w<=v} r_w > u * sum_w r_w.
+ * Greedy: x_i is accepted iff x_i == argmax zv_i (lowest index on ties) and
+ * next = argmax zv_k at the first rejection (or at gamma).
+ * u is [B][gamma+1][2].  Outputs n_accepted[b] and next_token[b].
+ */
+static void logits_of(const void* H, const void* W, int d, long long V, int dtype, long long row,
+                      double* z) {
+  for (long long v = 0; v < V; ++v) {
+    double acc = 0.0;
+    for (int k = 0; k < d; ++k) acc += elem(H, dtype, row * d + k) * elem(W, dtype, v * d + k);
+    z[v] = acc;
+  }
+}
+
+static double* g_sort_p;  /* comparator context (single-threaded use) */
+static int by_prob_then_index(const void* a, const void* b) {
+  const long long i = *(const long long*)a, j = *(const long long*)b;
+  if (g_sort_p[i] > g_sort_p[j]) return -1;
+  if (g_sort_p[i] < g_sort_p[j]) return 1;
+  return (i > j) - (i < j);
+}
+
+/* p <- nucleus(softmax(z / temperature)); order is scratch of V indices */
+static void nucleus_probs(const double* z, long long V, double temperature, double top_p, double* p,
+                          long long* order) {
+  double mx = -INFINITY;
+  for (long long v = 0; v < V; ++v)
+    if (z[v] > mx) mx = z[v];
+  double s = 0.0;
+  for (long long v = 0; v < V; ++v) s += exp((z[v] - mx) / temperature);
+  for (long long v = 0; v < V; ++v) p[v] = exp((z[v] - mx) / temperature) / s;
+  for (long long v = 0; v < V; ++v) order[v] = v;
+  g_sort_p = p;
+  qsort(order, (size_t)V, sizeof(long long), by_prob_then_index);
+  double cum = 0.0, kept = 0.0;
+  long long k = 0;
+  while (k < V) {
+    cum += p[order[k]];
+    ++k;
+    if (cum >= top_p) break;
+  }
+  for (long long i = 0; i < k; ++i) kept += p[order[i]];
+  for (long long i = k; i < V; ++i) p[order[i]] = 0.0;
+  for (long long i = 0; i < k; ++i) p[order[i]] /= kept;
+}
+
+static long long sample_index(const double* r, long long V, double u) {
+  double tot = 0.0;
+  for (long long v = 0; v < V; ++v) tot += r[v];
+  double cum = 0.0;
+  for (long long v = 0; v < V; ++v) {
+    cum += r[v];
+    if (cum > u * tot) return v;
+  }
+  return V - 1;
+}
+
+int mls_oracle_spec_verify(int B, int gamma, long long V, int d_draft, int d_verify, int dtype,
+                           double temperature, double top_p, int greedy, const void* Hd,
+                           const void* Wd, const void* Hv, const void* Wv, const int* draft,
+                           const double* u, int* n_accepted, int* next_token) {
+  if (B < 0 || gamma < 0 || V < 1 || d_draft < 1 || d_verify < 1 || !(temperature > 0.0) ||
+      !(top_p > 0.0 && top_p <= 1.0) || dtype < 0 || dtype > 2)
+    return 1;
+  double* zd = (double*)malloc(sizeof(double) * (size_t)V * 4);
+  long long* order = (long long*)malloc(sizeof(long long) * (size_t)V);
+  if (!zd || !order) {
+    free(zd);
+    free(order);
+    return 4;
+  }
+  double *zv = zd + V, *q = zd + 2 * V, *p = zd + 3 * V;
+  for (int b = 0; b < B; ++b) {
+    int k = 0, next = -1;
+    for (; k < gamma; ++k) {
+      const long long pos_d = (long long)b * gamma + k, pos_v = (long long)b * (gamma + 1) + k;
+      const int x = draft[pos_d];
+      logits_of(Hv, Wv, d_verify, V, dtype, pos_v, zv);
+      if (greedy) {
+        const int best = argmax_lowest(zv, V);
+        if (x != best) {
+          next = best;
+          break;
+        }
+        continue;
+      }
+      logits_of(Hd, Wd, d_draft, V, dtype, pos_d, zd);
+      nucleus_probs(zd, V, temperature, top_p, q, order);
+      nucleus_probs(zv, V, temperature, top_p, p, order);
+      const double uacc = u[((long long)b * (gamma + 1) + k) * 2 + 0];
+      const int ok = x >= 0 && x < V && q[x] > 0.0 && uacc * q[x] < p[x];
+      if (!ok) {
+        double any = 0.0;
+        for (long long v = 0; v < V; ++v) {
+          q[v] = p[v] - q[v] > 0.0 ? p[v] - q[v] : 0.0;
+          any += q[v];
+        }
+        next = (int)sample_index(any > 0.0 ? q : p, V, u[((long long)b * (gamma + 1) + k) * 2 + 1]);
+        break;
+      }
+    }
+    if (next < 0) {
+      const long long pos_v = (long long)b * (gamma + 1) + gamma;
+      logits_of(Hv, Wv, d_verify, V, dtype, pos_v, zv);
+      if (greedy) {
+        next = argmax_lowest(zv, V);
+      } else {
+        nucleus_probs(zv, V, temperature, top_p, p, order);
+        next = (int)sample_index(p, V, u[((long long)b * (gamma + 1) + gamma) * 2 + 1]);
+      }
+    }
+    n_accepted[b] = k;
+    next_token[b] = next;
+  }
+  free(zd);
+  free(order);
+  return 0;
+}

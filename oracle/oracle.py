@@ -79,6 +79,12 @@ def _load():
                                                 ctypes.c_int, ctypes.c_int, ctypes.c_void_p,
                                                 ctypes.c_void_p, ctypes.c_void_p, dp, dp]
         lib.mls_oracle_junction_bwd.restype = ctypes.c_int
+        lib.mls_oracle_spec_verify.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_longlong,
+                                               ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                               ctypes.c_double, ctypes.c_double, ctypes.c_int,
+                                               ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
+                                               ctypes.c_void_p, ip, dp, ip, ip]
+        lib.mls_oracle_spec_verify.restype = ctypes.c_int
         lib.mls_oracle_threads.argtypes = []
         lib.mls_oracle_threads.restype = ctypes.c_int
         _lib = lib
@@ -236,3 +242,25 @@ def junction_bwd(o, e, g, embed_first=False):
                                          e.ctypes.data, g.ctypes.data, _dp(d_o), _dp(d_e))
     _check(rc, "mls_oracle_junction_bwd")
     return d_o, d_e
+
+
+def spec_verify(Hd, Wd, Hv, Wv, draft, u, temperature=0.4, top_p=0.9, greedy=False):
+    """Speculative-decoding verify step (fp64): Hd [B*gamma, d_d], Hv [B*(gamma+1), d_v],
+    heads Wd [V, d_d], Wv [V, d_v], draft tokens [B, gamma], uniforms u [B, gamma+1, 2].
+    Returns (n_accepted [B], next_token [B])."""
+    (Hd, dt), (Wd, _), (Hv, _), (Wv, _) = (_as_input(a) for a in (Hd, Wd, Hv, Wv))
+    draft = np.ascontiguousarray(np.asarray(draft, np.int32))
+    B, gamma = draft.shape
+    u = np.ascontiguousarray(np.asarray(u, np.float64))
+    assert u.shape == (B, gamma + 1, 2)
+    V = Wv.shape[0]
+    n = np.zeros(B, np.int32)
+    nxt = np.zeros(B, np.int32)
+    ip_ = ctypes.POINTER(ctypes.c_int)
+    rc = _load().mls_oracle_spec_verify(B, gamma, V, Wd.shape[1], Wv.shape[1], dt, float(temperature),
+                                        float(top_p), int(bool(greedy)), Hd.ctypes.data,
+                                        Wd.ctypes.data, Hv.ctypes.data, Wv.ctypes.data,
+                                        draft.ctypes.data_as(ip_), _dp(u), n.ctypes.data_as(ip_),
+                                        nxt.ctypes.data_as(ip_))
+    _check(rc, "mls_oracle_spec_verify")
+    return n, nxt

@@ -442,3 +442,82 @@ def test_junction_pins(embed_first):
         if arr is o:
             mask[4] = False
         np.testing.assert_allclose(grad[mask], fd[mask], rtol=1e-6, atol=1e-8)
+
+
+# ---------------------------------------------------------------- speculative decoding verify
+def _onehot_rows(idx, d):
+    H = np.zeros((len(idx), d))
+    H[np.arange(len(idx)), idx] = 1.0
+    return H
+
+
+def test_spec_verify_greedy_by_construction():
+    """Greedy: one-hot hidden rows pick head columns, so the verifier's argmax at
+    every position is known; the draft agrees on the first two positions only."""
+    V, d, gamma = 6, 4, 3
+    Wv = np.zeros((V, d))
+    Wv[[2, 4, 1, 5], [0, 1, 2, 3]] = 1.0          # hidden unit k -> token (2, 4, 1, 5)[k]
+    Wd = Wv.copy()
+    Hv = _onehot_rows([0, 1, 2, 3], d)              # verifier argmax per position: 2, 4, 1, 5
+    Hd = _onehot_rows([0, 1, 2], d)
+    u = np.full((1, gamma + 1, 2), 0.5)
+    n, nxt = orc.spec_verify(Hd, Wd, Hv, Wv, [[2, 4, 0]], u, greedy=True)
+    assert (n[0], nxt[0]) == (2, 1)
+    n, nxt = orc.spec_verify(Hd, Wd, Hv, Wv, [[2, 4, 1]], u, greedy=True)
+    assert (n[0], nxt[0]) == (3, 5)                   # all accepted: bonus token
+
+
+def test_spec_verify_identical_models_accept_everything():
+    rng = np.random.default_rng(15)
+    B, gamma, V, d = 5, 4, 30, 8
+    W = rng.standard_normal((V, d))
+    Hv = rng.standard_normal((B * (gamma + 1), d))
+    Hd = np.concatenate([Hv.reshape(B, gamma + 1, d)[:, :gamma]]).reshape(B * gamma, d)
+    draft = rng.integers(0, 3, (B, gamma))
+    u = rng.random((B, gamma + 1, 2))
+    # a draft token outside the nucleus has q = 0 and is rejected; keep top_p = 1
+    n, _ = orc.spec_verify(Hd, W, Hv, W, draft, u, temperature=0.4, top_p=1.0)
+    assert (n == gamma).all()
+
+
+def test_spec_verify_nucleus_limits_and_hand_resample():
+    # top_p -> 0 keeps only the most likely token: sampling returns the argmax
+    V, d = 5, 5
+    Wv = np.eye(V) * np.array([1.0, 3.0, 2.0, 0.5, 2.9])[:, None]
+    Hv = np.ones((1, d))
+    u = np.array([[[0.3, 0.99]]])
+    n, nxt = orc.spec_verify(np.zeros((0, d)), Wv, Hv, Wv, np.zeros((1, 0), np.int32), u,
+                             temperature=1.0, top_p=1e-9)
+    assert (n[0], nxt[0]) == (0, 1)
+    # V = 2 by hand: q = (0.8, 0.2), p = (0.5, 0.5) at temperature 1, top_p = 1.
+    # draft x = 0: accept iff u * 0.8 < 0.5, i.e. u < 0.625; residual max(0, p - q) = (0, 0.3)
+    lq, lp = np.log([0.8, 0.2]), np.log([0.5, 0.5])
+    Wd2, Wv2 = np.diag(lq), np.diag(lp)
+    Hd2, Hv2 = np.ones((1, 2)), np.ones((2, 2))
+    for uacc, want_n in ((0.6, 1), (0.65, 0)):
+        uu = np.array([[[uacc, 0.1], [0.0, 0.7]]])
+        n, nxt = orc.spec_verify(Hd2, Wd2, Hv2, Wv2, [[0]], uu, temperature=1.0, top_p=1.0)
+        assert n[0] == want_n
+        if want_n == 0:
+            assert nxt[0] == 1                          # the residual puts all mass on token 1
+        else:
+            assert nxt[0] == 1                          # bonus from p = (0.5, 0.5) with u = 0.7
+
+
+def test_spec_verify_output_follows_the_verifier():
+    """The defining property of speculative sampling: with the draft token drawn
+    from q, the first emitted token is distributed as p (Monte Carlo)."""
+    rng = np.random.default_rng(16)
+    V, d, N = 6, 6, 20000
+    zq = np.array([1.0, 0.2, -0.5, 0.9, 0.0, -1.0])
+    zp = np.array([0.1, 1.1, -0.2, 0.6, 0.4, -0.8])
+    Wd, Wv = np.diag(zq), np.diag(zp)
+    q = np.exp(zq / 0.4) / np.exp(zq / 0.4).sum()
+    p = np.exp(zp / 0.4) / np.exp(zp / 0.4).sum()
+    draft = rng.choice(V, size=(N, 1), p=q)
+    u = rng.random((N, 2, 2))
+    Hd, Hv = np.ones((N, d)), np.ones((2 * N, d))
+    n, nxt = orc.spec_verify(Hd, Wd, Hv, Wv, draft, u, temperature=0.4, top_p=1.0)
+    first = np.where(n == 1, draft[:, 0], nxt)
+    freq = np.bincount(first, minlength=V) / N
+    assert np.abs(freq - p).max() < 4.5 * np.sqrt(p * (1 - p) / N).max()
