@@ -371,6 +371,11 @@ def gpu_arm(args, rank, world, local):
     if not args.no_junction:
         junction = junction_run(args, wl, dev, float(pk["hbm_gbs"]))
 
+    # ---- speculative-decoding verify step (draft 1024 / verifier 3072 of the suite)
+    spec = None
+    if not args.no_spec:
+        spec = spec_run(args, dev, pk)
+
     # ---- end to end through the C ABI with host buffers (pinned), copies timed
     e2e = None
     if not args.no_e2e:
@@ -395,7 +400,7 @@ def gpu_arm(args, rank, world, local):
         "tensor_frac_step_sustained": step_flops / (ms_max / 1e3) / 1e12 / peak,
         "roofline": roofline, "kernels": per_kernel, "gpu_launches": gpu_launches,
         "clocks": clocks, "e2e": e2e, "cpu_baseline": cpu, "pairwise_eval": pairwise,
-        "junction": junction,
+        "junction": junction, "spec_verify": spec,
     }
     print(json.dumps(line), flush=True)
 
@@ -523,6 +528,59 @@ def e2e_run(args, op, H, W, y, world, stream, wl):
     return e2e
 
 
+def spec_run(args, dev, pk):
+    """The speculative-decoding verify step on the suite's draft / verifier pair
+    at the paper's batch (102 sequences, draft length 6, V = 50304), bf16,
+    nucleus sampling (T = 0.4, p = 0.9) and greedy, timed with CUDA events.
+    The logits GEMM is 2 V (B gamma d_draft + B (gamma + 1) d_verify) FLOPs; the
+    selection kernels are reported against one read of every logits row."""
+    import torch
+
+    from paper_2608_09703_gb300 import binding as B
+    from paper_2608_09703_gb300 import synth
+
+    wl = synth.SPEC_WORKLOADS["spec_suite3"]
+    Hd, Wd, Hv, Wv = synth.make_spec_inputs(wl, 7, device=dev)
+    u = synth.make_uniforms(wl.B, wl.gamma, 7, device=dev)
+    g = torch.Generator(device=dev)
+    g.manual_seed(8)
+    draft = torch.randint(0, wl.V, (wl.B, wl.gamma), generator=g, device=dev, dtype=torch.int32)
+    Pd, Pv = wl.B * wl.gamma, wl.B * (wl.gamma + 1)
+    flops = 2 * wl.V * (Pd * wl.d_draft + Pv * wl.d_verify)
+    stream = torch.cuda.current_stream()
+    out = {"config": {"B": wl.B, "gamma": wl.gamma, "V": wl.V, "d_draft": wl.d_draft,
+                      "d_verify": wl.d_verify, "temperature": wl.temperature, "top_p": wl.top_p}}
+    for mode, greedy in (("nucleus", False), ("greedy", True)):
+        op = B.SpecVerify(wl.B, wl.gamma, wl.V, wl.d_draft, wl.d_verify, wl.temperature,
+                          wl.top_p, greedy, dtype=torch.bfloat16, device=dev)
+        for _ in range(3):
+            op(Hd, Wd, Hv, Wv, draft, u)
+        torch.cuda.synchronize()
+        n = max(5, args.steps // 2)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        B.mls_profile_enable(True)
+        e0.record(stream)
+        for _ in range(n):
+            op(Hd, Wd, Hv, Wv, draft, u)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        kp = B.mls_profile_read()
+        B.mls_profile_enable(False)
+        ms = e0.elapsed_time(e1) / n
+        gemm_ms = kp["spec_logits"][1] / n
+        f = flops if not greedy else 2 * wl.V * Pv * wl.d_verify
+        rows = (Pv if greedy else Pv + Pd)
+        sel_ms = kp["spec_position"][1] / n
+        out[mode] = {
+            "ms_per_call": ms, "positions_per_s": Pv / (ms / 1e3),
+            "kernel_ms": {k: v[1] / n for k, v in kp.items()},
+            "logits_tflops": f / (gemm_ms / 1e3) / 1e12,
+            "logits_frac_of_sustained": f / (gemm_ms / 1e3) / 1e12 / float(pk["bf16_tflops_sustained"]),
+            "selection_gbs_one_read": rows * wl.V * 4 / (sel_ms / 1e3) / 1e9,
+        }
+    return out
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -534,6 +592,7 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-pairwise", action="store_true")
     ap.add_argument("--no-junction", action="store_true")
+    ap.add_argument("--no-spec", action="store_true")
     ap.add_argument("--tokens", type=int, default=0, help="override T (profiling captures)")
     ap.add_argument("--vocab", type=int, default=0, help="override V (profiling captures)")
     ap.add_argument("--vocab-group", type=int, default=0,

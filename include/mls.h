@@ -156,6 +156,60 @@ int mls_junction_bwd(int64_t T, int32_t d_prev, int32_t d_next, int32_t in_dtype
                      void* d_o, void* d_e, mls_stream_t stream);
 
 /*
+ * Speculative-decoding verify step for a nested draft / verifier pair
+ * (Sec. 2, "Speculative Decoding": sub-model m drafts gamma tokens, a larger
+ * sub-model m' verifies them in one pass; Sec. 3.2.3 samples with temperature
+ * 0.4 and nucleus p = 0.9, or greedily).  Standard speculative sampling over
+ * B independent sequences; position i of sequence b is row b*gamma + i of
+ * H_draft and row b*(gamma+1) + i of H_verify.
+ *   q_i = nucleus(softmax(H_draft[i] W_draft^T / temperature))     i < gamma
+ *   p_i = nucleus(softmax(H_verify[i] W_verify^T / temperature))   i <= gamma
+ *   nucleus(r): tokens ordered by probability (descending, then by index) are
+ *   kept through the first one at which the cumulative probability reaches
+ *   top_p, then renormalised (top_p = 1 keeps every token).
+ *   Drafted token x_i is accepted iff q_i(x_i) > 0 and u[b,i,0] q_i(x_i) < p_i(x_i);
+ *   n_accepted[b] = k, the number accepted before the first rejection, and
+ *   next_token[b] = sample(max(0, p_k - q_k), u[b,k,1]) (sample(p_k, u[b,k,1])
+ *   when that residual is all zero), or sample(p_gamma, u[b,gamma,1]) when all
+ *   gamma were accepted, with sample(r, u) = the smallest v such that
+ *   sum_{w <= v} r_w > u * sum_w r_w.
+ *   greedy != 0: x_i is accepted iff it is the argmax of the verifier's
+ *   logits (lowest index on ties) and next_token is that argmax at position k;
+ *   the draft model, temperature, top_p and uniforms are not used (H_draft,
+ *   W_draft and uniforms may be NULL).
+ * Arguments (device pointers unless stated):
+ *   p            host; d_draft/d_verify: widths; in_dtype: storage of H and W
+ *   H_draft      [B*gamma, d_draft], W_draft [V, d_draft]      (in_dtype)
+ *   H_verify     [B*(gamma+1), d_verify], W_verify [V, d_verify]
+ *   draft_tokens int32 [B, gamma]; a token outside [0, V) is rejected
+ *   uniforms     fp32 [B, gamma+1, 2] in [0, 1): acceptance and sampling draws
+ *   n_accepted   int32 [B] (written), next_token int32 [B] (written)
+ *   ws           workspace of mls_spec_workspace_size(p) bytes, 256-byte aligned;
+ *                it holds the fp32 logits of every verify position.
+ * Logits are fp32 sums of the stored-type products; probabilities are fp32, so a
+ * decision that the exact values leave within rounding of a threshold may go
+ * either way.  Asynchronous; returns 0 or a negative MLS_ERR_* code (nothing
+ * launched).  B = 0 is a no-op.
+ */
+typedef struct {
+  int32_t B;            /* sequences, >= 0 */
+  int32_t gamma;        /* drafted tokens per sequence, >= 0 */
+  int64_t V;            /* vocabulary, 1 .. 2^31 - 1 */
+  int32_t d_draft;      /* width of the draft sub-model (unused when greedy) */
+  int32_t d_verify;     /* width of the verifier sub-model */
+  float temperature;    /* > 0 (paper: 0.4) */
+  float top_p;          /* (0, 1] (paper: 0.9) */
+  int32_t greedy;       /* non-zero: greedy verification */
+  int32_t in_dtype;     /* MLS_BF16 or MLS_FP32 */
+} mls_spec_problem;
+
+size_t mls_spec_workspace_size(const mls_spec_problem* p);
+int mls_spec_verify(const mls_spec_problem* p, const void* H_draft, const void* W_draft,
+                    const void* H_verify, const void* W_verify, const int32_t* draft_tokens,
+                    const float* uniforms, int32_t* n_accepted, int32_t* next_token, void* ws,
+                    size_t ws_bytes, mls_stream_t stream);
+
+/*
  * Synchronises `stream`, then returns the status bits (MLS_STATUS_*) recorded by
  * the device on the current device since the last call and clears them; returns
  * a negative MLS_ERR_CUDA if the synchronisation or the read failed.

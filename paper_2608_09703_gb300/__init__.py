@@ -9,12 +9,15 @@ from .binding import (  # noqa: F401
     HeadLoss,
     MLSError,
     Problem,
+    SpecVerify,
     mls_get_status,
     mls_head_loss_bwd,
     mls_head_loss_fwd,
     mls_head_pairwise,
     mls_junction_bwd,
     mls_junction_fwd,
+    mls_spec_verify,
+    mls_spec_workspace_size,
     mls_strerror,
     mls_workspace_size,
 )

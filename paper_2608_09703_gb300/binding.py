@@ -45,6 +45,20 @@ class mls_problem(ctypes.Structure):
     ]
 
 
+class mls_spec_problem(ctypes.Structure):
+    _fields_ = [
+        ("B", ctypes.c_int32),
+        ("gamma", ctypes.c_int32),
+        ("V", ctypes.c_int64),
+        ("d_draft", ctypes.c_int32),
+        ("d_verify", ctypes.c_int32),
+        ("temperature", ctypes.c_float),
+        ("top_p", ctypes.c_float),
+        ("greedy", ctypes.c_int32),
+        ("in_dtype", ctypes.c_int32),
+    ]
+
+
 class mls_kernel_time(ctypes.Structure):
     _fields_ = [("name", ctypes.c_char_p), ("launches", ctypes.c_int), ("total_ms", ctypes.c_double)]
 
@@ -84,6 +98,11 @@ def lib():
         L.mls_junction_bwd.restype = ctypes.c_int
         L.mls_head_loss_fwd_noalloc.argtypes = [P, vpp, vpp, vp, vp, vp, vp, vp, vp, vp]
         L.mls_head_loss_fwd_noalloc.restype = ctypes.c_int
+        SP = ctypes.POINTER(mls_spec_problem)
+        L.mls_spec_workspace_size.argtypes = [SP]
+        L.mls_spec_workspace_size.restype = ctypes.c_size_t
+        L.mls_spec_verify.argtypes = [SP, vp, vp, vp, vp, vp, vp, vp, vp, vp, ctypes.c_size_t, vp]
+        L.mls_spec_verify.restype = ctypes.c_int
         L.mls_profile_enable.argtypes = [ctypes.c_int]
         L.mls_profile_enable.restype = ctypes.c_int
         L.mls_profile_read.argtypes = [ctypes.POINTER(mls_kernel_time), ctypes.c_int]
@@ -185,6 +204,27 @@ def mls_junction_bwd(o, e, g, d_o, d_e, embed_first=False, stream=None) -> None:
     _check(rc, "mls_junction_bwd")
 
 
+def spec_problem(B: int, gamma: int, V: int, d_draft: int, d_verify: int,
+                 temperature: float = 0.4, top_p: float = 0.9, greedy: bool = False,
+                 in_dtype: int = MLS_BF16) -> mls_spec_problem:
+    return mls_spec_problem(int(B), int(gamma), int(V), int(d_draft), int(d_verify),
+                            float(temperature), float(top_p), int(bool(greedy)), int(in_dtype))
+
+
+def mls_spec_workspace_size(p: mls_spec_problem) -> int:
+    return int(lib().mls_spec_workspace_size(ctypes.byref(p)))
+
+
+def mls_spec_verify(p: mls_spec_problem, H_draft, W_draft, H_verify, W_verify, draft_tokens,
+                    uniforms, n_accepted, next_token, ws, stream=None) -> None:
+    """Speculative-decoding verify step (see include/mls.h)."""
+    rc = lib().mls_spec_verify(ctypes.byref(p), _ptr(H_draft), _ptr(W_draft), _ptr(H_verify),
+                               _ptr(W_verify), _ptr(draft_tokens), _ptr(uniforms),
+                               _ptr(n_accepted), _ptr(next_token), _ptr(ws),
+                               0 if ws is None else ws.numel() * ws.element_size(), _stream(stream))
+    _check(rc, "mls_spec_verify")
+
+
 def mls_head_loss_fwd_noalloc(prob: Problem, H, W, targets, loss, tok_loss, tok_diag, argmax,
                               stats, stream=None) -> None:
     """Forward with the library's built-in scratch instead of a workspace, for
@@ -272,3 +312,26 @@ class HeadLoss:
         mls_head_loss_bwd(self.prob, H, W, targets, self.stats, grad_scale, self.dH, self.dW,
                           self.ws, stream)
         return self.dH, self.dW
+
+
+class SpecVerify:
+    """Speculative-decoding verify step with its outputs and workspace
+    allocated once per shape.  H_draft: [B*gamma, d_draft], W_draft:
+    [V, d_draft], H_verify: [B*(gamma+1), d_verify], W_verify: [V, d_verify]
+    (bf16 or fp32); draft_tokens int32 [B, gamma]; uniforms fp32
+    [B, gamma+1, 2]."""
+
+    def __init__(self, B, gamma, V, d_draft, d_verify, temperature=0.4, top_p=0.9, greedy=False,
+                 dtype=torch.bfloat16, device="cuda"):
+        self.p = spec_problem(B, gamma, V, d_draft, d_verify, temperature, top_p, greedy,
+                              MLS_BF16 if dtype == torch.bfloat16 else MLS_FP32)
+        dev = torch.device(device)
+        self.n_accepted = torch.empty(B, dtype=torch.int32, device=dev)
+        self.next_token = torch.empty(B, dtype=torch.int32, device=dev)
+        self.ws = torch.empty(max(mls_spec_workspace_size(self.p), 1), dtype=torch.uint8,
+                              device=dev)
+
+    def __call__(self, H_draft, W_draft, H_verify, W_verify, draft_tokens, uniforms, stream=None):
+        mls_spec_verify(self.p, H_draft, W_draft, H_verify, W_verify, draft_tokens, uniforms,
+                        self.n_accepted, self.next_token, self.ws, stream)
+        return self.n_accepted, self.next_token

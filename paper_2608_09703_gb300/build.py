@@ -20,7 +20,7 @@ CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libmls.so")
 SOURCES = ["mls_api.cu", "mls_head.cu", "mls_gemm.cu", "mls_reduce.cu", "mls_eval.cu",
-           "mls_junction.cu"]
+           "mls_junction.cu", "mls_spec.cu"]
 HEADERS = ["mls_device.cuh", "mls_kernels.h"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

@@ -68,6 +68,8 @@ int device_state(DeviceState** out) {
       s.err = fail(MLS_ERR_CUDA, "gemm kernel attributes", e);
     } else if ((e = setup_eval_kernels()) != cudaSuccess) {
       s.err = fail(MLS_ERR_CUDA, "eval kernel attributes", e);
+    } else if ((e = setup_spec_kernels()) != cudaSuccess) {
+      s.err = fail(MLS_ERR_CUDA, "spec kernel attributes", e);
     } else if ((s.gemm_pairs = gemm_max_active_pairs()) <= 0) {
       s.err = fail(MLS_ERR_CUDA, "gemm cluster occupancy");
     } else if ((s.head_pairs = head_max_active_pairs()) <= 0) {
@@ -801,4 +803,136 @@ extern "C" int mls_junction_bwd(int64_t T, int32_t d_prev, int32_t d_next, int32
   JunctionParams jp{T, d_prev, d_next, embed_first ? 1 : 0, o, e, nullptr, g, d_o, d_e};
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   return timed("junction_bwd", s, [&] { return launch_junction_bwd(jp, in_dtype == MLS_FP32, s); });
+}
+
+// ------------------------------------------------------------------ speculative verify
+namespace {
+struct SpecPlan {
+  long long Pd = 0, Pv = 0, ldz = 0;
+  size_t off_zv = 0, off_zd = 0, off_sv = 0, off_sd = 0, off_acc = 0, off_tok = 0, total = 0;
+};
+
+int spec_validate(const mls_spec_problem* p) {
+  if (!p || p->B < 0 || p->gamma < 0 || p->V < 1 || p->V > INT_MAX) return MLS_ERR_ARG;
+  if (p->in_dtype != MLS_BF16 && p->in_dtype != MLS_FP32) return MLS_ERR_ARG;
+  if (static_cast<long long>(p->B) * (p->gamma + 1) > INT_MAX) return MLS_ERR_ARG;
+  const int elt = p->in_dtype == MLS_BF16 ? 2 : 4;
+  if (p->d_verify < 1) return MLS_ERR_ARG;
+  if ((static_cast<long long>(p->d_verify) * elt) % 16 != 0) return MLS_ERR_UNSUPPORTED;
+  if (!p->greedy) {
+    if (p->d_draft < 1) return MLS_ERR_ARG;
+    if ((static_cast<long long>(p->d_draft) * elt) % 16 != 0) return MLS_ERR_UNSUPPORTED;
+    if (!(p->temperature > 0.f) || !std::isfinite(p->temperature)) return MLS_ERR_ARG;
+    if (!(p->top_p > 0.f && p->top_p <= 1.f)) return MLS_ERR_ARG;
+  }
+  return MLS_OK;
+}
+
+SpecPlan spec_plan(const mls_spec_problem* p) {
+  SpecPlan pl;
+  pl.Pv = static_cast<long long>(p->B) * (p->gamma + 1);
+  pl.Pd = p->greedy ? 0 : static_cast<long long>(p->B) * p->gamma;
+  pl.ldz = ceil_div(p->V, 4) * 4;
+  size_t o = 0;
+  pl.off_zv = o;
+  o = align_up(o + sizeof(float) * static_cast<size_t>(pl.Pv) * pl.ldz);
+  pl.off_zd = o;
+  o = align_up(o + sizeof(float) * static_cast<size_t>(pl.Pd) * pl.ldz);
+  pl.off_sv = o;
+  o = align_up(o + sizeof(float) * kSpecStateWords * static_cast<size_t>(pl.Pv));
+  pl.off_sd = o;
+  o = align_up(o + sizeof(float) * kSpecStateWords * static_cast<size_t>(pl.Pd));
+  pl.off_acc = o;
+  o = align_up(o + sizeof(int) * static_cast<size_t>(pl.Pv));
+  pl.off_tok = o;
+  o = align_up(o + sizeof(int) * static_cast<size_t>(pl.Pv));
+  pl.total = o;
+  return pl;
+}
+}  // namespace
+
+extern "C" size_t mls_spec_workspace_size(const mls_spec_problem* p) {
+  if (spec_validate(p)) return 0;
+  return spec_plan(p).total;
+}
+
+extern "C" int mls_spec_verify(const mls_spec_problem* p, const void* H_draft, const void* W_draft,
+                               const void* H_verify, const void* W_verify,
+                               const int32_t* draft_tokens, const float* uniforms,
+                               int32_t* n_accepted, int32_t* next_token, void* ws, size_t ws_bytes,
+                               mls_stream_t stream) {
+  int rc = spec_validate(p);
+  if (rc) return rc;
+  if (p->B == 0) return MLS_OK;
+  if (!H_verify || !W_verify || !n_accepted || !next_token || (p->gamma > 0 && !draft_tokens))
+    return MLS_ERR_ARG;
+  if (!p->greedy && (!uniforms || (p->gamma > 0 && (!H_draft || !W_draft)))) return MLS_ERR_ARG;
+  if (!aligned16(H_verify) || !aligned16(W_verify) || !aligned16(H_draft) || !aligned16(W_draft))
+    return MLS_ERR_ALIGN;
+  const SpecPlan pl = spec_plan(p);
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) % kAlign) != 0 || ws_bytes < pl.total)
+    return MLS_ERR_WORKSPACE;
+  DeviceState* dev = nullptr;
+  if ((rc = device_state(&dev))) return rc;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  char* wsb = static_cast<char*>(ws);
+  const bool tf32 = p->in_dtype == MLS_FP32;
+  const int elt = tf32 ? 4 : 2, KE = 128 / elt;
+
+  SpecParams sp;
+  std::memset(&sp, 0, sizeof sp);
+  sp.V = p->V;
+  sp.ldz = pl.ldz;
+  sp.B = p->B;
+  sp.gamma = p->gamma;
+  sp.greedy = p->greedy ? 1 : 0;
+  sp.cap = kSpecListCap;
+  sp.scale = p->greedy ? 1.f : 1.4426950408889634f / p->temperature;
+  sp.top_p = p->greedy ? 1.f : p->top_p;
+  sp.zv = reinterpret_cast<float*>(wsb + pl.off_zv);
+  sp.zd = reinterpret_cast<float*>(wsb + pl.off_zd);
+  sp.draft = draft_tokens;
+  sp.u = uniforms;
+  sp.state_v = reinterpret_cast<float*>(wsb + pl.off_sv);
+  sp.state_d = reinterpret_cast<float*>(wsb + pl.off_sd);
+  sp.acc = reinterpret_cast<int*>(wsb + pl.off_acc);
+  sp.tok = reinterpret_cast<int*>(wsb + pl.off_tok);
+  sp.n_accepted = n_accepted;
+  sp.next_token = next_token;
+
+  // Logits of the verify positions: one GEMM launch over the verifier's rows
+  // and (sampling) the draft's, z = H W^T with both operands K-major.
+  GemmParams g;
+  std::memset(&g, 0, sizeof g);
+  const void* Hs[2] = {H_verify, H_draft};
+  const void* Ws[2] = {W_verify, W_draft};
+  const int ds[2] = {p->d_verify, p->d_draft};
+  const long long Ps[2] = {pl.Pv, pl.Pd};
+  float* Cs[2] = {const_cast<float*>(sp.zv), const_cast<float*>(sp.zd)};
+  int tiles = 0;
+  for (int m = 0; m < 2; ++m) {
+    if (Ps[m] == 0) continue;
+    const int i = g.nprob++;
+    if (encode(&g.mapA[i], Hs[m], elt, ds[m], Ps[m], ds[m], KE, kGemmBM) ||
+        encode(&g.mapB[i], Ws[m], elt, ds[m], p->V, ds[m], KE, kGemmBHalf))
+      return MLS_ERR_CUDA;
+    GemmProblem& pr = g.prob[i];
+    pr.Mrows = static_cast<int>(Ps[m]);
+    pr.Ncols = static_cast<int>(p->V);
+    pr.K = ds[m];
+    pr.a_map = pr.b_map = i;
+    pr.C = Cs[m];
+    pr.ldc = pl.ldz;
+    pr.tiles_n = static_cast<int>(ceil_div(p->V, kGemmBN));
+    pr.tiles_m = static_cast<int>(ceil_div(Ps[m], 2 * kGemmBM));
+    pr.m_fast = 1;
+    pr.tile_begin = tiles;
+    tiles += pr.tiles_m * pr.tiles_n;
+  }
+  g.total_tiles = tiles;
+  g.status = dev->status;
+  const int grid = 2 * (tiles < dev->gemm_pairs ? tiles : dev->gemm_pairs);
+  if ((rc = timed("spec_logits", s, [&] { return launch_gemm_kk(g, tf32, grid, s); }))) return rc;
+  if ((rc = timed("spec_position", s, [&] { return launch_spec_position(sp, s); }))) return rc;
+  return timed("spec_sample", s, [&] { return launch_spec_sample(sp, s); });
 }

@@ -60,6 +60,7 @@ __device__ __forceinline__ TileCoord decode_tile(const GemmParams& p, int t) {
   int i = 0;
   while (i + 1 < p.nprob && t >= p.prob[i + 1].tile_begin) ++i;
   const int local = t - p.prob[i].tile_begin;
+  if (p.prob[i].m_fast) return {i, local % p.prob[i].tiles_m, local / p.prob[i].tiles_m};
   return {i, local / p.prob[i].tiles_n, local % p.prob[i].tiles_n};
 }
 

@@ -98,6 +98,9 @@ struct GemmProblem {
   int accumulate;                // C += A*B if 1, C = A*B if 0
   int tiles_n;                   // ceil(Ncols / kGemmBN)
   int tile_begin;                // first linear pair tile (256 x kGemmBN) of this problem
+  int tiles_m;                   // ceil(Mrows / 256); used when m_fast is set
+  int m_fast;                    // 1: consecutive tiles walk M first (pairs running at the
+                                 //    same time share the B tile, read once from HBM)
 };
 
 struct GemmParams {
@@ -164,6 +167,34 @@ struct JunctionParams {
 };
 cudaError_t launch_junction_fwd(const JunctionParams& p, bool fp32, cudaStream_t s);
 cudaError_t launch_junction_bwd(const JunctionParams& p, bool fp32, cudaStream_t s);
+
+// ------------------------------------------------------------------ speculative verify
+// Per position of a sequence: the verifier's logits row (and the draft's for
+// the gamma drafted positions), fp32 with row pitch ldz (a multiple of 4).
+constexpr int kSpecStateWords = 8;   // per row: max, b, kept mass, c, ties, sum (+2 spare)
+constexpr int kSpecListCap = 12288;  // candidates per shared-memory list (two lists)
+
+struct SpecParams {
+  long long V, ldz;
+  int B, gamma;
+  int greedy;
+  int cap;                       // kSpecListCap
+  float scale;                   // log2(e) / temperature
+  float top_p;
+  const float* zd;               // [B * gamma][ldz] draft logits (sampling only)
+  const float* zv;               // [B * (gamma + 1)][ldz] verifier logits
+  const int* draft;              // [B * gamma]
+  const float* u;                // [B][gamma + 1][2]
+  float* state_d;                // [B * gamma][kSpecStateWords]
+  float* state_v;                // [B * (gamma + 1)][kSpecStateWords]
+  int* acc;                      // [B * (gamma + 1)] accepted flag per position
+  int* tok;                      // [B * (gamma + 1)] verifier argmax (greedy)
+  int* n_accepted;               // [B]
+  int* next_token;               // [B]
+};
+cudaError_t setup_spec_kernels();
+cudaError_t launch_spec_position(const SpecParams& p, cudaStream_t s);
+cudaError_t launch_spec_sample(const SpecParams& p, cudaStream_t s);
 
 // ------------------------------------------------------------------ reductions
 struct MergeParams {

@@ -124,3 +124,57 @@ def as_oracle_arrays(ts: Sequence[torch.Tensor]):
         else:
             raise TypeError(t.dtype)
     return out
+
+
+# Speculative-decoding verify inputs (Sec. 3.2.3: a 500M draft and a 3B
+# verifier of one suite, batch up to 102, draft length 6, vocabulary of the
+# suite).  Nested like the suite: the verifier's hidden state at a drafted
+# position extends the draft's (first d_draft channels shared) and its head
+# extends the draft's head, so the verifier's logits are the draft's plus an
+# independent part whose spread is `extra` times the draft's.
+@dataclasses.dataclass(frozen=True)
+class SpecWorkload:
+    name: str
+    B: int
+    gamma: int
+    V: int
+    d_draft: int
+    d_verify: int
+    dtype: str = "bf16"
+    temperature: float = 0.4
+    top_p: float = 0.9
+    z_std: float = 2.5       # spread of the draft's logits
+    extra: float = 0.2       # spread of the verifier's extra logit part / z_std
+
+
+SPEC_WORKLOADS = {
+    "spec_suite3": SpecWorkload("spec_suite3", B=102, gamma=6, V=50304, d_draft=1024, d_verify=3072),
+}
+
+
+def make_spec_inputs(wl: SpecWorkload, seed: int = 0, device="cpu"):
+    """Draw (H_draft [B*gamma, d_d], W_draft [V, d_d], H_verify [B*(gamma+1), d_v],
+    W_verify [V, d_v]) in the workload's storage dtype.  fp32 workloads hold
+    bf16-representable values.  Seeds: hidden states seed + 0, heads seed + 1."""
+    dt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+    gH, gW = _gen(seed, device), _gen(seed + 1, device)
+    dd, dv, G1 = wl.d_draft, wl.d_verify, wl.gamma + 1
+    f32 = dict(device=device, dtype=torch.float32)
+    hv = torch.randn(wl.B, G1, dv, generator=gH, **f32)
+    wd = torch.randn(wl.V, dd, generator=gW, **f32) * (wl.z_std / dd ** 0.5)
+    de = dv - dd
+    we = torch.randn(wl.V, de, generator=gW, **f32) * (wl.extra * wl.z_std / max(de, 1) ** 0.5)
+    Wv = torch.cat([wd, we], 1)
+    Hd = hv[:, :wl.gamma, :dd].reshape(wl.B * wl.gamma, dd)
+    Hv = hv.reshape(wl.B * G1, dv)
+
+    def st(t):
+        return t.to(torch.bfloat16).to(dt).contiguous()
+
+    return st(Hd), st(wd), st(Hv), st(Wv)
+
+
+def make_uniforms(B: int, gamma: int, seed: int = 0, device="cpu") -> torch.Tensor:
+    """Acceptance and sampling draws u [B, gamma+1, 2] in [0, 1), fp32 (seed + 2)."""
+    return torch.rand(B, gamma + 1, 2, generator=_gen(seed + 2, device), device=device,
+                      dtype=torch.float32)

@@ -86,3 +86,37 @@ def test_workspace_size(lib):
     g256 = B.mls_workspace_size(B.Problem([1024, 2048, 3072], 8192, 50304, vocab_group=256))
     assert g256 < big
     assert B.mls_workspace_size(B.Problem([64, 64], 10, 100, tau=-1.0)) == 0
+
+
+def test_spec_verify_validation_without_gpu(lib):
+    """The verify step's host checks: invalid problems and arguments are
+    rejected before any CUDA call; the workspace holds the fp32 logits of every
+    verify position plus small per-row state."""
+    ws = ctypes.c_void_p(0x100000)
+
+    def call(p, h=0x1000, t=0x2000, u=0x3000, size=1 << 40):
+        return lib.mls_spec_verify(ctypes.byref(p), h, h, h, h, t, u, t, t, ws, size, None)
+
+    for kw in (dict(top_p=0.0), dict(top_p=1.5), dict(temperature=0.0), dict(temperature=-1.0)):
+        args = dict(B=4, gamma=2, V=100, d_draft=64, d_verify=64)
+        args.update(kw)
+        p = B.spec_problem(**args)
+        assert call(p) == B.MLS_ERR_ARG
+        assert B.mls_spec_workspace_size(p) == 0
+    assert call(B.spec_problem(-1, 2, 100, 64, 64)) == B.MLS_ERR_ARG
+    assert call(B.spec_problem(4, -1, 100, 64, 64)) == B.MLS_ERR_ARG
+    assert call(B.spec_problem(4, 2, 0, 64, 64)) == B.MLS_ERR_ARG
+    assert call(B.spec_problem(4, 2, 100, 60, 64)) == B.MLS_ERR_UNSUPPORTED
+    assert call(B.spec_problem(4, 2, 100, 64, 60)) == B.MLS_ERR_UNSUPPORTED
+    # greedy ignores the draft model's width, temperature and top_p
+    assert B.mls_spec_workspace_size(B.spec_problem(4, 2, 100, 60, 64, 0.0, 0.0, True)) > 0
+    assert call(B.spec_problem(4, 2, 100, 64, 64), h=0x1008) == B.MLS_ERR_ALIGN
+    assert call(B.spec_problem(4, 2, 100, 64, 64), u=0) == B.MLS_ERR_ARG
+    assert call(B.spec_problem(4, 2, 100, 64, 64), size=1024) == B.MLS_ERR_WORKSPACE
+    assert call(B.spec_problem(0, 2, 100, 64, 64)) == B.MLS_OK  # nothing to do
+    # sizes: logits rows padded to 4 floats; the draft's only when sampling
+    ldz = 4 * ((101 + 3) // 4)
+    samp = B.mls_spec_workspace_size(B.spec_problem(4, 2, 101, 64, 64))
+    greedy = B.mls_spec_workspace_size(B.spec_problem(4, 2, 101, 64, 64, greedy=True))
+    assert samp >= 4 * (4 * 3 + 4 * 2) * ldz and greedy >= 4 * 4 * 3 * ldz
+    assert samp - greedy >= 4 * 4 * 2 * ldz
