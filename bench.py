@@ -569,15 +569,16 @@ def spec_run(args, dev, pk):
         ms = e0.elapsed_time(e1) / n
         gemm_ms = kp["spec_logits"][1] / n
         f = flops if not greedy else 2 * wl.V * Pv * wl.d_verify
-        rows = (Pv if greedy else Pv + Pd)
-        sel_ms = kp["spec_position"][1] / n
         out[mode] = {
             "ms_per_call": ms, "positions_per_s": Pv / (ms / 1e3),
             "kernel_ms": {k: v[1] / n for k, v in kp.items()},
             "logits_tflops": f / (gemm_ms / 1e3) / 1e12,
             "logits_frac_of_sustained": f / (gemm_ms / 1e3) / 1e12 / float(pk["bf16_tflops_sustained"]),
-            "selection_gbs_one_read": rows * wl.V * 4 / (sel_ms / 1e3) / 1e9,
         }
+        if not greedy:
+            # the selection kernels against one read of every probability row
+            sel_ms = (kp["spec_position"][1] + kp["spec_sample"][1]) / n
+            out[mode]["selection_gbs_one_read"] = (Pv + Pd) * wl.V * 4 / (sel_ms / 1e3) / 1e9
     return out
 
 

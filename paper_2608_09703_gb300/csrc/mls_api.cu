@@ -808,8 +808,9 @@ extern "C" int mls_junction_bwd(int64_t T, int32_t d_prev, int32_t d_next, int32
 // ------------------------------------------------------------------ speculative verify
 namespace {
 struct SpecPlan {
-  long long Pd = 0, Pv = 0, ldz = 0;
-  size_t off_zv = 0, off_zd = 0, off_sv = 0, off_sd = 0, off_acc = 0, off_tok = 0, total = 0;
+  long long Pd = 0, Pv = 0, ldz = 0, tiles = 0;
+  size_t off_ev = 0, off_ed = 0, off_sv = 0, off_sd = 0, off_fv = 0, off_fd = 0;
+  size_t off_stv = 0, off_std = 0, off_acc = 0, total = 0;
 };
 
 int spec_validate(const mls_spec_problem* p) {
@@ -824,6 +825,7 @@ int spec_validate(const mls_spec_problem* p) {
     if ((static_cast<long long>(p->d_draft) * elt) % 16 != 0) return MLS_ERR_UNSUPPORTED;
     if (!(p->temperature > 0.f) || !std::isfinite(p->temperature)) return MLS_ERR_ARG;
     if (!(p->top_p > 0.f && p->top_p <= 1.f)) return MLS_ERR_ARG;
+    if (p->V > static_cast<long long>(kSpecMaxTiles) * kGemmBN) return MLS_ERR_UNSUPPORTED;
   }
   return MLS_OK;
 }
@@ -833,19 +835,22 @@ SpecPlan spec_plan(const mls_spec_problem* p) {
   pl.Pv = static_cast<long long>(p->B) * (p->gamma + 1);
   pl.Pd = p->greedy ? 0 : static_cast<long long>(p->B) * p->gamma;
   pl.ldz = ceil_div(p->V, 4) * 4;
+  pl.tiles = ceil_div(p->V, kGemmBN);
+  const size_t rows_e = p->greedy ? 0 : static_cast<size_t>(pl.Pv);  // e_t is only stored when sampling
   size_t o = 0;
-  pl.off_zv = o;
-  o = align_up(o + sizeof(float) * static_cast<size_t>(pl.Pv) * pl.ldz);
-  pl.off_zd = o;
-  o = align_up(o + sizeof(float) * static_cast<size_t>(pl.Pd) * pl.ldz);
-  pl.off_sv = o;
-  o = align_up(o + sizeof(float) * kSpecStateWords * static_cast<size_t>(pl.Pv));
-  pl.off_sd = o;
-  o = align_up(o + sizeof(float) * kSpecStateWords * static_cast<size_t>(pl.Pd));
-  pl.off_acc = o;
-  o = align_up(o + sizeof(int) * static_cast<size_t>(pl.Pv));
-  pl.off_tok = o;
-  o = align_up(o + sizeof(int) * static_cast<size_t>(pl.Pv));
+  auto take = [&](size_t& off, size_t bytes) {
+    off = o;
+    o = align_up(o + bytes);
+  };
+  take(pl.off_ev, sizeof(float) * rows_e * pl.ldz);
+  take(pl.off_ed, sizeof(float) * static_cast<size_t>(pl.Pd) * pl.ldz);
+  take(pl.off_stv, sizeof(float) * 2 * static_cast<size_t>(pl.Pv) * pl.tiles);
+  take(pl.off_std, sizeof(float) * 2 * static_cast<size_t>(pl.Pd) * pl.tiles);
+  take(pl.off_fv, sizeof(float) * rows_e * pl.tiles);
+  take(pl.off_fd, sizeof(float) * static_cast<size_t>(pl.Pd) * pl.tiles);
+  take(pl.off_sv, sizeof(float) * kSpecStateWords * static_cast<size_t>(pl.Pv));
+  take(pl.off_sd, sizeof(float) * kSpecStateWords * static_cast<size_t>(pl.Pd));
+  take(pl.off_acc, sizeof(int) * static_cast<size_t>(pl.Pv));
   pl.total = o;
   return pl;
 }
@@ -878,6 +883,7 @@ extern "C" int mls_spec_verify(const mls_spec_problem* p, const void* H_draft, c
   char* wsb = static_cast<char*>(ws);
   const bool tf32 = p->in_dtype == MLS_FP32;
   const int elt = tf32 ? 4 : 2, KE = 128 / elt;
+  auto at = [&](size_t off) { return reinterpret_cast<float*>(wsb + off); };
 
   SpecParams sp;
   std::memset(&sp, 0, sizeof sp);
@@ -886,35 +892,42 @@ extern "C" int mls_spec_verify(const mls_spec_problem* p, const void* H_draft, c
   sp.B = p->B;
   sp.gamma = p->gamma;
   sp.greedy = p->greedy ? 1 : 0;
-  sp.cap = kSpecListCap;
+  sp.tiles = static_cast<int>(pl.tiles);
   sp.scale = p->greedy ? 1.f : 1.4426950408889634f / p->temperature;
   sp.top_p = p->greedy ? 1.f : p->top_p;
-  sp.zv = reinterpret_cast<float*>(wsb + pl.off_zv);
-  sp.zd = reinterpret_cast<float*>(wsb + pl.off_zd);
+  sp.ev = at(pl.off_ev);
+  sp.ed = at(pl.off_ed);
+  sp.stats_v = at(pl.off_stv);
+  sp.stats_d = at(pl.off_std);
+  sp.f_v = at(pl.off_fv);
+  sp.f_d = at(pl.off_fd);
   sp.draft = draft_tokens;
   sp.u = uniforms;
-  sp.state_v = reinterpret_cast<float*>(wsb + pl.off_sv);
-  sp.state_d = reinterpret_cast<float*>(wsb + pl.off_sd);
+  sp.state_v = at(pl.off_sv);
+  sp.state_d = at(pl.off_sd);
   sp.acc = reinterpret_cast<int*>(wsb + pl.off_acc);
-  sp.tok = reinterpret_cast<int*>(wsb + pl.off_tok);
   sp.n_accepted = n_accepted;
   sp.next_token = next_token;
 
   // Logits of the verify positions: one GEMM launch over the verifier's rows
-  // and (sampling) the draft's, z = H W^T with both operands K-major.
+  // and (sampling) the draft's, z = H W^T with both operands K-major; its
+  // epilogue leaves per-tile softmax statistics (sampling) or the per-tile
+  // maximum and argmax (greedy) instead of the logits.
   GemmParams g;
   std::memset(&g, 0, sizeof g);
   const void* Hs[2] = {H_verify, H_draft};
   const void* Ws[2] = {W_verify, W_draft};
   const int ds[2] = {p->d_verify, p->d_draft};
   const long long Ps[2] = {pl.Pv, pl.Pd};
-  float* Cs[2] = {const_cast<float*>(sp.zv), const_cast<float*>(sp.zd)};
+  float* Cs[2] = {at(pl.off_ev), at(pl.off_ed)};
+  float* Ss[2] = {at(pl.off_stv), at(pl.off_std)};
   int tiles = 0;
   for (int m = 0; m < 2; ++m) {
     if (Ps[m] == 0) continue;
     const int i = g.nprob++;
     if (encode(&g.mapA[i], Hs[m], elt, ds[m], Ps[m], ds[m], KE, kGemmBM) ||
-        encode(&g.mapB[i], Ws[m], elt, ds[m], p->V, ds[m], KE, kGemmBHalf))
+        encode(&g.mapB[i], Ws[m], elt, ds[m], p->V, ds[m], KE, kGemmBHalf) ||
+        (!p->greedy && encode(&g.mapC[i], Cs[m], 4, p->V, Ps[m], pl.ldz, 32, 32)))
       return MLS_ERR_CUDA;
     GemmProblem& pr = g.prob[i];
     pr.Mrows = static_cast<int>(Ps[m]);
@@ -923,16 +936,22 @@ extern "C" int mls_spec_verify(const mls_spec_problem* p, const void* H_draft, c
     pr.a_map = pr.b_map = i;
     pr.C = Cs[m];
     pr.ldc = pl.ldz;
-    pr.tiles_n = static_cast<int>(ceil_div(p->V, kGemmBN));
+    pr.tiles_n = static_cast<int>(pl.tiles);
     pr.tiles_m = static_cast<int>(ceil_div(Ps[m], 2 * kGemmBM));
     pr.m_fast = 1;
     pr.tile_begin = tiles;
+    pr.epi = p->greedy ? kEpiArgmax : kEpiSoftmax;
+    pr.epi_scale = sp.scale;
+    pr.stats = Ss[m];
+    pr.stats_ld = 2 * pl.tiles;
     tiles += pr.tiles_m * pr.tiles_n;
   }
   g.total_tiles = tiles;
   g.status = dev->status;
   const int grid = 2 * (tiles < dev->gemm_pairs ? tiles : dev->gemm_pairs);
   if ((rc = timed("spec_logits", s, [&] { return launch_gemm_kk(g, tf32, grid, s); }))) return rc;
-  if ((rc = timed("spec_position", s, [&] { return launch_spec_position(sp, s); }))) return rc;
+  if (!p->greedy &&
+      (rc = timed("spec_position", s, [&] { return launch_spec_position(sp, s); })))
+    return rc;
   return timed("spec_sample", s, [&] { return launch_spec_sample(sp, s); });
 }

@@ -45,8 +45,15 @@ struct GemmSmem {
   static constexpr uint32_t kTmemSlot = kBar + 8u * (2 * kGemmStages + 5);
   static constexpr uint32_t kAbort = kTmemSlot + 4;
   static constexpr uint32_t kEnd = kAbort + 4;
+  // kEpiSoftmax output staging: per epilogue warp two 32 x 32 fp32 chunks
+  // (128B-swizzled) written out by TMA stores.  It lies in the slack past the
+  // operand stages, which only the MN-major (plain-epilogue) GEMMs over-read.
+  static constexpr uint32_t kChunk = 32 * 32 * 4;
+  static constexpr uint32_t kStaging = (kEnd + 1023u) & ~1023u;
 };
 static_assert(GemmSmem::kEnd + 1024 <= kGemmSmem, "gemm shared memory map overflows");
+static_assert(GemmSmem::kStaging + kGemmEpiWarps * 2 * GemmSmem::kChunk + 1023 <= kGemmSmem,
+              "gemm output staging overflows");
 
 constexpr uint32_t kTmemCols = 512;
 constexpr uint64_t kDrainNs = 100000000ull;
@@ -177,22 +184,94 @@ __device__ __forceinline__ void gemm_mma(const GemmParams& p, uint32_t base, uin
   mbar_wait_drain(GemmSmem::drain(base), 0, kDrainNs);
 }
 
+// Row statistics epilogues (kEpiSoftmax, kEpiArgmax) of one 128 x kGemmBN
+// accumulator tile: each lane owns one row.  The maximum (and its first
+// column) come from one read of the row's accumulators; kEpiSoftmax reads
+// them again to store 2^((z - m_t) scale) and sum it in column order.
+__device__ __noinline__ void epilogue_stats(const GemmProblem& pr, const CUtensorMap* mapC,
+                                            uint32_t stage, uint32_t& count, uint32_t tacc,
+                                            int tn, long long row, bool row_ok, int row0,
+                                            int lane) {
+  float v[32];
+  float mt = -INFINITY;
+  int mi = tn * kGemmBN;
+#pragma unroll 1
+  for (int c = 0; c < kGemmBN / 32; ++c) {
+    tmem_ld32(tacc + c * 32, v);
+    const int col = tn * kGemmBN + c * 32;
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+      if (col + i < pr.Ncols && v[i] > mt) {
+        mt = v[i];
+        mi = col + i;
+      }
+  }
+  float* srow = pr.stats + (row_ok ? row : 0) * pr.stats_ld + 2 * tn;
+  if (pr.epi == kEpiArgmax) {
+    if (row_ok) {
+      srow[0] = mt;
+      srow[1] = __int_as_float(mi);
+    }
+    return;
+  }
+  float st = 0.f;
+#pragma unroll 1
+  for (int c = 0; c < kGemmBN / 32; ++c) {
+    tmem_ld32(tacc + c * 32, v);
+    const int col = tn * kGemmBN + c * 32;
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      v[i] = col + i < pr.Ncols ? fast_exp2((v[i] - mt) * pr.epi_scale) : 0.f;
+      st += v[i];
+    }
+    if (col >= pr.Ncols) continue;  // warp-uniform
+    // 32 rows x 32 columns through shared memory; the TMA store drops rows
+    // and columns outside C.
+    const uint32_t buf = stage + (count & 1u) * GemmSmem::kChunk;
+    if (lane == 0) bulk_wait_read<1>();  // the store that last used this buffer has read it
+    __syncwarp();
+    const uint32_t rowaddr = buf + lane * 128;
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+      st_shared_v4(rowaddr + ((j ^ (lane & 7)) << 4), __float_as_uint(v[4 * j]),
+                   __float_as_uint(v[4 * j + 1]), __float_as_uint(v[4 * j + 2]),
+                   __float_as_uint(v[4 * j + 3]));
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      tma_store_2d(mapC, buf, col, row0);
+      bulk_commit();
+    }
+    ++count;
+  }
+  if (row_ok) {
+    srow[0] = mt;
+    srow[1] = st;
+  }
+}
+
 __device__ __forceinline__ void gemm_epilogue(const GemmParams& p, uint32_t base, uint32_t tmem,
                                               uint32_t rank, int warp, int lane,
                                               volatile int* abort_flag) {
   const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
-  uint32_t acc = 0, acc_par = 0;
+  uint32_t acc = 0, acc_par = 0, stores = 0;
   const uint32_t tl = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+  const uint32_t stage = base + GemmSmem::kStaging + static_cast<uint32_t>(warp) * 2 * GemmSmem::kChunk;
   for (int t = pair; t < p.total_tiles; t += npairs) {
     const TileCoord tc = decode_tile(p, t);
     const GemmProblem& pr = p.prob[tc.prob];
     const bool ok = mbar_wait(GemmSmem::accf(base, acc), acc_par, abort_flag, p.status);
-    if (!__all_sync(0xffffffffu, ok)) return;
+    if (!__all_sync(0xffffffffu, ok)) break;
     tc_fence_after();
     const long long row = static_cast<long long>(tc.tm) * kPairM + rank * kGemmBM + warp * 32 + lane;
     const bool row_ok = row < pr.Mrows;
-    float* crow = pr.C + (row_ok ? row : 0) * pr.ldc;
     float v[32];
+    if (pr.epi != kEpiPlain) {
+      const int row0 = tc.tm * kPairM + static_cast<int>(rank) * kGemmBM + warp * 32;
+      epilogue_stats(pr, &p.mapC[tc.prob], stage, stores, tl + acc * kGemmBN, tc.tn, row, row_ok,
+                     row0, lane);
+    } else {
+    float* crow = pr.C + (row_ok ? row : 0) * pr.ldc;
 #pragma unroll 1
     for (int c = 0; c < kGemmBN / 32; ++c) {
       tmem_ld32(tl + acc * kGemmBN + c * 32, v);
@@ -220,12 +299,14 @@ __device__ __forceinline__ void gemm_epilogue(const GemmParams& p, uint32_t base
         }
       }
     }
+    }
     tc_fence_before();
     __syncwarp();
     if (lane == 0) mbar_arrive_remote(map_to_rank(GemmSmem::acce(base, acc), 0));
     acc ^= 1u;
     if (acc == 0) acc_par ^= 1u;
   }
+  if (stores && lane == 0) bulk_wait_all();  // staging must outlive the stores reading it
 }
 
 template <bool kTF32, bool kAMN, bool kBMN>

@@ -101,11 +101,22 @@ struct GemmProblem {
   int tiles_m;                   // ceil(Mrows / 256); used when m_fast is set
   int m_fast;                    // 1: consecutive tiles walk M first (pairs running at the
                                  //    same time share the B tile, read once from HBM)
+  // Epilogue (accumulate must be 0 unless kEpiPlain).  Per row and column tile
+  // (kGemmBN columns) the statistics go to stats[row * stats_ld + 2 * tile]:
+  //   kEpiSoftmax: C = 2^((z - m_t) epi_scale), stats = (m_t, sum of C over the tile)
+  //   kEpiArgmax:  C untouched, stats = (m_t, first column attaining m_t)
+  // with m_t the row's maximum over the tile.
+  int epi;
+  float epi_scale;
+  float* stats;
+  long long stats_ld;
 };
+enum GemmEpilogue { kEpiPlain = 0, kEpiSoftmax = 1, kEpiArgmax = 2 };
 
 struct GemmParams {
   CUtensorMap mapA[kMaxModels];
   CUtensorMap mapB[kMaxModels];
+  CUtensorMap mapC[kMaxModels];  // kEpiSoftmax: C fp32 [Mrows, Ncols], box {32, 32}, 128B swizzle
   int nprob;
   GemmProblem prob[kMaxModels];
   int total_tiles;
@@ -171,24 +182,31 @@ cudaError_t launch_junction_bwd(const JunctionParams& p, bool fp32, cudaStream_t
 // ------------------------------------------------------------------ speculative verify
 // Per position of a sequence: the verifier's logits row (and the draft's for
 // the gamma drafted positions), fp32 with row pitch ldz (a multiple of 4).
-constexpr int kSpecStateWords = 8;   // per row: max, b, kept mass, c, ties, sum (+2 spare)
-constexpr int kSpecListCap = 12288;  // candidates per shared-memory list (two lists)
+// The logits GEMM's epilogue leaves, per row, e_t[v] = 2^((z[v] - m_t) log2(e) / T)
+// relative to the maximum m_t of v's column tile, and per tile (m_t, sum of e_t)
+// (kEpiSoftmax); greedy verification only needs per tile (m_t, argmax) (kEpiArgmax).
+constexpr int kSpecStateWords = 8;    // per row: max, b, kept mass, c, ties, sum (+2 spare)
+constexpr int kSpecListCap = 8192;    // candidates per shared-memory list (two lists)
+constexpr int kSpecMaxTiles = 4096;   // column tiles of a row (V <= 4096 * kGemmBN when sampling)
 
 struct SpecParams {
   long long V, ldz;
   int B, gamma;
   int greedy;
-  int cap;                       // kSpecListCap
+  int tiles;                     // column tiles of kGemmBN per row
   float scale;                   // log2(e) / temperature
   float top_p;
-  const float* zd;               // [B * gamma][ldz] draft logits (sampling only)
-  const float* zv;               // [B * (gamma + 1)][ldz] verifier logits
+  const float* ed;               // [B * gamma][ldz] draft e_t (sampling only)
+  const float* ev;               // [B * (gamma + 1)][ldz] verifier e_t (sampling only)
+  const float* stats_d;          // [B * gamma][tiles][2]
+  const float* stats_v;          // [B * (gamma + 1)][tiles][2]
+  float* f_d;                    // [B * gamma][tiles]: 2^((m_t - max) log2(e) / T)
+  float* f_v;                    // [B * (gamma + 1)][tiles]
   const int* draft;              // [B * gamma]
   const float* u;                // [B][gamma + 1][2]
   float* state_d;                // [B * gamma][kSpecStateWords]
   float* state_v;                // [B * (gamma + 1)][kSpecStateWords]
   int* acc;                      // [B * (gamma + 1)] accepted flag per position
-  int* tok;                      // [B * (gamma + 1)] verifier argmax (greedy)
   int* n_accepted;               // [B]
   int* next_token;               // [B]
 };

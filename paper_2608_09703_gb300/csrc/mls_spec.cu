@@ -11,18 +11,22 @@
 // cumulative probability reaches top_p, then renormalised.  Greedy: accept
 // while x_i == argmax of the verifier's logits (lowest index on ties).
 //
-// The logits of the few verify positions are produced by the tensor-core GEMM
-// (fp32, one row per position).  Here, in units e_v = 2^((z_v - max) log2(e) / T):
-//   spec_position_kernel (one CTA per position) finds each row's nucleus: the
-//     boundary value b = the largest e with mass(e' >= b) >= top_p * S, by
-//     bisection over the bit patterns of e (non-negative floats order like
-//     their bits), each pass narrowing the bracket to its surviving keys and
-//     compacting the survivors into shared memory once they fit; then the c
+// The logits GEMM's epilogue (mls_gemm.cu) leaves, per row and column tile t
+// of 256, e_t[v] = 2^((z[v] - m_t) log2(e) / T) and (m_t, sum_t), or for greedy
+// only (m_t, argmax_t).  Here, with m = max_t m_t and f_t = 2^((m_t - m) log2(e)/T),
+// every token's unnormalised probability is e[v] = e_t[v] f_t (<= 1) and
+// S = sum_t sum_t f_t:
+//   spec_position_kernel (one CTA per position, sampling only) finds each
+//     row's nucleus: the boundary value b = the largest e with
+//     mass(e' >= b) >= top_p S, by bisection over the bit patterns of e
+//     (non-negative floats order like their bits), each pass narrowing the
+//     bracket to its surviving keys; survivors are compacted into shared memory
+//     once they fit and the last <= 256 are resolved exactly; then the c
 //     lowest-index tokens with e == b that the cumulative needs.  It then
 //     decides acceptance of the drafted token of that position.
 //   spec_sample_kernel (one CTA per sequence) takes the first rejection and
 //     samples by inverse CDF in index order, each warp walking a contiguous
-//     segment of the vocabulary.
+//     segment of the vocabulary; for greedy it reduces the tile argmaxes.
 // Every reduction has a fixed order, so a call is deterministic.
 #include "mls_device.cuh"
 #include "mls_kernels.h"
@@ -32,8 +36,13 @@ namespace {
 
 constexpr int kThreads = 512;
 constexpr int kWarps = kThreads / 32;
-constexpr int kStep = 128;  // elements one warp covers per float4 step
+constexpr int kStep = 128;              // elements one warp covers per float4 step
+constexpr int kUnroll = 4;              // independent float4 loads in flight per lane
+constexpr int kFinish = 256;            // candidates resolved exactly
 constexpr uint32_t kInfKey = 0x7f800000u;
+constexpr uint32_t kFirstMid = 0x3b800000u;  // 2^-8: first split of the bracket [0, inf)
+constexpr size_t kPositionSmem = sizeof(float) * (kSpecMaxTiles + 2 * kSpecListCap);
+static_assert(kFinish <= kThreads, "one candidate per thread in the exact finish");
 
 struct Shared {
   float f[kWarps][2];
@@ -69,10 +78,6 @@ __device__ __forceinline__ float warp_incl_scan(float v) {
     if (l >= o) v += t;
   }
   return v;
-}
-
-__device__ __forceinline__ float e_of(float z, float m, float scale) {
-  return fast_exp2((z - m) * scale);
 }
 
 __device__ __forceinline__ float comp(const float4& v, int j) {
@@ -123,20 +128,66 @@ __device__ void block_sum2(float& f, int& n, Shared& sh) {
   }
 }
 
-// Visits a logits row of V elements, warp w taking the 128-element steps
-// w, w + 16, ...: `f(i0, z4, V)` gets the lane's 4 consecutive elements from
-// index i0 (entries at or past V are not meaningful).  The loop is
-// warp-uniform, so f may use warp collectives.  Rows are 16-byte aligned and
-// padded to a multiple of 4 elements.
+__device__ uint32_t block_max_u(uint32_t v, Shared& sh) {
+  v = __reduce_max_sync(0xffffffffu, v);
+  __syncthreads();
+  if (lane_id() == 0) sh.k[warp_id()][0] = v;
+  __syncthreads();
+  uint32_t r = 0;
+  for (int w = 0; w < kWarps; ++w) r = max(r, sh.k[w][0]);
+  return r;
+}
+
+// Per-row softmax statistics from the per-tile ones: m, S and f_t (into the
+// shared table and, if fg is not null, into global memory).
+__device__ void row_stats(const float* st, int tiles, float scale, float* ftab, float* fg,
+                          float& m, float& S, Shared& sh) {
+  float mv = -INFINITY;
+  int unused = 0;
+  for (int t = threadIdx.x; t < tiles; t += kThreads) mv = fmaxf(mv, st[2 * t]);
+  block_argmax(mv, unused, sh);
+  m = mv;
+  float s = 0.f;
+  for (int t = threadIdx.x; t < tiles; t += kThreads) {
+    const float f = fast_exp2((st[2 * t] - m) * scale);
+    ftab[t] = f;
+    if (fg) fg[t] = f;
+    s = fmaf(st[2 * t + 1], f, s);
+  }
+  block_sum2(s, unused, sh);  // its barriers also publish ftab
+  S = s;
+}
+
+// Visits a row of unnormalised probabilities e[v] = e_t[v] f_t, warp w taking
+// the 128-element steps w, w + 16, ... (kUnroll of them per iteration):
+// `f(i0, e4, V)` gets the lane's 4 consecutive elements from index i0 (those
+// at or past V are not meaningful).  The loop is warp-uniform, so f may use
+// warp collectives.  Rows are 16-byte aligned and padded to 4 elements.
 template <typename F>
-__device__ __forceinline__ void for_row(const float* z, long long V, F&& f) {
+__device__ __forceinline__ void for_row(const float* et, const float* ftab, long long V, F&& f) {
   const int l = lane_id();
+  constexpr long long kStride = static_cast<long long>(kWarps) * kStep;
   for (long long base = static_cast<long long>(warp_id()) * kStep; base < V;
-       base += static_cast<long long>(kWarps) * kStep) {
-    const long long i0 = base + l * 4;
-    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (i0 < V) v = __ldg(reinterpret_cast<const float4*>(z + i0));
-    f(i0, v, V);
+       base += kUnroll * kStride) {
+    float4 v[kUnroll];
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const long long i0 = base + u * kStride + l * 4;
+      v[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (i0 < V) v[u] = __ldg(reinterpret_cast<const float4*>(et + i0));
+    }
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const long long i0 = base + u * kStride + l * 4;
+      if (i0 < V) {
+        const float fm = ftab[i0 / kGemmBN];
+        v[u].x *= fm;
+        v[u].y *= fm;
+        v[u].z *= fm;
+        v[u].w *= fm;
+      }
+      f(i0, v[u], V);
+    }
   }
 }
 
@@ -147,7 +198,8 @@ struct PassStats {
   float mass_ge = 0.f;
   int cnt_ge = 0, cnt_lt = 0;
   uint32_t min_ge = 0xffffffffu, max_ge = 0u, min_lt = 0xffffffffu, max_lt = 0u;
-  __device__ __forceinline__ void add(float e, uint32_t key, uint32_t lo, uint32_t mid, uint32_t hi) {
+  __device__ __forceinline__ void add(float e, uint32_t lo, uint32_t mid, uint32_t hi) {
+    const uint32_t key = __float_as_uint(e);
     if (key < lo || key >= hi) return;
     if (key >= mid) {
       mass_ge += e;
@@ -216,62 +268,63 @@ struct RowNucleus {
   int c, eq;
 };
 
-// Nucleus of softmax(z / T) for one logits row (scale = log2(e) / T); listA
-// and listB hold `cap` floats each.
-__device__ RowNucleus nucleus(const float* z, long long V, float scale, float top_p, float* listA,
-                              float* listB, int cap, Shared& sh) {
+// Exact boundary among the n <= kFinish candidates L (all keys in the current
+// bracket; mass_hi is the mass above it): b = the largest candidate key whose
+// mass(e >= key) = mass_hi + sum of the candidates >= it reaches the target
+// (each candidate's sum is taken over L in index order, so it is monotone in
+// the key), then the mass above b and the ties at b.
+__device__ void finish_exact(const float* L, int n, float target, float mass_hi, uint32_t lo,
+                             uint32_t& b, float& gt, int& eq, Shared& sh) {
+  const int t = threadIdx.x;
+  uint32_t kt = 0, best = 0;
+  float et = 0.f;
+  if (t < n) {
+    et = L[t];
+    kt = __float_as_uint(et);
+    float M = 0.f;
+    for (int j = 0; j < n; ++j) {
+      const float ej = L[j];
+      M += __float_as_uint(ej) >= kt ? ej : 0.f;
+    }
+    if (mass_hi + M >= target) best = kt + 1u;
+  }
+  best = block_max_u(best, sh);
+  b = best ? best - 1u : lo;  // by rounding alone nothing may qualify: the bracket's bottom
+  float part = (t < n && kt > b) ? et : 0.f;
+  int ties = (t < n && kt == b) ? 1 : 0;
+  block_sum2(part, ties, sh);
+  gt = mass_hi + part;
+  eq = ties;
+}
+
+// Nucleus of one row (e_t, per-tile stats st); writes f_t to fg.
+__device__ RowNucleus nucleus(const float* et, const float* st, float* fg, long long V, int tiles,
+                              float scale, float top_p, float* ftab, float* listA, float* listB,
+                              Shared& sh) {
   RowNucleus r;
-  {
-    float mv = -INFINITY;
-    int mi = 0;
-    for_row(z, V, [&](long long i0, const float4& v, long long n) {
-#pragma unroll
-      for (int j = 0; j < 4; ++j)
-        if (i0 + j < n && comp(v, j) > mv) {
-          mv = comp(v, j);
-          mi = static_cast<int>(i0 + j);
-        }
-    });
-    block_argmax(mv, mi, sh);
-    r.m = mv;
-  }
-  {
-    float s = 0.f;
-    int unused = 0;
-    for_row(z, V, [&](long long i0, const float4& v, long long n) {
-#pragma unroll
-      for (int j = 0; j < 4; ++j)
-        if (i0 + j < n) s += e_of(comp(v, j), r.m, scale);
-    });
-    block_sum2(s, unused, sh);
-    r.S = s;
-  }
+  row_stats(st, tiles, scale, ftab, fg, r.m, r.S, sh);
   const float target = top_p * r.S;
   // Invariant: mass(e >= lo) >= target > mass(e >= hi) = mass_hi; the
   // candidates are the elements with key in [lo, hi).
   uint32_t lo = 0u, hi = kInfKey;
-  float mass_hi = 0.f;
+  float mass_hi = 0.f, gt = 0.f;
+  int eq = 0;
+  bool resolved = false;
   if (top_p < 1.f) {
     const float* list = nullptr;  // candidates in shared memory, once they fit
     int n_list = 0;
-    // Each pass at least halves hi - lo (< 2^31), so 32 passes always suffice.
-    for (int pass = 0; pass < 40 && hi - lo > 1u; ++pass) {
-      const uint32_t mid = lo + (hi - lo) / 2u;
+    // Each pass at least halves hi - lo (< 2^31), so 33 passes always suffice.
+    for (int pass = 0; pass < 40; ++pass) {
+      const uint32_t mid = pass == 0 ? kFirstMid : lo + (hi - lo) / 2u;
       PassStats ps;
       if (list == nullptr) {
-        for_row(z, V, [&](long long i0, const float4& v, long long n) {
+        for_row(et, ftab, V, [&](long long i0, const float4& v, long long n) {
 #pragma unroll
           for (int j = 0; j < 4; ++j)
-            if (i0 + j < n) {
-              const float e = e_of(comp(v, j), r.m, scale);
-              ps.add(e, __float_as_uint(e), lo, mid, hi);
-            }
+            if (i0 + j < n) ps.add(comp(v, j), lo, mid, hi);
         });
       } else {
-        for (int i = threadIdx.x; i < n_list; i += kThreads) {
-          const float e = list[i];
-          ps.add(e, __float_as_uint(e), lo, mid, hi);
-        }
+        for (int i = threadIdx.x; i < n_list; i += kThreads) ps.add(list[i], lo, mid, hi);
       }
       reduce_pass(ps, sh);
       int side, cnt;
@@ -292,31 +345,34 @@ __device__ RowNucleus nucleus(const float* z, long long V, float scale, float to
         lo = old_lo;
         break;
       }
-      if (hi - lo <= 1u) break;
+      if (hi - lo <= 1u) {  // one key left: the candidates are the ties at b
+        gt = mass_hi;
+        eq = cnt;
+        resolved = true;
+        break;
+      }
+      const bool finish = cnt <= kFinish;
       // Compact the survivors (keys in the new [lo, hi)) when that pays.
-      const bool from_row = list == nullptr && cnt <= cap;
-      const bool shrink = list != nullptr && 2 * cnt <= n_list;
-      if (from_row || shrink) {
+      if ((list == nullptr && cnt <= kSpecListCap) ||
+          (list != nullptr && (2 * cnt <= n_list || (finish && cnt < n_list)))) {
         float* dst = list == listA ? listB : listA;
         warp_bases(side, sh);
         int run = sh.wbase[warp_id()];
-        if (from_row) {
-          for_row(z, V, [&](long long i0, const float4& v, long long n) {
-            float e[4];
+        if (list == nullptr) {
+          for_row(et, ftab, V, [&](long long i0, const float4& v, long long n) {
             int k = 0;
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
-              e[j] = e_of(comp(v, j), r.m, scale);
-              const uint32_t key = __float_as_uint(e[j]);
-              const bool keep = i0 + j < n && key >= lo && key < hi;
-              k += keep;
-              if (!keep) e[j] = -1.f;
+              const uint32_t key = __float_as_uint(comp(v, j));
+              k += i0 + j < n && key >= lo && key < hi;
             }
             const int incl = warp_incl_scan(k);
             int at = run + incl - k;
 #pragma unroll
-            for (int j = 0; j < 4; ++j)
-              if (e[j] >= 0.f && at < cnt) dst[at++] = e[j];
+            for (int j = 0; j < 4; ++j) {
+              const uint32_t key = __float_as_uint(comp(v, j));
+              if (i0 + j < n && key >= lo && key < hi && at < cnt) dst[at++] = comp(v, j);
+            }
             run += __shfl_sync(0xffffffffu, incl, 31);
           });
         } else {
@@ -339,22 +395,30 @@ __device__ RowNucleus nucleus(const float* z, long long V, float scale, float to
         list = dst;
         n_list = cnt;
       }
+      if (finish && list != nullptr && n_list == cnt) {
+        finish_exact(list, n_list, target, mass_hi, lo, lo, gt, eq, sh);
+        resolved = true;
+        break;
+      }
     }
   }
   r.b = __uint_as_float(lo);
-  // Mass strictly above b, and the tokens tied at b.
-  float gt = 0.f;
-  int eq = 0;
-  for_row(z, V, [&](long long i0, const float4& v, long long n) {
+  if (!resolved) {  // top_p = 1, or the rounding exit: one more pass over the row
+    float g = 0.f;
+    int q = 0;
+    for_row(et, ftab, V, [&](long long i0, const float4& v, long long n) {
 #pragma unroll
-    for (int j = 0; j < 4; ++j)
-      if (i0 + j < n) {
-        const float e = e_of(comp(v, j), r.m, scale);
-        if (e > r.b) gt += e;
-        else if (e == r.b) ++eq;
-      }
-  });
-  block_sum2(gt, eq, sh);
+      for (int j = 0; j < 4; ++j)
+        if (i0 + j < n) {
+          const float e = comp(v, j);
+          if (e > r.b) g += e;
+          else if (e == r.b) ++q;
+        }
+    });
+    block_sum2(g, q, sh);
+    gt = g;
+    eq = q;
+  }
   r.eq = eq;
   int c = eq;
   if (top_p < 1.f && r.b > 0.f) {
@@ -368,9 +432,9 @@ __device__ RowNucleus nucleus(const float* z, long long V, float scale, float to
 
 // Nucleus probability of token x (block-wide: when x is tied at the boundary
 // and only some ties are kept, its rank among them is counted).
-__device__ float prob_of(const float* z, long long V, float scale, const RowNucleus& n, int x,
-                         Shared& sh) {
-  const float e = e_of(z[x], n.m, scale);
+__device__ float prob_of(const float* et, const float* ftab, long long V, const RowNucleus& n,
+                         int x, Shared& sh) {
+  const float e = et[x] * ftab[x / kGemmBN];
   bool member = e > n.b;
   if (e == n.b) {
     if (n.c >= n.eq) {
@@ -378,10 +442,10 @@ __device__ float prob_of(const float* z, long long V, float scale, const RowNucl
     } else {
       float unused = 0.f;
       int below = 0;
-      for_row(z, V, [&](long long i0, const float4& v, long long cnt) {
+      for_row(et, ftab, V, [&](long long i0, const float4& v, long long cnt) {
 #pragma unroll
         for (int j = 0; j < 4; ++j)
-          if (i0 + j < x && i0 + j < cnt && e_of(comp(v, j), n.m, scale) == n.b) ++below;
+          if (i0 + j < x && i0 + j < cnt && comp(v, j) == n.b) ++below;
       });
       block_sum2(unused, below, sh);
       member = below < n.c;
@@ -411,42 +475,32 @@ __device__ __forceinline__ RowNucleus load_state(const float* st) {
 }
 
 __global__ void __launch_bounds__(kThreads, 2) spec_position_kernel(const SpecParams p) {
-  extern __shared__ __align__(16) float lists[];
+  extern __shared__ __align__(16) float smem[];
   __shared__ Shared sh;
+  float* ftab = smem;
+  float* listA = smem + kSpecMaxTiles;
+  float* listB = listA + kSpecListCap;
   const int G1 = p.gamma + 1;
   const int b = blockIdx.x / G1, i = blockIdx.x % G1;
   const long long pos_v = static_cast<long long>(b) * G1 + i;
-  const float* zv = p.zv + pos_v * p.ldz;
-  if (p.greedy) {
-    float mv = -INFINITY;
-    int mi = 0;
-    for_row(zv, p.V, [&](long long i0, const float4& v, long long n) {
-#pragma unroll
-      for (int j = 0; j < 4; ++j)
-        if (i0 + j < n && comp(v, j) > mv) {
-          mv = comp(v, j);
-          mi = static_cast<int>(i0 + j);
-        }
-    });
-    block_argmax(mv, mi, sh);
-    if (threadIdx.x == 0) {
-      p.tok[pos_v] = mi;
-      p.acc[pos_v] = i < p.gamma && p.draft[static_cast<long long>(b) * p.gamma + i] == mi;
-    }
-    return;
-  }
-  const RowNucleus np = nucleus(zv, p.V, p.scale, p.top_p, lists, lists + p.cap, p.cap, sh);
+  const long long sld = 2LL * p.tiles;
+  const float* ev = p.ev + pos_v * p.ldz;
+  const RowNucleus np = nucleus(ev, p.stats_v + pos_v * sld, p.f_v + pos_v * p.tiles, p.V,
+                                p.tiles, p.scale, p.top_p, ftab, listA, listB, sh);
   if (threadIdx.x == 0) store_state(p.state_v + pos_v * kSpecStateWords, np);
   if (i == p.gamma) return;
+  const int x = p.draft[static_cast<long long>(b) * p.gamma + i];
+  float px = 0.f;
+  if (x >= 0 && x < p.V) px = prob_of(ev, ftab, p.V, np, x, sh);
+  __syncthreads();  // ftab is rewritten for the draft row
   const long long pos_d = static_cast<long long>(b) * p.gamma + i;
-  const float* zd = p.zd + pos_d * p.ldz;
-  const RowNucleus nq = nucleus(zd, p.V, p.scale, p.top_p, lists, lists + p.cap, p.cap, sh);
+  const float* ed = p.ed + pos_d * p.ldz;
+  const RowNucleus nq = nucleus(ed, p.stats_d + pos_d * sld, p.f_d + pos_d * p.tiles, p.V,
+                                p.tiles, p.scale, p.top_p, ftab, listA, listB, sh);
   if (threadIdx.x == 0) store_state(p.state_d + pos_d * kSpecStateWords, nq);
-  const int x = p.draft[pos_d];
   int ok = 0;
   if (x >= 0 && x < p.V) {
-    const float qx = prob_of(zd, p.V, p.scale, nq, x, sh);
-    const float px = prob_of(zv, p.V, p.scale, np, x, sh);
+    const float qx = prob_of(ed, ftab, p.V, nq, x, sh);
     ok = qx > 0.f && p.u[pos_v * 2] * qx < px;
   }
   if (threadIdx.x == 0) p.acc[pos_v] = ok;
@@ -467,10 +521,17 @@ __device__ __forceinline__ Segment my_segment(long long V) {
 // Nucleus probabilities of the lane's 4 elements from i0 in one step of a
 // segment ending at `end`; `tie_run` (warp-uniform) counts the ties at b
 // before this step in index order.
-__device__ __forceinline__ void probs4(const float* z, const RowNucleus& n, float scale,
+__device__ __forceinline__ void probs4(const float* et, const float* ftab, const RowNucleus& n,
                                        long long i0, long long end, int& tie_run, float (&pr)[4]) {
   float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-  if (i0 < end) v = __ldg(reinterpret_cast<const float4*>(z + i0));
+  if (i0 < end) {
+    v = __ldg(reinterpret_cast<const float4*>(et + i0));
+    const float fm = ftab[i0 / kGemmBN];
+    v.x *= fm;
+    v.y *= fm;
+    v.z *= fm;
+    v.w *= fm;
+  }
   const float inv = 1.f / n.kept;
   float e[4];
   bool valid[4];
@@ -478,7 +539,7 @@ __device__ __forceinline__ void probs4(const float* z, const RowNucleus& n, floa
 #pragma unroll
   for (int j = 0; j < 4; ++j) {
     valid[j] = i0 + j < end;
-    e[j] = e_of(comp(v, j), n.m, scale);
+    e[j] = comp(v, j);
     ties += valid[j] && e[j] == n.b;
   }
   if (n.c >= n.eq) {
@@ -498,14 +559,16 @@ __device__ __forceinline__ void probs4(const float* z, const RowNucleus& n, floa
 }
 
 // Ties at b in this warp's segment (the bases of the tie ranks).
-__device__ int segment_ties(const float* z, const RowNucleus& n, float scale, const Segment& sg) {
+__device__ int segment_ties(const float* et, const float* ftab, const RowNucleus& n,
+                            const Segment& sg) {
   int t = 0;
   for (long long base = sg.begin; base < sg.end; base += kStep) {
     const long long i0 = base + lane_id() * 4;
     if (i0 < sg.end) {
-      const float4 v = __ldg(reinterpret_cast<const float4*>(z + i0));
+      const float4 v = __ldg(reinterpret_cast<const float4*>(et + i0));
+      const float fm = ftab[i0 / kGemmBN];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) t += (i0 + j < sg.end) && e_of(comp(v, j), n.m, scale) == n.b;
+      for (int j = 0; j < 4; ++j) t += (i0 + j < sg.end) && comp(v, j) * fm == n.b;
     }
   }
   return static_cast<int>(__reduce_add_sync(0xffffffffu, static_cast<unsigned>(t)));
@@ -513,15 +576,16 @@ __device__ int segment_ties(const float* z, const RowNucleus& n, float scale, co
 
 // sample(r, u) over r_v = max(0, p_v - q_v) (have_q) or r_v = p_v; -1 when r
 // is all zero.
-__device__ int sample(const float* zp, const RowNucleus& np, const float* zq, const RowNucleus& nq,
-                      bool have_q, float scale, long long V, float u, Shared& sh) {
+__device__ int sample(const float* ep, const float* fp, const RowNucleus& np, const float* eq,
+                      const float* fq, const RowNucleus& nq, bool have_q, long long V, float u,
+                      Shared& sh) {
   const Segment sg = my_segment(V);
   const int w = warp_id(), l = lane_id();
   int base_p = 0, base_q = 0;
   const bool tp = np.c < np.eq, tq = have_q && nq.c < nq.eq;
   if (tp || tq) {
-    const int cp = tp ? segment_ties(zp, np, scale, sg) : 0;
-    const int cq = tq ? segment_ties(zq, nq, scale, sg) : 0;
+    const int cp = tp ? segment_ties(ep, fp, np, sg) : 0;
+    const int cq = tq ? segment_ties(eq, fq, nq, sg) : 0;
     __syncthreads();
     if (l == 0) {
       sh.n[w][1] = cp;
@@ -539,8 +603,8 @@ __device__ int sample(const float* zp, const RowNucleus& np, const float* zq, co
     int rp = base_p, rq = base_q;
     for (long long base = sg.begin; base < sg.end; base += kStep) {
       float a[4], c[4] = {0.f, 0.f, 0.f, 0.f};
-      probs4(zp, np, scale, base + l * 4, sg.end, rp, a);
-      if (have_q) probs4(zq, nq, scale, base + l * 4, sg.end, rq, c);
+      probs4(ep, fp, np, base + l * 4, sg.end, rp, a);
+      if (have_q) probs4(eq, fq, nq, base + l * 4, sg.end, rq, c);
 #pragma unroll
       for (int j = 0; j < 4; ++j) mine += fmaxf(0.f, a[j] - c[j]);
     }
@@ -580,8 +644,8 @@ __device__ int sample(const float* zp, const RowNucleus& np, const float* zq, co
     for (long long base = sg.begin; base < sg.end && found < 0; base += kStep) {
       float a[4], c[4] = {0.f, 0.f, 0.f, 0.f};
       const long long i0 = base + l * 4;
-      probs4(zp, np, scale, i0, sg.end, rp, a);
-      if (have_q) probs4(zq, nq, scale, i0, sg.end, rq, c);
+      probs4(ep, fp, np, i0, sg.end, rp, a);
+      if (have_q) probs4(eq, fq, nq, i0, sg.end, rq, c);
       float r[4], lane_sum = 0.f;
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
@@ -610,26 +674,49 @@ __device__ int sample(const float* zp, const RowNucleus& np, const float* zq, co
   return sh.n[0][0];
 }
 
+// Greedy: the verifier's argmax of row `pos` from its tile (max, argmax) pairs.
+__device__ int row_argmax(const float* st, int tiles, Shared& sh) {
+  float mv = -INFINITY;
+  int mi = 0;
+  for (int t = threadIdx.x; t < tiles; t += kThreads)
+    if (st[2 * t] > mv) {
+      mv = st[2 * t];
+      mi = __float_as_int(st[2 * t + 1]);
+    }
+  block_argmax(mv, mi, sh);
+  return mi;
+}
+
 __global__ void __launch_bounds__(kThreads) spec_sample_kernel(const SpecParams p) {
   __shared__ Shared sh;
+  __shared__ float fp[kSpecMaxTiles], fq[kSpecMaxTiles];
   const int b = blockIdx.x, G1 = p.gamma + 1;
-  int k = 0;
-  while (k < p.gamma && p.acc[static_cast<long long>(b) * G1 + k]) ++k;
-  const long long pos_v = static_cast<long long>(b) * G1 + k;
-  int next;
+  const long long sld = 2LL * p.tiles;
+  int k = 0, next = -1;
   if (p.greedy) {
-    next = p.tok[pos_v];
+    for (;; ++k) {
+      const int best = row_argmax(p.stats_v + (static_cast<long long>(b) * G1 + k) * sld, p.tiles, sh);
+      if (k == p.gamma || p.draft[static_cast<long long>(b) * p.gamma + k] != best) {
+        next = best;
+        break;
+      }
+    }
   } else {
+    while (k < p.gamma && p.acc[static_cast<long long>(b) * G1 + k]) ++k;
+    const long long pos_v = static_cast<long long>(b) * G1 + k;
     const RowNucleus np = load_state(p.state_v + pos_v * kSpecStateWords);
-    const float* zv = p.zv + pos_v * p.ldz;
+    const float* ev = p.ev + pos_v * p.ldz;
+    for (int t = threadIdx.x; t < p.tiles; t += kThreads) fp[t] = p.f_v[pos_v * p.tiles + t];
     const float u = p.u[pos_v * 2 + 1];
-    next = -1;
     if (k < p.gamma) {
       const long long pos_d = static_cast<long long>(b) * p.gamma + k;
       const RowNucleus nq = load_state(p.state_d + pos_d * kSpecStateWords);
-      next = sample(zv, np, p.zd + pos_d * p.ldz, nq, true, p.scale, p.V, u, sh);
+      for (int t = threadIdx.x; t < p.tiles; t += kThreads) fq[t] = p.f_d[pos_d * p.tiles + t];
+      __syncthreads();
+      next = sample(ev, fp, np, p.ed + pos_d * p.ldz, fq, nq, true, p.V, u, sh);
     }
-    if (next < 0) next = sample(zv, np, zv, np, false, p.scale, p.V, u, sh);
+    __syncthreads();
+    if (next < 0) next = sample(ev, fp, np, ev, fp, np, false, p.V, u, sh);
     if (next < 0) next = static_cast<int>(p.V - 1);  // unreachable: the maximum has e = 1
   }
   if (threadIdx.x == 0) {
@@ -642,14 +729,13 @@ __global__ void __launch_bounds__(kThreads) spec_sample_kernel(const SpecParams 
 
 cudaError_t setup_spec_kernels() {
   return cudaFuncSetAttribute(spec_position_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              static_cast<int>(2 * kSpecListCap * sizeof(float)));
+                              static_cast<int>(kPositionSmem));
 }
 
 cudaError_t launch_spec_position(const SpecParams& p, cudaStream_t s) {
   const long long blocks = static_cast<long long>(p.B) * (p.gamma + 1);
-  if (blocks <= 0) return cudaSuccess;
-  const size_t smem = p.greedy ? 0 : 2 * static_cast<size_t>(p.cap) * sizeof(float);
-  spec_position_kernel<<<static_cast<unsigned>(blocks), kThreads, smem, s>>>(p);
+  if (blocks <= 0 || p.greedy) return cudaSuccess;
+  spec_position_kernel<<<static_cast<unsigned>(blocks), kThreads, kPositionSmem, s>>>(p);
   return cudaGetLastError();
 }
 

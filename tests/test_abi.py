@@ -114,9 +114,13 @@ def test_spec_verify_validation_without_gpu(lib):
     assert call(B.spec_problem(4, 2, 100, 64, 64), u=0) == B.MLS_ERR_ARG
     assert call(B.spec_problem(4, 2, 100, 64, 64), size=1024) == B.MLS_ERR_WORKSPACE
     assert call(B.spec_problem(0, 2, 100, 64, 64)) == B.MLS_OK  # nothing to do
-    # sizes: logits rows padded to 4 floats; the draft's only when sampling
+    # sizes: sampling keeps a row of fp32 probabilities per verify position
+    # (padded to 4 floats); greedy keeps only per-tile maxima
     ldz = 4 * ((101 + 3) // 4)
     samp = B.mls_spec_workspace_size(B.spec_problem(4, 2, 101, 64, 64))
     greedy = B.mls_spec_workspace_size(B.spec_problem(4, 2, 101, 64, 64, greedy=True))
-    assert samp >= 4 * (4 * 3 + 4 * 2) * ldz and greedy >= 4 * 4 * 3 * ldz
-    assert samp - greedy >= 4 * 4 * 2 * ldz
+    assert samp - greedy >= 4 * (4 * 3 + 4 * 2) * ldz
+    assert 0 < greedy < 4 * 4 * 3 * ldz
+    # sampling keeps a per-tile table in shared memory: V <= 4096 tiles of 256
+    assert call(B.spec_problem(4, 2, 4096 * 256 + 1, 64, 64)) == B.MLS_ERR_UNSUPPORTED
+    assert B.mls_spec_workspace_size(B.spec_problem(4, 2, 4096 * 256 + 1, 64, 64, greedy=True)) > 0
