@@ -577,7 +577,7 @@ def spec_run(args, dev, pk):
         }
         if not greedy:
             # the selection kernels against one read of every probability row
-            sel_ms = (kp["spec_position"][1] + kp["spec_sample"][1]) / n
+            sel_ms = (kp["spec_rows"][1] + kp["spec_sample"][1]) / n
             out[mode]["selection_gbs_one_read"] = (Pv + Pd) * wl.V * 4 / (sel_ms / 1e3) / 1e9
     return out
 

@@ -187,7 +187,8 @@ int mls_junction_bwd(int64_t T, int32_t d_prev, int32_t d_next, int32_t in_dtype
  *   ws           workspace of mls_spec_workspace_size(p) bytes, 256-byte aligned;
  *                when sampling it holds an fp32 row of unnormalised
  *                probabilities per verify position (greedy: per-tile maxima only).
- * Sampling supports V <= 4096 * 256 (MLS_ERR_UNSUPPORTED above); greedy any V.
+ * Sampling supports V <= 4096 * 256 and gamma <= 1024 (MLS_ERR_UNSUPPORTED
+ * beyond); greedy has neither limit.
  * Logits are fp32 sums of the stored-type products; probabilities are fp32, so a
  * decision that the exact values leave within rounding of a threshold may go
  * either way.  Asynchronous; returns 0 or a negative MLS_ERR_* code (nothing

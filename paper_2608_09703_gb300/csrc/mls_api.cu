@@ -810,7 +810,7 @@ namespace {
 struct SpecPlan {
   long long Pd = 0, Pv = 0, ldz = 0, tiles = 0;
   size_t off_ev = 0, off_ed = 0, off_sv = 0, off_sd = 0, off_fv = 0, off_fd = 0;
-  size_t off_stv = 0, off_std = 0, off_acc = 0, total = 0;
+  size_t off_stv = 0, off_std = 0, total = 0;
 };
 
 int spec_validate(const mls_spec_problem* p) {
@@ -825,7 +825,8 @@ int spec_validate(const mls_spec_problem* p) {
     if ((static_cast<long long>(p->d_draft) * elt) % 16 != 0) return MLS_ERR_UNSUPPORTED;
     if (!(p->temperature > 0.f) || !std::isfinite(p->temperature)) return MLS_ERR_ARG;
     if (!(p->top_p > 0.f && p->top_p <= 1.f)) return MLS_ERR_ARG;
-    if (p->V > static_cast<long long>(kSpecMaxTiles) * kGemmBN) return MLS_ERR_UNSUPPORTED;
+    if (p->V > static_cast<long long>(kSpecMaxTiles) * kGemmBN || p->gamma > kSpecMaxGamma)
+      return MLS_ERR_UNSUPPORTED;
   }
   return MLS_OK;
 }
@@ -850,7 +851,6 @@ SpecPlan spec_plan(const mls_spec_problem* p) {
   take(pl.off_fd, sizeof(float) * static_cast<size_t>(pl.Pd) * pl.tiles);
   take(pl.off_sv, sizeof(float) * kSpecStateWords * static_cast<size_t>(pl.Pv));
   take(pl.off_sd, sizeof(float) * kSpecStateWords * static_cast<size_t>(pl.Pd));
-  take(pl.off_acc, sizeof(int) * static_cast<size_t>(pl.Pv));
   pl.total = o;
   return pl;
 }
@@ -905,7 +905,6 @@ extern "C" int mls_spec_verify(const mls_spec_problem* p, const void* H_draft, c
   sp.u = uniforms;
   sp.state_v = at(pl.off_sv);
   sp.state_d = at(pl.off_sd);
-  sp.acc = reinterpret_cast<int*>(wsb + pl.off_acc);
   sp.n_accepted = n_accepted;
   sp.next_token = next_token;
 
@@ -950,8 +949,7 @@ extern "C" int mls_spec_verify(const mls_spec_problem* p, const void* H_draft, c
   g.status = dev->status;
   const int grid = 2 * (tiles < dev->gemm_pairs ? tiles : dev->gemm_pairs);
   if ((rc = timed("spec_logits", s, [&] { return launch_gemm_kk(g, tf32, grid, s); }))) return rc;
-  if (!p->greedy &&
-      (rc = timed("spec_position", s, [&] { return launch_spec_position(sp, s); })))
+  if (!p->greedy && (rc = timed("spec_rows", s, [&] { return launch_spec_rows(sp, s); })))
     return rc;
   return timed("spec_sample", s, [&] { return launch_spec_sample(sp, s); });
 }

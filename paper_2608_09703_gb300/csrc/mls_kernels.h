@@ -186,8 +186,9 @@ cudaError_t launch_junction_bwd(const JunctionParams& p, bool fp32, cudaStream_t
 // relative to the maximum m_t of v's column tile, and per tile (m_t, sum of e_t)
 // (kEpiSoftmax); greedy verification only needs per tile (m_t, argmax) (kEpiArgmax).
 constexpr int kSpecStateWords = 8;    // per row: max, b, kept mass, c, ties, sum (+2 spare)
-constexpr int kSpecListCap = 8192;    // candidates per shared-memory list (two lists)
+constexpr int kSpecListCap = 4096;    // candidates per shared-memory list (two lists)
 constexpr int kSpecMaxTiles = 4096;   // column tiles of a row (V <= 4096 * kGemmBN when sampling)
+constexpr int kSpecMaxGamma = 1024;   // drafted tokens per sequence when sampling
 
 struct SpecParams {
   long long V, ldz;
@@ -206,12 +207,11 @@ struct SpecParams {
   const float* u;                // [B][gamma + 1][2]
   float* state_d;                // [B * gamma][kSpecStateWords]
   float* state_v;                // [B * (gamma + 1)][kSpecStateWords]
-  int* acc;                      // [B * (gamma + 1)] accepted flag per position
   int* n_accepted;               // [B]
   int* next_token;               // [B]
 };
 cudaError_t setup_spec_kernels();
-cudaError_t launch_spec_position(const SpecParams& p, cudaStream_t s);
+cudaError_t launch_spec_rows(const SpecParams& p, cudaStream_t s);
 cudaError_t launch_spec_sample(const SpecParams& p, cudaStream_t s);
 
 // ------------------------------------------------------------------ reductions

@@ -16,17 +16,18 @@
 // only (m_t, argmax_t).  Here, with m = max_t m_t and f_t = 2^((m_t - m) log2(e)/T),
 // every token's unnormalised probability is e[v] = e_t[v] f_t (<= 1) and
 // S = sum_t sum_t f_t:
-//   spec_position_kernel (one CTA per position, sampling only) finds each
-//     row's nucleus: the boundary value b = the largest e with
-//     mass(e' >= b) >= top_p S, by bisection over the bit patterns of e
-//     (non-negative floats order like their bits), each pass narrowing the
-//     bracket to its surviving keys; survivors are compacted into shared memory
-//     once they fit and the last <= 256 are resolved exactly; then the c
-//     lowest-index tokens with e == b that the cumulative needs.  It then
-//     decides acceptance of the drafted token of that position.
-//   spec_sample_kernel (one CTA per sequence) takes the first rejection and
-//     samples by inverse CDF in index order, each warp walking a contiguous
-//     segment of the vocabulary; for greedy it reduces the tile argmaxes.
+//   spec_row_kernel (one CTA per row, sampling only) finds the row's nucleus:
+//     the boundary value b = the largest e with mass(e' >= b) >= top_p S, by
+//     bisection over the bit patterns of e (non-negative floats order like
+//     their bits).  The first pass splits at 2^-8 of the maximum and keeps the
+//     few tokens above it in shared memory; later passes narrow the bracket,
+//     compacting survivors into shared memory once they fit, and the last
+//     <= 256 are resolved exactly.  Then the c lowest-index tokens with e == b
+//     that the cumulative needs.
+//   spec_sample_kernel (one CTA per sequence) decides acceptance of every
+//     drafted token from the rows' nucleus states, takes the first rejection
+//     and samples by inverse CDF in index order; for greedy it reduces the
+//     tile argmaxes.
 // Every reduction has a fixed order, so a call is deterministic.
 #include "mls_device.cuh"
 #include "mls_kernels.h"
@@ -34,22 +35,31 @@
 namespace mls {
 namespace {
 
-constexpr int kThreads = 512;
+constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
 constexpr int kStep = 128;              // elements one warp covers per float4 step
-constexpr int kUnroll = 4;              // independent float4 loads in flight per lane
+constexpr int kUnroll = 6;              // independent float4 loads in flight per lane
 constexpr int kFinish = 256;            // candidates resolved exactly
-constexpr uint32_t kInfKey = 0x7f800000u;
-constexpr uint32_t kFirstMid = 0x3b800000u;  // 2^-8: first split of the bracket [0, inf)
-constexpr size_t kPositionSmem = sizeof(float) * (kSpecMaxTiles + 2 * kSpecListCap);
+constexpr uint32_t kOneKey = 0x3f800000u;     // bit pattern of 1.0f
+constexpr uint32_t kFirstMid = 0x3b800000u;   // 2^-8
+constexpr uint32_t kSecondMid = 0x37800000u;  // 2^-16
 static_assert(kFinish <= kThreads, "one candidate per thread in the exact finish");
 
-struct Shared {
-  float f[kWarps][2];
-  int n[kWarps][3];
-  uint32_t k[kWarps][4];
-  int wbase[kWarps];
+// Per-warp partials of a block reduction (f, n, k) and the combined results
+// (rf, rn, rk) that warp 0 writes for everyone.
+template <int NW>
+struct SharedT {
+  float f[NW][2];
+  int n[NW][3];
+  uint32_t k[NW][4];
+  int wbase[NW];
+  int wcnt[NW];
+  float rf[2];
+  int rn[3];
+  uint32_t rk[4];
 };
+using Shared = SharedT<kWarps>;
+constexpr int kSampleWarps = 32;  // the per-sequence sampler runs 1024 threads
 
 __device__ __forceinline__ int lane_id() { return threadIdx.x & 31; }
 __device__ __forceinline__ int warp_id() { return threadIdx.x >> 5; }
@@ -84,34 +94,58 @@ __device__ __forceinline__ float comp(const float4& v, int j) {
   return j == 0 ? v.x : j == 1 ? v.y : j == 2 ? v.z : v.w;
 }
 
-// Block-wide (max value, lowest index attaining it).
-__device__ void block_argmax(float& v, int& idx, Shared& sh) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const float ov = __shfl_xor_sync(0xffffffffu, v, o);
-    const int oi = __shfl_xor_sync(0xffffffffu, idx, o);
-    if (ov > v || (ov == v && oi < idx)) {
-      v = ov;
-      idx = oi;
-    }
+// Prefetches a row of `bytes` (a multiple of 16) into L2 in 16 KB pieces, one
+// per thread of the first warps.
+__device__ __forceinline__ void prefetch_row(const float* row, long long bytes) {
+  constexpr long long kPiece = 16384;
+  const long long off = static_cast<long long>(threadIdx.x) * kPiece;
+  if (off < bytes)
+    prefetch_l2_bulk(reinterpret_cast<const char*>(row) + off,
+                     static_cast<uint32_t>(bytes - off < kPiece ? bytes - off : kPiece));
+}
+
+// Block reductions: each warp reduces by a butterfly, lane 0 parks the
+// warp's partial, warp 0 combines the 16 partials by a butterfly and parks the
+// result for every thread.  Fixed order throughout.
+__device__ __forceinline__ void argmax_step(float& v, int& idx, float ov, int oi) {
+  if (ov > v || (ov == v && oi < idx)) {
+    v = ov;
+    idx = oi;
   }
+}
+
+// (max value, lowest index attaining it).
+template <int NW>
+__device__ void block_argmax(float& v, int& idx, SharedT<NW>& sh) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1)
+    argmax_step(v, idx, __shfl_xor_sync(0xffffffffu, v, o), __shfl_xor_sync(0xffffffffu, idx, o));
   __syncthreads();
   if (lane_id() == 0) {
     sh.f[warp_id()][0] = v;
     sh.n[warp_id()][0] = idx;
   }
   __syncthreads();
-  v = sh.f[0][0];
-  idx = sh.n[0][0];
-  for (int w = 1; w < kWarps; ++w)
-    if (sh.f[w][0] > v || (sh.f[w][0] == v && sh.n[w][0] < idx)) {
-      v = sh.f[w][0];
-      idx = sh.n[w][0];
+  if (warp_id() == 0) {
+    const int l = lane_id();
+    float wv = l < NW ? sh.f[l][0] : -INFINITY;
+    int wi = l < NW ? sh.n[l][0] : 0x7fffffff;
+#pragma unroll
+    for (int o = NW / 2; o > 0; o >>= 1)
+      argmax_step(wv, wi, __shfl_xor_sync(0xffffffffu, wv, o), __shfl_xor_sync(0xffffffffu, wi, o));
+    if (l == 0) {
+      sh.rf[0] = wv;
+      sh.rn[0] = wi;
     }
+  }
+  __syncthreads();
+  v = sh.rf[0];
+  idx = sh.rn[0];
 }
 
-// Block sums of a float and an int (fixed order: lanes by a butterfly, warps 0..15).
-__device__ void block_sum2(float& f, int& n, Shared& sh) {
+// Sums of a float and an int.
+template <int NW>
+__device__ void block_sum2(float& f, int& n, SharedT<NW>& sh) {
   f = warp_sum(f);
   n = static_cast<int>(__reduce_add_sync(0xffffffffu, static_cast<unsigned>(n)));
   __syncthreads();
@@ -120,22 +154,37 @@ __device__ void block_sum2(float& f, int& n, Shared& sh) {
     sh.n[warp_id()][0] = n;
   }
   __syncthreads();
-  f = 0.f;
-  n = 0;
-  for (int w = 0; w < kWarps; ++w) {
-    f += sh.f[w][0];
-    n += sh.n[w][0];
+  if (warp_id() == 0) {
+    const int l = lane_id();
+    float wf = l < NW ? sh.f[l][0] : 0.f;
+    int wn = l < NW ? sh.n[l][0] : 0;
+#pragma unroll
+    for (int o = NW / 2; o > 0; o >>= 1) {
+      wf += __shfl_xor_sync(0xffffffffu, wf, o);
+      wn += __shfl_xor_sync(0xffffffffu, wn, o);
+    }
+    if (l == 0) {
+      sh.rf[0] = wf;
+      sh.rn[0] = wn;
+    }
   }
+  __syncthreads();
+  f = sh.rf[0];
+  n = sh.rn[0];
 }
 
-__device__ uint32_t block_max_u(uint32_t v, Shared& sh) {
+template <int NW>
+__device__ uint32_t block_max_u(uint32_t v, SharedT<NW>& sh) {
   v = __reduce_max_sync(0xffffffffu, v);
   __syncthreads();
   if (lane_id() == 0) sh.k[warp_id()][0] = v;
   __syncthreads();
-  uint32_t r = 0;
-  for (int w = 0; w < kWarps; ++w) r = max(r, sh.k[w][0]);
-  return r;
+  if (warp_id() == 0) {
+    const uint32_t w = __reduce_max_sync(0xffffffffu, lane_id() < NW ? sh.k[lane_id()][0] : 0u);
+    if (lane_id() == 0) sh.rk[0] = w;
+  }
+  __syncthreads();
+  return sh.rk[0];
 }
 
 // Per-row softmax statistics from the per-tile ones: m, S and f_t (into the
@@ -163,10 +212,10 @@ __device__ void row_stats(const float* st, int tiles, float scale, float* ftab, 
 // `f(i0, e4, V)` gets the lane's 4 consecutive elements from index i0 (those
 // at or past V are not meaningful).  The loop is warp-uniform, so f may use
 // warp collectives.  Rows are 16-byte aligned and padded to 4 elements.
-template <typename F>
+template <int NW, typename F>
 __device__ __forceinline__ void for_row(const float* et, const float* ftab, long long V, F&& f) {
   const int l = lane_id();
-  constexpr long long kStride = static_cast<long long>(kWarps) * kStep;
+  constexpr long long kStride = static_cast<long long>(NW) * kStep;
   for (long long base = static_cast<long long>(warp_id()) * kStep; base < V;
        base += kUnroll * kStride) {
     float4 v[kUnroll];
@@ -192,27 +241,159 @@ __device__ __forceinline__ void for_row(const float* et, const float* ftab, long
 }
 
 // Statistics of one bisection pass over the candidates with key in [lo, hi),
-// split at mid: mass and count of the upper side, count of the lower side,
-// and the smallest and largest key on each side.
+// split at mid.  With d = key - lo (unsigned), mo = mid - lo, w = hi - lo and
+// wm = w - mo: the lower side is d < mo, the upper side d - mo < wm.  Kept:
+// mass and count of the upper side, count of the lower side and, when
+// tracked, the smallest and largest key on each side.
 struct PassStats {
   float mass_ge = 0.f;
   int cnt_ge = 0, cnt_lt = 0;
   uint32_t min_ge = 0xffffffffu, max_ge = 0u, min_lt = 0xffffffffu, max_lt = 0u;
-  __device__ __forceinline__ void add(float e, uint32_t lo, uint32_t mid, uint32_t hi) {
+  template <bool kTrack>
+  __device__ __forceinline__ void add(float e, uint32_t lo, uint32_t mo, uint32_t wm) {
     const uint32_t key = __float_as_uint(e);
-    if (key < lo || key >= hi) return;
-    if (key >= mid) {
-      mass_ge += e;
-      ++cnt_ge;
-      min_ge = min(min_ge, key);
-      max_ge = max(max_ge, key);
-    } else {
-      ++cnt_lt;
-      min_lt = min(min_lt, key);
-      max_lt = max(max_lt, key);
+    const uint32_t d = key - lo;
+    const bool lt = d < mo, ge = d - mo < wm;
+    cnt_lt += lt;
+    cnt_ge += ge;
+    mass_ge += ge ? e : 0.f;
+    if (kTrack) {
+      if (lt) {
+        min_lt = min(min_lt, key);
+        max_lt = max(max_lt, key);
+      }
+      if (ge) {
+        min_ge = min(min_ge, key);
+        max_ge = max(max_ge, key);
+      }
     }
   }
 };
+
+// One bisection pass over a whole row (e = e_t f_t), warps taking 128-token
+// steps w, w + 16, ..., kUnroll steps per iteration; only the row's last
+// float4 can be partial.
+template <bool kTrack>
+__device__ __forceinline__ void row_pass(const float* et, const float* ftab, int V, uint32_t lo,
+                                         uint32_t mo, uint32_t wm, PassStats& ps) {
+  const int l = lane_id();
+  constexpr int kStride = kWarps * kStep;
+  for (int base = warp_id() * kStep; base < V; base += kUnroll * kStride) {
+    float4 v[kUnroll];
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const int i0 = base + u * kStride + l * 4;
+      v[u] = i0 < V ? __ldg(reinterpret_cast<const float4*>(et + i0)) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const int i0 = base + u * kStride + l * 4;
+      if (i0 < V) {
+        const float fm = ftab[static_cast<unsigned>(i0) / kGemmBN];
+        const float e0 = v[u].x * fm, e1 = v[u].y * fm, e2 = v[u].z * fm, e3 = v[u].w * fm;
+        ps.add<kTrack>(e0, lo, mo, wm);
+        if (i0 + 4 <= V) {
+          ps.add<kTrack>(e1, lo, mo, wm);
+          ps.add<kTrack>(e2, lo, mo, wm);
+          ps.add<kTrack>(e3, lo, mo, wm);
+        } else {
+          if (i0 + 1 < V) ps.add<kTrack>(e1, lo, mo, wm);
+          if (i0 + 2 < V) ps.add<kTrack>(e2, lo, mo, wm);
+        }
+      }
+    }
+  }
+}
+
+// The first bisection pass over a whole row: the split at 2^-8 of the maximum
+// over [0, 1].  Mass and count of the upper side, smallest and largest key of
+// the lower side; the few upper-side tokens are also appended, in this warp's
+// visiting order, to its own region of kSpecListCap / kWarps slots of
+// `regions` (wrun counts them, also past the region's end).
+constexpr int kRegion = kSpecListCap / kWarps;
+__device__ __forceinline__ void first_pass(const float* et, const float* ftab, int V, float* regions,
+                                           PassStats& ps, int& wrun) {
+  const int l = lane_id();
+  constexpr int kStride = kWarps * kStep;
+  float* reg = regions + warp_id() * kRegion;
+  wrun = 0;
+  for (int base = warp_id() * kStep; base < V; base += kUnroll * kStride) {
+    float4 v[kUnroll];
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const int i0 = base + u * kStride + l * 4;
+      v[u] = i0 < V ? __ldg(reinterpret_cast<const float4*>(et + i0)) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const int i0 = base + u * kStride + l * 4;
+      const int nv = min(max(V - i0, 0), 4);
+      const float fm = nv > 0 ? ftab[static_cast<unsigned>(i0) / kGemmBN] : 0.f;
+      const float e[4] = {v[u].x * fm, v[u].y * fm, v[u].z * fm, v[u].w * fm};
+      bool ge[4];
+      int k = 0;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const uint32_t key = __float_as_uint(e[j]);
+        ge[j] = j < nv && key >= kFirstMid;
+        if (ge[j]) {
+          ps.mass_ge += e[j];
+          ++k;
+        } else if (j < nv) {
+          ps.min_lt = min(ps.min_lt, key);
+          ps.max_lt = max(ps.max_lt, key);
+        }
+      }
+      ps.cnt_ge += k;
+      if (__any_sync(0xffffffffu, k > 0)) {
+        const int incl = warp_incl_scan(k);
+        int at = wrun + incl - k;
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          if (ge[j]) {
+            if (at < kRegion) reg[at] = e[j];
+            ++at;
+          }
+        wrun += __shfl_sync(0xffffffffu, incl, 31);
+      }
+    }
+  }
+}
+
+// Writes the row's tokens with key in [lo, lo + w) to dst in warp order,
+// this warp from slot `run`, never past cnt.
+__device__ __forceinline__ void row_compact(const float* et, const float* ftab, int V, uint32_t lo,
+                                            uint32_t w, float* dst, int run, int cnt) {
+  const int l = lane_id();
+  constexpr int kStride = kWarps * kStep;
+  for (int base = warp_id() * kStep; base < V; base += kUnroll * kStride) {
+    float4 v[kUnroll];
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const int i0 = base + u * kStride + l * 4;
+      v[u] = i0 < V ? __ldg(reinterpret_cast<const float4*>(et + i0)) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const int i0 = base + u * kStride + l * 4;
+      const float fm = i0 < V ? ftab[static_cast<unsigned>(i0) / kGemmBN] : 0.f;
+      float e[4] = {v[u].x * fm, v[u].y * fm, v[u].z * fm, v[u].w * fm};
+      bool keep[4];
+      int k = 0;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        keep[j] = i0 + j < V && __float_as_uint(e[j]) - lo < w;
+        k += keep[j];
+      }
+      const int incl = warp_incl_scan(k);
+      int at = run + incl - k;
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (keep[j] && at < cnt) dst[at++] = e[j];
+      run += __shfl_sync(0xffffffffu, incl, 31);
+    }
+  }
+}
 
 // Block-wide combination; the per-warp counts stay in sh.n[w][1] (upper) and
 // sh.n[w][2] (lower) for the compaction that may follow.
@@ -237,17 +418,36 @@ __device__ void reduce_pass(PassStats& s, Shared& sh) {
     sh.k[w][3] = s.max_lt;
   }
   __syncthreads();
-  PassStats r;
-  for (int w = 0; w < kWarps; ++w) {
-    r.mass_ge += sh.f[w][0];
-    r.cnt_ge += sh.n[w][1];
-    r.cnt_lt += sh.n[w][2];
-    r.min_ge = min(r.min_ge, sh.k[w][0]);
-    r.max_ge = max(r.max_ge, sh.k[w][1]);
-    r.min_lt = min(r.min_lt, sh.k[w][2]);
-    r.max_lt = max(r.max_lt, sh.k[w][3]);
+  if (warp_id() == 0) {
+    const int l = lane_id();
+    const bool has = l < kWarps;
+    float m = has ? sh.f[l][0] : 0.f;
+#pragma unroll
+    for (int o = kWarps / 2; o > 0; o >>= 1) m += __shfl_xor_sync(full, m, o);
+    const unsigned cg = __reduce_add_sync(full, has ? static_cast<unsigned>(sh.n[l][1]) : 0u);
+    const unsigned cl = __reduce_add_sync(full, has ? static_cast<unsigned>(sh.n[l][2]) : 0u);
+    const uint32_t a = __reduce_min_sync(full, has ? sh.k[l][0] : 0xffffffffu);
+    const uint32_t b = __reduce_max_sync(full, has ? sh.k[l][1] : 0u);
+    const uint32_t c = __reduce_min_sync(full, has ? sh.k[l][2] : 0xffffffffu);
+    const uint32_t d = __reduce_max_sync(full, has ? sh.k[l][3] : 0u);
+    if (l == 0) {
+      sh.rf[0] = m;
+      sh.rn[1] = static_cast<int>(cg);
+      sh.rn[2] = static_cast<int>(cl);
+      sh.rk[0] = a;
+      sh.rk[1] = b;
+      sh.rk[2] = c;
+      sh.rk[3] = d;
+    }
   }
-  s = r;
+  __syncthreads();
+  s.mass_ge = sh.rf[0];
+  s.cnt_ge = sh.rn[1];
+  s.cnt_lt = sh.rn[2];
+  s.min_ge = sh.rk[0];
+  s.max_ge = sh.rk[1];
+  s.min_lt = sh.rk[2];
+  s.max_lt = sh.rk[3];
 }
 
 // After reduce_pass: each warp's first output slot when the survivors of
@@ -306,25 +506,69 @@ __device__ RowNucleus nucleus(const float* et, const float* st, float* fg, long 
   const float target = top_p * r.S;
   // Invariant: mass(e >= lo) >= target > mass(e >= hi) = mass_hi; the
   // candidates are the elements with key in [lo, hi).
-  uint32_t lo = 0u, hi = kInfKey;
+  uint32_t lo = 0u, hi = kOneKey + 1u;  // every e lies in [0, 1]
   float mass_hi = 0.f, gt = 0.f;
   int eq = 0;
   bool resolved = false;
   if (top_p < 1.f) {
     const float* list = nullptr;  // candidates in shared memory, once they fit
     int n_list = 0;
-    // Each pass at least halves hi - lo (< 2^31), so 33 passes always suffice.
-    for (int pass = 0; pass < 40; ++pass) {
-      const uint32_t mid = pass == 0 ? kFirstMid : lo + (hi - lo) / 2u;
+    bool done = false, probe2 = false;
+    // ---- first pass: split at 2^-8
+    {
       PassStats ps;
-      if (list == nullptr) {
-        for_row(et, ftab, V, [&](long long i0, const float4& v, long long n) {
-#pragma unroll
-          for (int j = 0; j < 4; ++j)
-            if (i0 + j < n) ps.add(comp(v, j), lo, mid, hi);
-        });
+      int wrun = 0;
+      first_pass(et, ftab, static_cast<int>(V), listA, ps, wrun);
+      if (lane_id() == 0) sh.wcnt[warp_id()] = wrun;
+      reduce_pass(ps, sh);  // its barriers also publish wcnt
+      int cnt;
+      if (ps.mass_ge >= target) {
+        cnt = ps.cnt_ge;
+        lo = kFirstMid;
+        // the upper side is in the warps' regions unless one overflowed
+        bool fits = true;
+        for (int w = 0; w < kWarps; ++w) fits = fits && sh.wcnt[w] <= kRegion;
+        if (fits) {
+          int at = 0;
+          for (int w = 0; w < warp_id(); ++w) at += sh.wcnt[w];
+          const float* reg = listA + warp_id() * kRegion;
+          for (int i = lane_id(); i < sh.wcnt[warp_id()]; i += 32) listB[at + i] = reg[i];
+          __syncthreads();
+          list = listB;
+          n_list = cnt;
+        }
       } else {
-        for (int i = threadIdx.x; i < n_list; i += kThreads) ps.add(list[i], lo, mid, hi);
+        cnt = static_cast<int>(V) - ps.cnt_ge;
+        mass_hi = ps.mass_ge;
+        lo = ps.min_lt;
+        hi = ps.max_lt + 1u;
+        probe2 = true;
+      }
+      if (cnt == 0) {  // only by rounding, with top_p within an ulp of 1
+        lo = 0u;
+        done = true;
+      } else if (list != nullptr && cnt <= kFinish) {
+        finish_exact(list, n_list, target, mass_hi, lo, lo, gt, eq, sh);
+        resolved = done = true;
+      } else if (hi - lo <= 1u) {
+        gt = mass_hi;
+        eq = cnt;
+        resolved = done = true;
+      }
+    }
+    // ---- then bisection: untracked passes over the row, tracked ones over a list
+    // Each pass at least halves hi - lo (< 2^30), so 32 passes always suffice.
+    for (int pass = 1; !done && pass < 40; ++pass) {
+      uint32_t mid = lo + (hi - lo) / 2u;
+      if (probe2 && lo < kSecondMid && kSecondMid < hi) mid = kSecondMid;  // probe 2^-16 next
+      probe2 = false;
+      const bool track = list != nullptr;
+      const uint32_t mo = mid - lo, wm = hi - mid;
+      PassStats ps;
+      if (list != nullptr) {
+        for (int i = threadIdx.x; i < n_list; i += kThreads) ps.add<true>(list[i], lo, mo, wm);
+      } else {
+        row_pass<false>(et, ftab, static_cast<int>(V), lo, mo, wm, ps);
       }
       reduce_pass(ps, sh);
       int side, cnt;
@@ -332,14 +576,22 @@ __device__ RowNucleus nucleus(const float* et, const float* st, float* fg, long 
       if (mass_hi + ps.mass_ge >= target) {
         side = 1;
         cnt = ps.cnt_ge;
-        lo = ps.min_ge;
-        hi = ps.max_ge + 1u;
+        if (track) {
+          lo = ps.min_ge;
+          hi = ps.max_ge + 1u;
+        } else {
+          lo = mid;
+        }
       } else {
         side = 2;
         cnt = ps.cnt_lt;
         mass_hi += ps.mass_ge;
-        lo = ps.min_lt;
-        hi = ps.max_lt + 1u;
+        if (track) {
+          lo = ps.min_lt;
+          hi = ps.max_lt + 1u;
+        } else {
+          hi = mid;
+        }
       }
       if (cnt == 0) {  // only by rounding, with top_p within an ulp of 1
         lo = old_lo;
@@ -359,22 +611,7 @@ __device__ RowNucleus nucleus(const float* et, const float* st, float* fg, long 
         warp_bases(side, sh);
         int run = sh.wbase[warp_id()];
         if (list == nullptr) {
-          for_row(et, ftab, V, [&](long long i0, const float4& v, long long n) {
-            int k = 0;
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-              const uint32_t key = __float_as_uint(comp(v, j));
-              k += i0 + j < n && key >= lo && key < hi;
-            }
-            const int incl = warp_incl_scan(k);
-            int at = run + incl - k;
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-              const uint32_t key = __float_as_uint(comp(v, j));
-              if (i0 + j < n && key >= lo && key < hi && at < cnt) dst[at++] = comp(v, j);
-            }
-            run += __shfl_sync(0xffffffffu, incl, 31);
-          });
+          row_compact(et, ftab, static_cast<int>(V), lo, hi - lo, dst, run, cnt);
         } else {
           for (int base = warp_id() * 32; base < n_list; base += kThreads) {
             const int i = base + lane_id();
@@ -382,8 +619,7 @@ __device__ RowNucleus nucleus(const float* et, const float* st, float* fg, long 
             bool keep = false;
             if (i < n_list) {
               e = list[i];
-              const uint32_t key = __float_as_uint(e);
-              keep = key >= lo && key < hi;
+              keep = __float_as_uint(e) - lo < hi - lo;
             }
             const unsigned bal = __ballot_sync(0xffffffffu, keep);
             const int at = run + __popc(bal & ((1u << lane_id()) - 1u));
@@ -406,7 +642,7 @@ __device__ RowNucleus nucleus(const float* et, const float* st, float* fg, long 
   if (!resolved) {  // top_p = 1, or the rounding exit: one more pass over the row
     float g = 0.f;
     int q = 0;
-    for_row(et, ftab, V, [&](long long i0, const float4& v, long long n) {
+    for_row<kWarps>(et, ftab, V, [&](long long i0, const float4& v, long long n) {
 #pragma unroll
       for (int j = 0; j < 4; ++j)
         if (i0 + j < n) {
@@ -432,8 +668,9 @@ __device__ RowNucleus nucleus(const float* et, const float* st, float* fg, long 
 
 // Nucleus probability of token x (block-wide: when x is tied at the boundary
 // and only some ties are kept, its rank among them is counted).
+template <int NW>
 __device__ float prob_of(const float* et, const float* ftab, long long V, const RowNucleus& n,
-                         int x, Shared& sh) {
+                         int x, SharedT<NW>& sh) {
   const float e = et[x] * ftab[x / kGemmBN];
   bool member = e > n.b;
   if (e == n.b) {
@@ -442,7 +679,7 @@ __device__ float prob_of(const float* et, const float* ftab, long long V, const 
     } else {
       float unused = 0.f;
       int below = 0;
-      for_row(et, ftab, V, [&](long long i0, const float4& v, long long cnt) {
+      for_row<NW>(et, ftab, V, [&](long long i0, const float4& v, long long cnt) {
 #pragma unroll
         for (int j = 0; j < 4; ++j)
           if (i0 + j < x && i0 + j < cnt && comp(v, j) == n.b) ++below;
@@ -451,7 +688,7 @@ __device__ float prob_of(const float* et, const float* ftab, long long V, const 
       member = below < n.c;
     }
   }
-  return member ? e / n.kept : 0.f;
+  return member ? e * (1.f / n.kept) : 0.f;
 }
 
 __device__ __forceinline__ void store_state(float* st, const RowNucleus& n) {
@@ -474,57 +711,44 @@ __device__ __forceinline__ RowNucleus load_state(const float* st) {
   return n;
 }
 
-__global__ void __launch_bounds__(kThreads, 2) spec_position_kernel(const SpecParams p) {
+// Shared memory of spec_row_kernel: the row's f_t table, then two lists.
+__host__ __device__ __forceinline__ size_t row_smem(int tiles) {
+  return sizeof(float) * ((static_cast<size_t>(tiles) + 3) / 4 * 4 + 2 * kSpecListCap);
+}
+
+// One CTA per logits row: rows [0, B (gamma + 1)) are the verifier's, the
+// rest the draft's.  Leaves the row's nucleus state and its f_t table.
+__global__ void __launch_bounds__(kThreads, 4) spec_row_kernel(const SpecParams p) {
   extern __shared__ __align__(16) float smem[];
   __shared__ Shared sh;
+  const int tiles_pad = (p.tiles + 3) / 4 * 4;
   float* ftab = smem;
-  float* listA = smem + kSpecMaxTiles;
+  float* listA = smem + tiles_pad;
   float* listB = listA + kSpecListCap;
-  const int G1 = p.gamma + 1;
-  const int b = blockIdx.x / G1, i = blockIdx.x % G1;
-  const long long pos_v = static_cast<long long>(b) * G1 + i;
+  const long long Pv = static_cast<long long>(p.B) * (p.gamma + 1);
   const long long sld = 2LL * p.tiles;
-  const float* ev = p.ev + pos_v * p.ldz;
-  const RowNucleus np = nucleus(ev, p.stats_v + pos_v * sld, p.f_v + pos_v * p.tiles, p.V,
-                                p.tiles, p.scale, p.top_p, ftab, listA, listB, sh);
-  if (threadIdx.x == 0) store_state(p.state_v + pos_v * kSpecStateWords, np);
-  if (i == p.gamma) return;
-  const int x = p.draft[static_cast<long long>(b) * p.gamma + i];
-  float px = 0.f;
-  if (x >= 0 && x < p.V) px = prob_of(ev, ftab, p.V, np, x, sh);
-  __syncthreads();  // ftab is rewritten for the draft row
-  const long long pos_d = static_cast<long long>(b) * p.gamma + i;
-  const float* ed = p.ed + pos_d * p.ldz;
-  const RowNucleus nq = nucleus(ed, p.stats_d + pos_d * sld, p.f_d + pos_d * p.tiles, p.V,
-                                p.tiles, p.scale, p.top_p, ftab, listA, listB, sh);
-  if (threadIdx.x == 0) store_state(p.state_d + pos_d * kSpecStateWords, nq);
-  int ok = 0;
-  if (x >= 0 && x < p.V) {
-    const float qx = prob_of(ed, ftab, p.V, nq, x, sh);
-    ok = qx > 0.f && p.u[pos_v * 2] * qx < px;
-  }
-  if (threadIdx.x == 0) p.acc[pos_v] = ok;
+  long long r = blockIdx.x;
+  const bool verifier = r < Pv;
+  if (!verifier) r -= Pv;
+  const float* et = (verifier ? p.ev : p.ed) + r * p.ldz;
+  prefetch_row(et, p.ldz * 4);
+  const RowNucleus n = nucleus(et, (verifier ? p.stats_v : p.stats_d) + r * sld,
+                               (verifier ? p.f_v : p.f_d) + r * p.tiles, p.V, p.tiles, p.scale,
+                               p.top_p, ftab, listA, listB, sh);
+  if (threadIdx.x == 0) store_state((verifier ? p.state_v : p.state_d) + r * kSpecStateWords, n);
 }
 
 // ------------------------------------------------------------------ sampling
-// Per-warp contiguous segments of the vocabulary, in index order.
-struct Segment {
-  long long begin, end;
-};
-__device__ __forceinline__ Segment my_segment(long long V) {
-  const long long steps = (V + kStep - 1) / kStep;
-  const long long per = (steps + kWarps - 1) / kWarps * kStep;
-  const long long b = min(V, per * warp_id());
-  return {b, min(V, b + per)};
-}
+// Inverse-CDF sampling in index order over steps of 128 tokens: one pass gives
+// every step's mass (warps take steps w, w + 16, ...), one thread accumulates
+// them in index order, and one warp walks the step in which the cumulative
+// passes u * total.
 
-// Nucleus probabilities of the lane's 4 elements from i0 in one step of a
-// segment ending at `end`; `tie_run` (warp-uniform) counts the ties at b
-// before this step in index order.
-__device__ __forceinline__ void probs4(const float* et, const float* ftab, const RowNucleus& n,
-                                       long long i0, long long end, int& tie_run, float (&pr)[4]) {
+// Unnormalised probabilities e of the lane's 4 tokens from i0 (zeros past V).
+__device__ __forceinline__ float4 load_e(const float* et, const float* ftab, long long i0,
+                                         long long V) {
   float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-  if (i0 < end) {
+  if (i0 < V) {
     v = __ldg(reinterpret_cast<const float4*>(et + i0));
     const float fm = ftab[i0 / kGemmBN];
     v.x *= fm;
@@ -532,13 +756,19 @@ __device__ __forceinline__ void probs4(const float* et, const float* ftab, const
     v.z *= fm;
     v.w *= fm;
   }
-  const float inv = 1.f / n.kept;
+  return v;
+}
+
+// Nucleus probabilities of those 4 tokens; rank0 (warp-uniform) counts the
+// ties at b before this step in index order (only read when some ties are out).
+__device__ __forceinline__ void probs4(const float4& v, long long i0, long long V,
+                                       const RowNucleus& n, float inv, int rank0, float (&pr)[4]) {
   float e[4];
   bool valid[4];
   int ties = 0;
 #pragma unroll
   for (int j = 0; j < 4; ++j) {
-    valid[j] = i0 + j < end;
+    valid[j] = i0 + j < V;
     e[j] = comp(v, j);
     ties += valid[j] && e[j] == n.b;
   }
@@ -548,137 +778,166 @@ __device__ __forceinline__ void probs4(const float* et, const float* ftab, const
     return;
   }
   const int incl = warp_incl_scan(ties);
-  int rank = tie_run + incl - ties;
+  int rank = rank0 + incl - ties;
 #pragma unroll
   for (int j = 0; j < 4; ++j) {
     bool in = valid[j] && e[j] > n.b;
     if (valid[j] && e[j] == n.b) in = rank++ < n.c;
     pr[j] = in ? e[j] * inv : 0.f;
   }
-  tie_run += __shfl_sync(0xffffffffu, incl, 31);
 }
 
-// Ties at b in this warp's segment (the bases of the tie ranks).
-__device__ int segment_ties(const float* et, const float* ftab, const RowNucleus& n,
-                            const Segment& sg) {
-  int t = 0;
-  for (long long base = sg.begin; base < sg.end; base += kStep) {
-    const long long i0 = base + lane_id() * 4;
-    if (i0 < sg.end) {
-      const float4 v = __ldg(reinterpret_cast<const float4*>(et + i0));
-      const float fm = ftab[i0 / kGemmBN];
+// In-place inclusive prefix sum of a[0, n) in index order: each thread sums a
+// contiguous run of entries, the runs' totals are scanned across the block
+// (warps by shuffles, then warp 0 over the warp totals), and each run is
+// rewritten from its offset.  Fixed order, so deterministic.
+template <int NW>
+__device__ void block_inclusive_scan(float* a, int n, SharedT<NW>& sh) {
+  const int per = (n + (NW * 32) - 1) / (NW * 32);
+  const int b0 = min(n, static_cast<int>(threadIdx.x) * per), b1 = min(n, b0 + per);
+  float t = 0.f;
+  for (int i = b0; i < b1; ++i) t += a[i];
+  const float incl = warp_incl_scan(t);
+  __syncthreads();
+  if (lane_id() == 31) sh.f[warp_id()][1] = incl;
+  __syncthreads();
+  if (warp_id() == 0) {
+    const float wt = lane_id() < NW ? sh.f[lane_id()][1] : 0.f;
+    const float wi = warp_incl_scan(wt);
+    if (lane_id() < NW) sh.f[lane_id()][0] = wi - wt;  // exclusive warp offsets
+  }
+  __syncthreads();
+  float run = sh.f[warp_id()][0] + (incl - t);
+  for (int i = b0; i < b1; ++i) {
+    run += a[i];
+    a[i] = run;
+  }
+  __syncthreads();
+}
+
+// Per step: the ties at b, then (thread 0, in index order) their exclusive prefix.
+template <int NW>
+__device__ void step_tie_bases(const float* et, const float* ftab, const RowNucleus& n, long long V,
+                               int nsteps, int* base) {
+  const int w = warp_id(), l = lane_id();
+  for (int st = w; st < nsteps; st += NW) {
+    const long long i0 = static_cast<long long>(st) * kStep + l * 4;
+    const float4 v = load_e(et, ftab, i0, V);
+    int t = 0;
 #pragma unroll
-      for (int j = 0; j < 4; ++j) t += (i0 + j < sg.end) && comp(v, j) * fm == n.b;
+    for (int j = 0; j < 4; ++j) t += i0 + j < V && comp(v, j) == n.b;
+    t = static_cast<int>(__reduce_add_sync(0xffffffffu, static_cast<unsigned>(t)));
+    if (l == 0) base[st] = t;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int run = 0;
+    for (int st = 0; st < nsteps; ++st) {
+      const int t = base[st];
+      base[st] = run;
+      run += t;
     }
   }
-  return static_cast<int>(__reduce_add_sync(0xffffffffu, static_cast<unsigned>(t)));
+  __syncthreads();
 }
 
 // sample(r, u) over r_v = max(0, p_v - q_v) (have_q) or r_v = p_v; -1 when r
-// is all zero.
+// is all zero.  cum: nsteps floats; tp/tq: nsteps ints each.
+template <int NW>
 __device__ int sample(const float* ep, const float* fp, const RowNucleus& np, const float* eq,
                       const float* fq, const RowNucleus& nq, bool have_q, long long V, float u,
-                      Shared& sh) {
-  const Segment sg = my_segment(V);
+                      float* cum, int* tp, int* tq, SharedT<NW>& sh) {
+  const int nsteps = static_cast<int>((V + kStep - 1) / kStep);
   const int w = warp_id(), l = lane_id();
-  int base_p = 0, base_q = 0;
-  const bool tp = np.c < np.eq, tq = have_q && nq.c < nq.eq;
-  if (tp || tq) {
-    const int cp = tp ? segment_ties(ep, fp, np, sg) : 0;
-    const int cq = tq ? segment_ties(eq, fq, nq, sg) : 0;
-    __syncthreads();
-    if (l == 0) {
-      sh.n[w][1] = cp;
-      sh.n[w][2] = cq;
-    }
-    __syncthreads();
-    for (int k = 0; k < w; ++k) {
-      base_p += sh.n[k][1];
-      base_q += sh.n[k][2];
-    }
-  }
-  // mass of each warp's segment
-  float mine = 0.f;
-  {
-    int rp = base_p, rq = base_q;
-    for (long long base = sg.begin; base < sg.end; base += kStep) {
-      float a[4], c[4] = {0.f, 0.f, 0.f, 0.f};
-      probs4(ep, fp, np, base + l * 4, sg.end, rp, a);
-      if (have_q) probs4(eq, fq, nq, base + l * 4, sg.end, rq, c);
+  const float ip = 1.f / np.kept, iq = have_q ? 1.f / nq.kept : 0.f;
+  const bool part_p = np.c < np.eq, part_q = have_q && nq.c < nq.eq;
+  if (part_p) step_tie_bases<NW>(ep, fp, np, V, nsteps, tp);
+  if (part_q) step_tie_bases<NW>(eq, fq, nq, V, nsteps, tq);
+  // mass of every step
+  constexpr int kU = 2;
+  for (int s0 = w; s0 < nsteps; s0 += kU * NW) {
+    float4 vp[kU], vq[kU];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) mine += fmaxf(0.f, a[j] - c[j]);
+    for (int k = 0; k < kU; ++k) {
+      const long long i0 = static_cast<long long>(s0 + k * NW) * kStep + l * 4;
+      vp[k] = load_e(ep, fp, i0, V);
+      vq[k] = have_q ? load_e(eq, fq, i0, V) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int k = 0; k < kU; ++k) {
+      const int st = s0 + k * NW;
+      if (st >= nsteps) break;
+      const long long i0 = static_cast<long long>(st) * kStep + l * 4;
+      float a[4], c[4] = {0.f, 0.f, 0.f, 0.f};
+      probs4(vp[k], i0, V, np, ip, part_p ? tp[st] : 0, a);
+      if (have_q) probs4(vq[k], i0, V, nq, iq, part_q ? tq[st] : 0, c);
+      float m = 0.f;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) m += fmaxf(0.f, a[j] - c[j]);
+      m = warp_sum(m);
+      if (l == 0) cum[st] = m;
     }
   }
-  mine = warp_sum(mine);
   __syncthreads();
-  if (l == 0) sh.f[w][0] = mine;
-  __syncthreads();
-  float total = 0.f;
-  for (int k = 0; k < kWarps; ++k) total += sh.f[k][0];
+  block_inclusive_scan(cum, nsteps, sh);
+  const float total = cum[nsteps - 1];
   if (!(total > 0.f)) return -1;
   const float want = u * total;
-  // the segment in which the cumulative passes want, and the mass before it
-  int owner = -1;
-  float before = 0.f;
-  {
-    float incl = 0.f;
-    for (int k = 0; k < kWarps; ++k) {
-      const float next = incl + sh.f[k][0];
-      if (owner < 0 && next > want && sh.f[k][0] > 0.f) {
-        owner = k;
-        before = incl;
-      }
-      incl = next;
+  if (w == 0) {
+    // the first step whose cumulative passes want (and that has mass)
+    int owner = -1;
+    for (int s0 = 0; s0 < nsteps && owner < 0; s0 += 32) {
+      const int st = s0 + l;
+      const float prev = st > 0 && st < nsteps ? cum[st - 1] : 0.f;
+      const bool hit = st < nsteps && cum[st] > want && cum[st] > prev;
+      const unsigned bal = __ballot_sync(0xffffffffu, hit);
+      if (bal) owner = s0 + __ffs(bal) - 1;
     }
-    if (owner < 0) {  // rounding put want past the end: the last token with mass
-      for (int k = kWarps - 1; k >= 0 && owner < 0; --k)
-        if (sh.f[k][0] > 0.f) owner = k;
-      before = -INFINITY;
+    float before = 0.f;
+    if (owner < 0) {  // rounding put want at the total: the last step with mass
+      for (int st = nsteps - 1; st >= 0 && owner < 0; --st)
+        if (cum[st] > (st > 0 ? cum[st - 1] : 0.f)) owner = st;
+      before = -INFINITY;  // pick its last token with mass
+    } else {
+      before = owner > 0 ? cum[owner - 1] : 0.f;
     }
-  }
-  __syncthreads();
-  if (w == owner) {
-    int rp = base_p, rq = base_q;
-    float cum = before;
-    long long found = -1, last = -1;
-    for (long long base = sg.begin; base < sg.end && found < 0; base += kStep) {
-      float a[4], c[4] = {0.f, 0.f, 0.f, 0.f};
-      const long long i0 = base + l * 4;
-      probs4(ep, fp, np, i0, sg.end, rp, a);
-      if (have_q) probs4(eq, fq, nq, i0, sg.end, rq, c);
-      float r[4], lane_sum = 0.f;
+    const long long i0 = static_cast<long long>(owner) * kStep + l * 4;
+    float a[4], c[4] = {0.f, 0.f, 0.f, 0.f};
+    probs4(load_e(ep, fp, i0, V), i0, V, np, ip, part_p ? tp[owner] : 0, a);
+    if (have_q) probs4(load_e(eq, fq, i0, V), i0, V, nq, iq, part_q ? tq[owner] : 0, c);
+    float r[4], lane_sum = 0.f;
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        r[j] = fmaxf(0.f, a[j] - c[j]);
-        lane_sum += r[j];
-      }
-      const float incl = warp_incl_scan(lane_sum);
-      float run = cum + (incl - lane_sum);
-      long long my_found = -1, my_last = -1;
-#pragma unroll
-      for (int j = 0; j < 4; ++j)
-        if (r[j] > 0.f) {
-          my_last = i0 + j;
-          run += r[j];
-          if (my_found < 0 && run > want) my_found = i0 + j;
-        }
-      const unsigned fb = __ballot_sync(0xffffffffu, my_found >= 0);
-      const unsigned lb = __ballot_sync(0xffffffffu, my_last >= 0);
-      if (fb) found = __shfl_sync(0xffffffffu, my_found, __ffs(fb) - 1);
-      if (lb) last = __shfl_sync(0xffffffffu, my_last, 31 - __clz(lb));
-      cum += __shfl_sync(0xffffffffu, incl, 31);
+    for (int j = 0; j < 4; ++j) {
+      r[j] = fmaxf(0.f, a[j] - c[j]);
+      lane_sum += r[j];
     }
-    if (l == 0) sh.n[0][0] = static_cast<int>(found >= 0 ? found : last);
+    const float incl = warp_incl_scan(lane_sum);
+    float run = before + (incl - lane_sum);
+    long long my_found = -1, my_last = -1;
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      if (r[j] > 0.f) {
+        my_last = i0 + j;
+        run += r[j];
+        if (my_found < 0 && run > want) my_found = i0 + j;
+      }
+    const unsigned fb = __ballot_sync(0xffffffffu, my_found >= 0);
+    const unsigned lb = __ballot_sync(0xffffffffu, my_last >= 0);
+    long long res = static_cast<long long>(owner) * kStep;  // unreachable fallbacks
+    if (fb) res = __shfl_sync(0xffffffffu, my_found, __ffs(fb) - 1);
+    else if (lb) res = __shfl_sync(0xffffffffu, my_last, 31 - __clz(lb));
+    if (l == 0) sh.n[0][0] = static_cast<int>(res);
   }
   __syncthreads();
   return sh.n[0][0];
 }
 
 // Greedy: the verifier's argmax of row `pos` from its tile (max, argmax) pairs.
-__device__ int row_argmax(const float* st, int tiles, Shared& sh) {
+template <int NW>
+__device__ int row_argmax(const float* st, int tiles, SharedT<NW>& sh) {
   float mv = -INFINITY;
   int mi = 0;
-  for (int t = threadIdx.x; t < tiles; t += kThreads)
+  for (int t = threadIdx.x; t < tiles; t += (NW * 32))
     if (st[2 * t] > mv) {
       mv = st[2 * t];
       mi = __float_as_int(st[2 * t + 1]);
@@ -687,9 +946,9 @@ __device__ int row_argmax(const float* st, int tiles, Shared& sh) {
   return mi;
 }
 
-__global__ void __launch_bounds__(kThreads) spec_sample_kernel(const SpecParams p) {
-  __shared__ Shared sh;
-  __shared__ float fp[kSpecMaxTiles], fq[kSpecMaxTiles];
+__global__ void __launch_bounds__(kSampleWarps * 32) spec_sample_kernel(const SpecParams p) {
+  extern __shared__ __align__(16) float smem[];
+  __shared__ SharedT<kSampleWarps> sh;
   const int b = blockIdx.x, G1 = p.gamma + 1;
   const long long sld = 2LL * p.tiles;
   int k = 0, next = -1;
@@ -702,21 +961,72 @@ __global__ void __launch_bounds__(kThreads) spec_sample_kernel(const SpecParams 
       }
     }
   } else {
-    while (k < p.gamma && p.acc[static_cast<long long>(b) * G1 + k]) ++k;
+    const int nsteps = static_cast<int>((p.V + kStep - 1) / kStep);
+    float* fp = smem;
+    float* fq = fp + p.tiles;
+    float* cum = fq + p.tiles;
+    int* tp = reinterpret_cast<int*>(cum + nsteps);
+    int* tq = tp + nsteps;
+    int* acc = tq + nsteps;  // per drafted position: 1 accepted, 0 rejected, 2 undecided
+    // Acceptance of every drafted token, in parallel: q(x) and p(x) from the
+    // rows' nucleus states; a token tied at a boundary of which only some
+    // ties are kept needs its rank among them (a pass over the row, below).
+    for (int i = threadIdx.x; i < p.gamma; i += kSampleWarps * 32) {
+      const long long pos_d = static_cast<long long>(b) * p.gamma + i, pos_v = static_cast<long long>(b) * G1 + i;
+      const int x = p.draft[pos_d];
+      int f = 0;
+      if (x >= 0 && x < p.V) {
+        const RowNucleus nq = load_state(p.state_d + pos_d * kSpecStateWords);
+        const RowNucleus np = load_state(p.state_v + pos_v * kSpecStateWords);
+        const float eq = p.ed[pos_d * p.ldz + x] * p.f_d[pos_d * p.tiles + x / kGemmBN];
+        const float ep = p.ev[pos_v * p.ldz + x] * p.f_v[pos_v * p.tiles + x / kGemmBN];
+        const bool rank_q = eq == nq.b && nq.c < nq.eq, rank_p = ep == np.b && np.c < np.eq;
+        if (rank_q || rank_p) {
+          f = 2;
+        } else {
+          const float qx = eq >= nq.b ? eq * (1.f / nq.kept) : 0.f;
+          const float px = ep >= np.b ? ep * (1.f / np.kept) : 0.f;
+          f = qx > 0.f && p.u[pos_v * 2] * qx < px;
+        }
+      }
+      acc[i] = f;
+    }
+    __syncthreads();
+    for (; k < p.gamma; ++k) {
+      int f = acc[k];
+      if (f == 2) {  // block-wide: rank of x among the ties at the boundary
+        const long long pos_d = static_cast<long long>(b) * p.gamma + k, pos_v = static_cast<long long>(b) * G1 + k;
+        const int x = p.draft[pos_d];
+        for (int t = threadIdx.x; t < p.tiles; t += kSampleWarps * 32) {
+          fq[t] = p.f_d[pos_d * p.tiles + t];
+          fp[t] = p.f_v[pos_v * p.tiles + t];
+        }
+        __syncthreads();
+        const float qx = prob_of(p.ed + pos_d * p.ldz, fq, p.V,
+                                 load_state(p.state_d + pos_d * kSpecStateWords), x, sh);
+        const float px = prob_of(p.ev + pos_v * p.ldz, fp, p.V,
+                                 load_state(p.state_v + pos_v * kSpecStateWords), x, sh);
+        f = qx > 0.f && p.u[pos_v * 2] * qx < px;
+        __syncthreads();
+      }
+      if (!f) break;
+    }
     const long long pos_v = static_cast<long long>(b) * G1 + k;
     const RowNucleus np = load_state(p.state_v + pos_v * kSpecStateWords);
     const float* ev = p.ev + pos_v * p.ldz;
-    for (int t = threadIdx.x; t < p.tiles; t += kThreads) fp[t] = p.f_v[pos_v * p.tiles + t];
+    prefetch_row(ev, p.ldz * 4);
+    if (k < p.gamma) prefetch_row(p.ed + (static_cast<long long>(b) * p.gamma + k) * p.ldz, p.ldz * 4);
+    for (int t = threadIdx.x; t < p.tiles; t += kSampleWarps * 32) fp[t] = p.f_v[pos_v * p.tiles + t];
     const float u = p.u[pos_v * 2 + 1];
     if (k < p.gamma) {
       const long long pos_d = static_cast<long long>(b) * p.gamma + k;
       const RowNucleus nq = load_state(p.state_d + pos_d * kSpecStateWords);
-      for (int t = threadIdx.x; t < p.tiles; t += kThreads) fq[t] = p.f_d[pos_d * p.tiles + t];
+      for (int t = threadIdx.x; t < p.tiles; t += kSampleWarps * 32) fq[t] = p.f_d[pos_d * p.tiles + t];
       __syncthreads();
-      next = sample(ev, fp, np, p.ed + pos_d * p.ldz, fq, nq, true, p.V, u, sh);
+      next = sample(ev, fp, np, p.ed + pos_d * p.ldz, fq, nq, true, p.V, u, cum, tp, tq, sh);
     }
     __syncthreads();
-    if (next < 0) next = sample(ev, fp, np, ev, fp, np, false, p.V, u, sh);
+    if (next < 0) next = sample(ev, fp, np, ev, fp, np, false, p.V, u, cum, tp, tq, sh);
     if (next < 0) next = static_cast<int>(p.V - 1);  // unreachable: the maximum has e = 1
   }
   if (threadIdx.x == 0) {
@@ -725,23 +1035,34 @@ __global__ void __launch_bounds__(kThreads) spec_sample_kernel(const SpecParams 
   }
 }
 
+size_t sample_smem(long long V, int tiles, int gamma) {
+  const long long nsteps = (V + kStep - 1) / kStep;
+  return sizeof(float) * (2 * static_cast<size_t>(tiles) + 3 * static_cast<size_t>(nsteps) +
+                          static_cast<size_t>(gamma));
+}
+
 }  // namespace
 
 cudaError_t setup_spec_kernels() {
-  return cudaFuncSetAttribute(spec_position_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              static_cast<int>(kPositionSmem));
+  cudaError_t e = cudaFuncSetAttribute(spec_row_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(row_smem(kSpecMaxTiles)));
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(
+      spec_sample_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+      static_cast<int>(sample_smem(static_cast<long long>(kSpecMaxTiles) * kGemmBN, kSpecMaxTiles,
+                                   kSpecMaxGamma)));
 }
 
-cudaError_t launch_spec_position(const SpecParams& p, cudaStream_t s) {
-  const long long blocks = static_cast<long long>(p.B) * (p.gamma + 1);
-  if (blocks <= 0 || p.greedy) return cudaSuccess;
-  spec_position_kernel<<<static_cast<unsigned>(blocks), kThreads, kPositionSmem, s>>>(p);
+cudaError_t launch_spec_rows(const SpecParams& p, cudaStream_t s) {
+  const long long rows = static_cast<long long>(p.B) * (2 * p.gamma + 1);
+  if (rows <= 0 || p.greedy) return cudaSuccess;
+  spec_row_kernel<<<static_cast<unsigned>(rows), kThreads, row_smem(p.tiles), s>>>(p);
   return cudaGetLastError();
 }
 
 cudaError_t launch_spec_sample(const SpecParams& p, cudaStream_t s) {
   if (p.B <= 0) return cudaSuccess;
-  spec_sample_kernel<<<p.B, kThreads, 0, s>>>(p);
+  spec_sample_kernel<<<p.B, kSampleWarps * 32, p.greedy ? 0 : sample_smem(p.V, p.tiles, p.gamma), s>>>(p);
   return cudaGetLastError();
 }
 
