@@ -49,27 +49,20 @@ def peaks():
         return dict(FALLBACK_PEAKS), "fallback"
 
 
-def source_hash() -> str:
-    csrc = os.path.join(ROOT, "paper_2608_09703_gb300", "csrc")
-    h = hashlib.sha256()
-    for name in sorted(os.listdir(csrc)):
-        if name.endswith((".cu", ".cuh", ".h")):
-            with open(os.path.join(csrc, name), "rb") as fh:
-                h.update(fh.read())
-    return h.hexdigest()[:16]
-
-
 def traffic_for(kernel: str):
     """DRAM bytes per launch from the committed ncu summary, if it was taken
-    on the current kernel sources (else None)."""
+    on the current sources of that kernel (the files it lists); else None."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as fh:
-            d = json.load(fh)
+            e = json.load(fh).get(kernel)
+        h = hashlib.sha256()
+        for name in e["sources"]:
+            with open(os.path.join(ROOT, name), "rb") as fh:
+                h.update(fh.read())
     except Exception:
         return None
-    e = d.get(kernel)
-    if not e or e.get("source_hash") != source_hash():
+    if e.get("source_hash") != h.hexdigest()[:16]:
         return None
     return e.get("traffic_bytes_per_launch")
 
