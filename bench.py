@@ -35,7 +35,8 @@ sys.path.insert(0, ROOT)
 METRIC = "tokens/s fused head+CE+KL fwd+bwd (3-level suite) and % of dense BF16 tensor peak"
 UNIT = "tokens/s"
 WORKLOAD = "suite3"
-KERNELS = ("head_fwd", "head_bwd", "gemm_dw", "gemm_dh")   # each does 2*T*V*sum(d) FLOPs per step
+# FLOPs of each tensor kernel per step, in units of 2*T*V*sum(d) (gemm_bwd runs dW and dH together)
+KERNELS = {"head_fwd": 1, "head_bwd": 1, "gemm_dw": 1, "gemm_dh": 1, "gemm_bwd": 2}
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
@@ -315,12 +316,12 @@ def gpu_arm(args, rank, world, local):
     for name, (launches, total_ms) in kern.items():
         entry = {"launches_per_step": launches / args.steps, "ms_per_step": total_ms / args.steps}
         if name in KERNELS:
-            flops_launch = (step_flops / 4) / (launches / args.steps)
+            flops_launch = KERNELS[name] * (step_flops / 4) / (launches / args.steps)
             entry["tflops"] = flops_launch / (total_ms / launches / 1e3) / 1e12
         per_kernel[name] = entry
     dom = max((k for k in KERNELS if k in kern), key=lambda k: kern[k][1])
     launches, total_ms = kern[dom]
-    flops_launch = (step_flops / 4) / (launches / args.steps)
+    flops_launch = KERNELS[dom] * (step_flops / 4) / (launches / args.steps)
     achieved = flops_launch / (total_ms / launches / 1e3) / 1e12
     # The kernels are timed inside a loop of back-to-back steps, the regime in
     # which the clock settles under the power cap: the sustained bf16 figure

@@ -400,6 +400,26 @@ extern "C" int mls_head_loss_fwd(const mls_problem* p, const void* const* H, con
   return timed("final", s, [&] { return launch_final(mp.block_sum, mp.block_cnt, pl.merge_blocks, loss, s); });
 }
 
+// Two-class schedule of a persistent GEMM launch whose first n_long tiles take
+// cost_long and the other n_short cost_short (K-blocks plus a per-tile
+// allowance): see GemmParams.  The pairs that get one long tile fewer take
+// `catchup` short tiles first, about the cost of that long tile.
+void schedule_two_class(GemmParams& g, int pairs, int n_long, long long cost_long, int n_short,
+                        long long cost_short) {
+  g.two_class = 0;
+  if (pairs < 1 || n_long <= 0 || n_short <= 0) return;
+  g.two_class = 1;
+  g.n_long = n_long;
+  const int r = n_long % pairs;
+  int catchup = 0;
+  if (r > 0) {
+    catchup = static_cast<int>((cost_long + cost_short / 2) / cost_short);
+    const int most = n_short / (pairs - r);
+    if (catchup > most) catchup = most;
+  }
+  g.catchup = catchup;
+}
+
 extern "C" int mls_head_loss_bwd(const mls_problem* p, const void* const* H, const void* const* W,
                                  const int32_t* targets, const float* stats, float grad_scale,
                                  float* const* dH, float* const* dW, void* ws, size_t ws_bytes,
@@ -448,7 +468,7 @@ extern "C" int mls_head_loss_bwd(const mls_problem* p, const void* const* H, con
   // A = G K-major and B = W viewed N-major, all in place.
   // fp32 (tf32 MMA): dW reads A = G^T and B = H^T, dH reads A = G and B = W^T,
   // all K-major.
-  GemmParams gw, gh;
+  GemmParams gw, gh, gb;
   std::memset(&gw, 0, sizeof gw);
   std::memset(&gh, 0, sizeof gh);
   float* GT = tf32 ? reinterpret_cast<float*>(wsb + pl.off_GT) : nullptr;
@@ -534,10 +554,37 @@ extern "C" int mls_head_loss_bwd(const mls_problem* p, const void* const* H, con
     if (tf32) {
       if ((rc = timed("gemm_dw", s, [&] { return launch_gemm_kk(gw, true, grid_w, s); }))) return rc;
       if ((rc = timed("gemm_dh", s, [&] { return launch_gemm_kk(gh, true, grid_h, s); }))) return rc;
-    } else {
-      if ((rc = timed("gemm_dw", s, [&] { return launch_gemm_dw(gw, false, grid_w, s); }))) return rc;
-      if ((rc = timed("gemm_dh", s, [&] { return launch_gemm_dh(gh, false, grid_h, s); }))) return rc;
+      continue;
     }
+    // bf16: dW and dH of every sub-model in one persistent launch, the class
+    // with the longer reduction (dH: the group's columns, dW: T) scheduled first.
+    const bool dh_long = gc >= p->T;
+    const GemmParams& L = dh_long ? gh : gw;
+    const GemmParams& S = dh_long ? gw : gh;
+    std::memset(&gb, 0, sizeof gb);
+    const int M = p->M;
+    for (int m = 0; m < M; ++m) {
+      gb.mapA[m] = L.mapA[m];
+      gb.mapB[m] = L.mapB[m];
+      gb.prob[m] = L.prob[m];
+      gb.prob[m].a_map = gb.prob[m].b_map = m;
+      gb.prob[m].a_mn = dh_long ? 0 : 1;
+      gb.mapA[M + m] = S.mapA[m];
+      gb.mapB[M + m] = S.mapB[m];
+      gb.prob[M + m] = S.prob[m];
+      gb.prob[M + m].a_map = gb.prob[M + m].b_map = M + m;
+      gb.prob[M + m].a_mn = dh_long ? 1 : 0;
+      gb.prob[M + m].tile_begin += L.total_tiles;
+    }
+    gb.nprob = 2 * M;
+    gb.total_tiles = L.total_tiles + S.total_tiles;
+    gb.status = dev->status;
+    const int grid = 2 * (gb.total_tiles < pairs ? gb.total_tiles : pairs);
+    // cost of a tile: its K-blocks plus an allowance for draining its 256x256 accumulator
+    constexpr long long kDrainBlocks = 8;
+    schedule_two_class(gb, grid / 2, L.total_tiles, ceil_div(L.prob[0].K, KE) + kDrainBlocks,
+                       S.total_tiles, ceil_div(S.prob[0].K, KE) + kDrainBlocks);
+    if ((rc = timed("gemm_bwd", s, [&] { return launch_gemm_mixed(gb, grid, s); }))) return rc;
   }
   return MLS_OK;
 }

@@ -63,6 +63,31 @@ struct TileCoord {
   int prob, tm, tn;
 };
 
+// The j-th tile of this pair, or -1 when it has no more.
+__device__ __forceinline__ int pair_tile(const GemmParams& p, int pair, int npairs, int j) {
+  if (!p.two_class) {
+    const int t = pair + j * npairs;
+    return t < p.total_tiles ? t : -1;
+  }
+  const int r = p.n_long % npairs;
+  const int nl = p.n_long / npairs + (pair < r ? 1 : 0);
+  if (j < nl) return pair + j * npairs;
+  j -= nl;
+  const int n_short = p.total_tiles - p.n_long;
+  if (pair >= r) {
+    if (j < p.catchup) return p.n_long + (pair - r) + j * (npairs - r);
+    j -= p.catchup;
+  }
+  const int s = p.catchup * (npairs - r) + pair + j * npairs;
+  return s < n_short ? p.n_long + s : -1;
+}
+
+// A is MN-major for this problem.
+template <int kAMode>
+__device__ __forceinline__ bool a_mn_of(const GemmProblem& pr) {
+  return kAMode == 2 ? pr.a_mn != 0 : kAMode == 1;
+}
+
 __device__ __forceinline__ TileCoord decode_tile(const GemmParams& p, int t) {
   int i = 0;
   while (i + 1 < p.nprob && t >= p.prob[i + 1].tile_begin) ++i;
@@ -72,7 +97,7 @@ __device__ __forceinline__ TileCoord decode_tile(const GemmParams& p, int t) {
 }
 
 // This CTA's loads: its 128 rows of A and its 128 rows of B for every k-block.
-template <bool kTF32, bool kAMN, bool kBMN>
+template <bool kTF32, int kAMode, bool kBMN>
 __device__ __forceinline__ void gemm_producer(const GemmParams& p, uint32_t base, uint32_t rank,
                                               volatile int* abort_flag) {
   constexpr int KE = kTF32 ? 32 : 64;  // elements per 128-byte row
@@ -81,9 +106,11 @@ __device__ __forceinline__ void gemm_producer(const GemmParams& p, uint32_t base
   int stage = 0;
   uint32_t phase = 0, filled = 0, lastpar = 0;
   bool ok = true;
-  for (int t = pair; ok && t < p.total_tiles; t += npairs) {
+  int t;
+  for (int j = 0; ok && (t = pair_tile(p, pair, npairs, j)) >= 0; ++j) {
     const TileCoord tc = decode_tile(p, t);
     const GemmProblem& pr = p.prob[tc.prob];
+    const bool amn = a_mn_of<kAMode>(pr);
     const CUtensorMap* ma = &p.mapA[pr.a_map];
     const CUtensorMap* mb = &p.mapB[pr.b_map];
     const int nkb = (pr.K + KE - 1) / KE;
@@ -99,16 +126,16 @@ __device__ __forceinline__ void gemm_producer(const GemmParams& p, uint32_t base
       const uint32_t sa = base + GemmSmem::kA + stage * kGemmABytes;
       const uint32_t sb = base + GemmSmem::kB + stage * kGemmBBytes;
       const int ka = pr.a_k0 + kb * KE, kbb = pr.b_k0 + kb * KE;
-      if (kAMN) {
+      if (amn) {
 #pragma unroll
-        for (int j = 0; j < kGemmBM / KE; ++j) tma_load_2d_pair(sa + j * kBox, ma, fb, m0 + j * KE, ka);
+        for (int q = 0; q < kGemmBM / KE; ++q) tma_load_2d_pair(sa + q * kBox, ma, fb, m0 + q * KE, ka);
       } else {
         tma_load_2d_pair(sa, ma, fb, ka, m0);
       }
       if (kBMN) {
 #pragma unroll
-        for (int j = 0; j < kGemmBHalf / KE; ++j)
-          tma_load_2d_pair(sb + j * kBox, mb, fb, n0 + j * KE, kbb);
+        for (int q = 0; q < kGemmBHalf / KE; ++q)
+          tma_load_2d_pair(sb + q * kBox, mb, fb, n0 + q * KE, kbb);
       } else {
         tma_load_2d_pair(sb, mb, fb, kbb, n0);
       }
@@ -133,11 +160,10 @@ __device__ __forceinline__ void gemm_producer(const GemmParams& p, uint32_t base
   }
 }
 
-template <bool kTF32, bool kAMN, bool kBMN>
+template <bool kTF32, int kAMode, bool kBMN>
 __device__ __forceinline__ void gemm_mma(const GemmParams& p, uint32_t base, uint32_t tmem,
                                          volatile int* abort_flag) {
   constexpr int KE = kTF32 ? 32 : 64;
-  constexpr uint32_t kIdesc = make_idesc(kPairM, kGemmBN, kTF32, kAMN, kBMN);
   constexpr uint32_t kBox = KE * 128;
   // Advance per MMA (32 bytes of K): along a 128-byte row for K-major
   // operands, by (32 / element size) rows of 128 bytes for MN-major ones.
@@ -148,9 +174,12 @@ __device__ __forceinline__ void gemm_mma(const GemmParams& p, uint32_t base, uin
   int stage = 0;
   uint32_t phase = 0, acc = 0, acc_par = 0;
   bool ok = true;
-  for (int t = pair; ok && t < p.total_tiles; t += npairs) {
+  int t;
+  for (int j = 0; ok && (t = pair_tile(p, pair, npairs, j)) >= 0; ++j) {
     const TileCoord tc = decode_tile(p, t);
     const int nkb = (p.prob[tc.prob].K + KE - 1) / KE;
+    const bool amn = a_mn_of<kAMode>(p.prob[tc.prob]);
+    const uint32_t idesc = make_idesc(kPairM, kGemmBN, kTF32, amn, kBMN);
     if (!mbar_wait(GemmSmem::acce(base, acc), acc_par ^ 1u, abort_flag, p.status)) {
       ok = false;
       break;
@@ -163,12 +192,12 @@ __device__ __forceinline__ void gemm_mma(const GemmParams& p, uint32_t base, uin
         break;
       }
       tc_fence_after();
-      const uint64_t ad = make_sdesc(base + GemmSmem::kA + stage * kGemmABytes, kAMN ? kBox : 16u);
+      const uint64_t ad = make_sdesc(base + GemmSmem::kA + stage * kGemmABytes, amn ? kBox : 16u);
       const uint64_t bd = make_sdesc(base + GemmSmem::kB + stage * kGemmBBytes, kBMN ? kBox : 16u);
 #pragma unroll
       for (int kk = 0; kk < 4; ++kk)
-        mma_issue_pair<kTF32>(d, ad + kk * (kAMN ? kStepMN : kStepK),
-                              bd + kk * (kBMN ? kStepMN : kStepK), kIdesc, (kb | kk) != 0);
+        mma_issue_pair<kTF32>(d, ad + kk * (amn ? kStepMN : kStepK),
+                              bd + kk * (kBMN ? kStepMN : kStepK), idesc, (kb | kk) != 0);
       mma_commit_pair(GemmSmem::empty(base, stage), kBoth);
       if (++stage == kGemmStages) {
         stage = 0;
@@ -257,7 +286,8 @@ __device__ __forceinline__ void gemm_epilogue(const GemmParams& p, uint32_t base
   uint32_t acc = 0, acc_par = 0, stores = 0;
   const uint32_t tl = tmem + (static_cast<uint32_t>(warp * 32) << 16);
   const uint32_t stage = base + GemmSmem::kStaging + static_cast<uint32_t>(warp) * 2 * GemmSmem::kChunk;
-  for (int t = pair; t < p.total_tiles; t += npairs) {
+  int t;
+  for (int j = 0; (t = pair_tile(p, pair, npairs, j)) >= 0; ++j) {
     const TileCoord tc = decode_tile(p, t);
     const GemmProblem& pr = p.prob[tc.prob];
     const bool ok = mbar_wait(GemmSmem::accf(base, acc), acc_par, abort_flag, p.status);
@@ -309,7 +339,7 @@ __device__ __forceinline__ void gemm_epilogue(const GemmParams& p, uint32_t base
   if (stores && lane == 0) bulk_wait_all();  // staging must outlive the stores reading it
 }
 
-template <bool kTF32, bool kAMN, bool kBMN>
+template <bool kTF32, int kAMode, bool kBMN>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     gemm_kernel(const __grid_constant__ GemmParams p) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -350,9 +380,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
   const uint32_t tmem = *tmem_slot;
 
   if (warp == kGemmEpiWarps) {
-    if (lane == 0) gemm_producer<kTF32, kAMN, kBMN>(p, base, rank, abort_flag);
+    if (lane == 0) gemm_producer<kTF32, kAMode, kBMN>(p, base, rank, abort_flag);
   } else if (warp == kGemmEpiWarps + 1) {
-    if (lane == 0 && rank == 0) gemm_mma<kTF32, kAMN, kBMN>(p, base, tmem, abort_flag);
+    if (lane == 0 && rank == 0) gemm_mma<kTF32, kAMode, kBMN>(p, base, tmem, abort_flag);
     __syncwarp();
   } else {
     gemm_epilogue(p, base, tmem, rank, warp, lane, abort_flag);
@@ -366,26 +396,31 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
   }
 }
 
-template <bool kAMN, bool kBMN>
+template <int kAMode, bool kBMN>
 cudaError_t launch(const GemmParams& p, bool tf32, int grid, cudaStream_t s) {
   if (p.total_tiles <= 0 || grid <= 0) return cudaSuccess;
   if (tf32)
-    gemm_kernel<true, kAMN, kBMN><<<grid, kGemmThreads, kGemmSmem, s>>>(p);
+    gemm_kernel<true, kAMode, kBMN><<<grid, kGemmThreads, kGemmSmem, s>>>(p);
   else
-    gemm_kernel<false, kAMN, kBMN><<<grid, kGemmThreads, kGemmSmem, s>>>(p);
+    gemm_kernel<false, kAMode, kBMN><<<grid, kGemmThreads, kGemmSmem, s>>>(p);
   return cudaGetLastError();
 }
 
 }  // namespace
 
 cudaError_t launch_gemm_dw(const GemmParams& p, bool tf32, int grid, cudaStream_t s) {
-  return launch<true, true>(p, tf32, grid, s);
+  return launch<1, true>(p, tf32, grid, s);
 }
 cudaError_t launch_gemm_dh(const GemmParams& p, bool tf32, int grid, cudaStream_t s) {
-  return launch<false, true>(p, tf32, grid, s);
+  return launch<0, true>(p, tf32, grid, s);
 }
 cudaError_t launch_gemm_kk(const GemmParams& p, bool tf32, int grid, cudaStream_t s) {
-  return launch<false, false>(p, tf32, grid, s);
+  return launch<0, false>(p, tf32, grid, s);
+}
+cudaError_t launch_gemm_mixed(const GemmParams& p, int grid, cudaStream_t s) {
+  if (p.total_tiles <= 0 || grid <= 0) return cudaSuccess;
+  gemm_kernel<false, 2, true><<<grid, kGemmThreads, kGemmSmem, s>>>(p);
+  return cudaGetLastError();
 }
 
 // How many CTA pairs of the GEMM kernel can be resident at once (GPCs with an
@@ -396,7 +431,7 @@ int gemm_max_active_pairs() {
   cfg.blockDim = dim3(kGemmThreads);
   cfg.dynamicSmemBytes = kGemmSmem;
   int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, gemm_kernel<false, true, true>, &cfg) != cudaSuccess) {
+  if (cudaOccupancyMaxActiveClusters(&n, gemm_kernel<false, 1, true>, &cfg) != cudaSuccess) {
     cudaGetLastError();
     return 0;
   }
@@ -415,12 +450,13 @@ cudaError_t setup_gemm_kernels() {
     if (e != cudaSuccess) return e;                                                             \
     if (fa.maxThreadsPerBlock < kGemmThreads) return cudaErrorLaunchOutOfResources;             \
   }
-  MLS_SET(true, true, true)
-  MLS_SET(false, true, true)
-  MLS_SET(true, false, true)
-  MLS_SET(false, false, true)
-  MLS_SET(true, false, false)
-  MLS_SET(false, false, false)
+  MLS_SET(true, 1, true)
+  MLS_SET(false, 1, true)
+  MLS_SET(true, 0, true)
+  MLS_SET(false, 0, true)
+  MLS_SET(true, 0, false)
+  MLS_SET(false, 0, false)
+  MLS_SET(false, 2, true)
 #undef MLS_SET
   return cudaSuccess;
 }

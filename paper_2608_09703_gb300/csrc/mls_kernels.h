@@ -110,17 +110,30 @@ struct GemmProblem {
   float epi_scale;
   float* stats;
   long long stats_ld;
+  int a_mn;                      // A is MN-major (read by launches that take the layout per problem)
 };
 enum GemmEpilogue { kEpiPlain = 0, kEpiSoftmax = 1, kEpiArgmax = 2 };
 
+constexpr int kGemmMaxProblems = 2 * kMaxModels;
+
 struct GemmParams {
-  CUtensorMap mapA[kMaxModels];
-  CUtensorMap mapB[kMaxModels];
-  CUtensorMap mapC[kMaxModels];  // kEpiSoftmax: C fp32 [Mrows, Ncols], box {32, 32}, 128B swizzle
+  CUtensorMap mapA[kGemmMaxProblems];
+  CUtensorMap mapB[kGemmMaxProblems];
+  CUtensorMap mapC[kGemmMaxProblems];  // kEpiSoftmax: C fp32 [Mrows, Ncols], box {32, 32}, 128B swizzle
   int nprob;
-  GemmProblem prob[kMaxModels];
+  GemmProblem prob[kGemmMaxProblems];
   int total_tiles;
   int* status;
+  // Schedule.  two_class == 0: pair p takes tiles p, p + npairs, ...
+  // two_class == 1: tiles [0, n_long) are the long ones (larger K) and go
+  // round-robin first, so the first r = n_long % npairs pairs get one more.
+  // The other pairs then take `catchup` short tiles each, round-robin among
+  // themselves, to even out that extra long tile; the remaining short tiles go
+  // round-robin over all pairs.  Neighbouring tiles (which share operands in
+  // L2) keep running at the same time.
+  int two_class;
+  int n_long;
+  int catchup;
 };
 
 // ------------------------------------------------------------------ pairwise evaluation
@@ -239,6 +252,8 @@ cudaError_t launch_head_fwd(const HeadParams& p, bool tf32, bool tau_one, cudaSt
 cudaError_t launch_head_bwd(const HeadParams& p, bool tf32, bool tau_one, cudaStream_t s);
 cudaError_t launch_gemm_dw(const GemmParams& p, bool tf32, int grid, cudaStream_t s);
 cudaError_t launch_gemm_dh(const GemmParams& p, bool tf32, int grid, cudaStream_t s);
+// bf16, B MN-major, A's layout per problem (GemmProblem::a_mn): dW and dH in one launch.
+cudaError_t launch_gemm_mixed(const GemmParams& p, int grid, cudaStream_t s);
 // Both operands K-major (tf32 path: fp32 inputs with transposed copies).
 cudaError_t launch_gemm_kk(const GemmParams& p, bool tf32, int grid, cudaStream_t s);
 cudaError_t launch_transpose(const float* in, long long rows, long long cols, long long ld_in,
