@@ -94,16 +94,6 @@ __device__ __forceinline__ float comp(const float4& v, int j) {
   return j == 0 ? v.x : j == 1 ? v.y : j == 2 ? v.z : v.w;
 }
 
-// Prefetches a row of `bytes` (a multiple of 16) into L2 in 16 KB pieces, one
-// per thread of the first warps.
-__device__ __forceinline__ void prefetch_row(const float* row, long long bytes) {
-  constexpr long long kPiece = 16384;
-  const long long off = static_cast<long long>(threadIdx.x) * kPiece;
-  if (off < bytes)
-    prefetch_l2_bulk(reinterpret_cast<const char*>(row) + off,
-                     static_cast<uint32_t>(bytes - off < kPiece ? bytes - off : kPiece));
-}
-
 // Block reductions: each warp reduces by a butterfly, lane 0 parks the
 // warp's partial, warp 0 combines the 16 partials by a butterfly and parks the
 // result for every thread.  Fixed order throughout.
@@ -282,14 +272,18 @@ __device__ __forceinline__ void row_pass(const float* et, const float* ftab, int
     float4 v[kUnroll];
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u) {
-      const int i0 = base + u * kStride + l * 4;
-      v[u] = i0 < V ? __ldg(reinterpret_cast<const float4*>(et + i0)) : make_float4(0.f, 0.f, 0.f, 0.f);
+      const int s0 = base + u * kStride, i0 = s0 + l * 4;
+      // a tile whose maximum lies below the bracket holds no candidate
+      const bool live = s0 < V && __float_as_uint(ftab[static_cast<unsigned>(s0) / kGemmBN]) >= lo;
+      v[u] = live && i0 < V ? __ldg(reinterpret_cast<const float4*>(et + i0))
+                            : make_float4(0.f, 0.f, 0.f, 0.f);
     }
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u) {
       const int i0 = base + u * kStride + l * 4;
       if (i0 < V) {
         const float fm = ftab[static_cast<unsigned>(i0) / kGemmBN];
+        if (__float_as_uint(fm) < lo) continue;
         const float e0 = v[u].x * fm, e1 = v[u].y * fm, e2 = v[u].z * fm, e3 = v[u].w * fm;
         ps.add<kTrack>(e0, lo, mo, wm);
         if (i0 + 4 <= V) {
@@ -305,11 +299,11 @@ __device__ __forceinline__ void row_pass(const float* et, const float* ftab, int
   }
 }
 
-// The first bisection pass over a whole row: the split at 2^-8 of the maximum
-// over [0, 1].  Mass and count of the upper side, smallest and largest key of
-// the lower side; the few upper-side tokens are also appended, in this warp's
-// visiting order, to its own region of kSpecListCap / kWarps slots of
-// `regions` (wrun counts them, also past the region's end).
+// The first bisection pass over a row: the split at 2^-8 of the maximum.
+// Every e of column tile t is at most f_t, so only tiles with f_t >= 2^-8 are
+// read.  Mass and count of the upper side; its few tokens are also appended,
+// in this warp's visiting order, to its own region of kSpecListCap / kWarps
+// slots of `regions` (wrun counts them, also past the region's end).
 constexpr int kRegion = kSpecListCap / kWarps;
 __device__ __forceinline__ void first_pass(const float* et, const float* ftab, int V, float* regions,
                                            PassStats& ps, int& wrun) {
@@ -319,29 +313,29 @@ __device__ __forceinline__ void first_pass(const float* et, const float* ftab, i
   wrun = 0;
   for (int base = warp_id() * kStep; base < V; base += kUnroll * kStride) {
     float4 v[kUnroll];
+    float fm[kUnroll];
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u) {
-      const int i0 = base + u * kStride + l * 4;
-      v[u] = i0 < V ? __ldg(reinterpret_cast<const float4*>(et + i0)) : make_float4(0.f, 0.f, 0.f, 0.f);
+      const int s0 = base + u * kStride, i0 = s0 + l * 4;
+      fm[u] = s0 < V ? ftab[static_cast<unsigned>(s0) / kGemmBN] : 0.f;  // warp-uniform
+      v[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (__float_as_uint(fm[u]) >= kFirstMid && i0 < V)
+        v[u] = __ldg(reinterpret_cast<const float4*>(et + i0));
     }
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u) {
+      if (__float_as_uint(fm[u]) < kFirstMid) continue;  // warp-uniform: nothing reaches 2^-8
       const int i0 = base + u * kStride + l * 4;
       const int nv = min(max(V - i0, 0), 4);
-      const float fm = nv > 0 ? ftab[static_cast<unsigned>(i0) / kGemmBN] : 0.f;
-      const float e[4] = {v[u].x * fm, v[u].y * fm, v[u].z * fm, v[u].w * fm};
+      const float e[4] = {v[u].x * fm[u], v[u].y * fm[u], v[u].z * fm[u], v[u].w * fm[u]};
       bool ge[4];
       int k = 0;
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
-        const uint32_t key = __float_as_uint(e[j]);
-        ge[j] = j < nv && key >= kFirstMid;
+        ge[j] = j < nv && __float_as_uint(e[j]) >= kFirstMid;
         if (ge[j]) {
           ps.mass_ge += e[j];
           ++k;
-        } else if (j < nv) {
-          ps.min_lt = min(ps.min_lt, key);
-          ps.max_lt = max(ps.max_lt, key);
         }
       }
       ps.cnt_ge += k;
@@ -368,16 +362,19 @@ __device__ __forceinline__ void row_compact(const float* et, const float* ftab, 
   constexpr int kStride = kWarps * kStep;
   for (int base = warp_id() * kStep; base < V; base += kUnroll * kStride) {
     float4 v[kUnroll];
+    float fm[kUnroll];
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u) {
-      const int i0 = base + u * kStride + l * 4;
-      v[u] = i0 < V ? __ldg(reinterpret_cast<const float4*>(et + i0)) : make_float4(0.f, 0.f, 0.f, 0.f);
+      const int s0 = base + u * kStride, i0 = s0 + l * 4;
+      fm[u] = s0 < V ? ftab[static_cast<unsigned>(s0) / kGemmBN] : 0.f;  // warp-uniform
+      v[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (__float_as_uint(fm[u]) >= lo && i0 < V) v[u] = __ldg(reinterpret_cast<const float4*>(et + i0));
     }
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u) {
+      if (__float_as_uint(fm[u]) < lo) continue;  // warp-uniform: no candidate in this tile
       const int i0 = base + u * kStride + l * 4;
-      const float fm = i0 < V ? ftab[static_cast<unsigned>(i0) / kGemmBN] : 0.f;
-      float e[4] = {v[u].x * fm, v[u].y * fm, v[u].z * fm, v[u].w * fm};
+      float e[4] = {v[u].x * fm[u], v[u].y * fm[u], v[u].z * fm[u], v[u].w * fm[u]};
       bool keep[4];
       int k = 0;
 #pragma unroll
@@ -540,8 +537,7 @@ __device__ RowNucleus nucleus(const float* et, const float* st, float* fg, long 
       } else {
         cnt = static_cast<int>(V) - ps.cnt_ge;
         mass_hi = ps.mass_ge;
-        lo = ps.min_lt;
-        hi = ps.max_lt + 1u;
+        hi = kFirstMid;  // lo stays 0
         probe2 = true;
       }
       if (cnt == 0) {  // only by rounding, with top_p within an ulp of 1
@@ -731,7 +727,6 @@ __global__ void __launch_bounds__(kThreads, 4) spec_row_kernel(const SpecParams 
   const bool verifier = r < Pv;
   if (!verifier) r -= Pv;
   const float* et = (verifier ? p.ev : p.ed) + r * p.ldz;
-  prefetch_row(et, p.ldz * 4);
   const RowNucleus n = nucleus(et, (verifier ? p.stats_v : p.stats_d) + r * sld,
                                (verifier ? p.f_v : p.f_d) + r * p.tiles, p.V, p.tiles, p.scale,
                                p.top_p, ftab, listA, listB, sh);
@@ -822,6 +817,10 @@ __device__ void step_tie_bases(const float* et, const float* ftab, const RowNucl
   const int w = warp_id(), l = lane_id();
   for (int st = w; st < nsteps; st += NW) {
     const long long i0 = static_cast<long long>(st) * kStep + l * 4;
+    if (ftab[static_cast<long long>(st) * kStep / kGemmBN] < n.b) {  // no e reaches b here
+      if (l == 0) base[st] = 0;
+      continue;
+    }
     const float4 v = load_e(et, ftab, i0, V);
     int t = 0;
 #pragma unroll
@@ -853,20 +852,28 @@ __device__ int sample(const float* ep, const float* fp, const RowNucleus& np, co
   const bool part_p = np.c < np.eq, part_q = have_q && nq.c < nq.eq;
   if (part_p) step_tie_bases<NW>(ep, fp, np, V, nsteps, tp);
   if (part_q) step_tie_bases<NW>(eq, fq, nq, V, nsteps, tq);
-  // mass of every step
+  // mass of every step; p is 0 where e < b, so a step of a tile whose maximum
+  // f_t lies below b has none (and is not read)
   constexpr int kU = 2;
   for (int s0 = w; s0 < nsteps; s0 += kU * NW) {
     float4 vp[kU], vq[kU];
+    bool live[kU];
 #pragma unroll
     for (int k = 0; k < kU; ++k) {
-      const long long i0 = static_cast<long long>(s0 + k * NW) * kStep + l * 4;
-      vp[k] = load_e(ep, fp, i0, V);
-      vq[k] = have_q ? load_e(eq, fq, i0, V) : make_float4(0.f, 0.f, 0.f, 0.f);
+      const int st = s0 + k * NW;
+      const long long i0 = static_cast<long long>(st) * kStep + l * 4;
+      live[k] = st < nsteps && fp[static_cast<long long>(st) * kStep / kGemmBN] >= np.b;
+      vp[k] = live[k] ? load_e(ep, fp, i0, V) : make_float4(0.f, 0.f, 0.f, 0.f);
+      vq[k] = live[k] && have_q ? load_e(eq, fq, i0, V) : make_float4(0.f, 0.f, 0.f, 0.f);
     }
 #pragma unroll
     for (int k = 0; k < kU; ++k) {
       const int st = s0 + k * NW;
       if (st >= nsteps) break;
+      if (!live[k]) {  // warp-uniform
+        if (l == 0) cum[st] = 0.f;
+        continue;
+      }
       const long long i0 = static_cast<long long>(st) * kStep + l * 4;
       float a[4], c[4] = {0.f, 0.f, 0.f, 0.f};
       probs4(vp[k], i0, V, np, ip, part_p ? tp[st] : 0, a);
@@ -1014,8 +1021,6 @@ __global__ void __launch_bounds__(kSampleWarps * 32) spec_sample_kernel(const Sp
     const long long pos_v = static_cast<long long>(b) * G1 + k;
     const RowNucleus np = load_state(p.state_v + pos_v * kSpecStateWords);
     const float* ev = p.ev + pos_v * p.ldz;
-    prefetch_row(ev, p.ldz * 4);
-    if (k < p.gamma) prefetch_row(p.ed + (static_cast<long long>(b) * p.gamma + k) * p.ldz, p.ldz * 4);
     for (int t = threadIdx.x; t < p.tiles; t += kSampleWarps * 32) fp[t] = p.f_v[pos_v * p.tiles + t];
     const float u = p.u[pos_v * 2 + 1];
     if (k < p.gamma) {
