@@ -108,7 +108,7 @@ struct Plan {
   int elt = 2;
   int ntt = 0, nvt = 0;
   // forward
-  int S = 1, nparts = 0, merge_blocks = 0;
+  int S = 1, nparts = 0, merge_blocks = 0, eval_merge_blocks = 0;
   size_t off_part = 0, off_bsum = 0, off_bcnt = 0, fwd_bytes = 0;
   // backward
   long long group = 0, ngroups = 0;
@@ -174,7 +174,8 @@ Plan make_plan(const mls_problem* p, int pairs) {
   pl.nvt = static_cast<int>(ceil_div(V, kHeadBN));
   pl.S = choose_splits(pl.ntt, pl.nvt, pairs);
   pl.nparts = pl.S;
-  pl.merge_blocks = static_cast<int>(ceil_div(T, kMergeThreads));
+  pl.merge_blocks = static_cast<int>(ceil_div(T, kMergeTokens));
+  pl.eval_merge_blocks = static_cast<int>(ceil_div(T, kEvalMergeTokens));
   size_t o = 0;
   pl.off_part = o;
   o = align_up(o + sizeof(float) * static_cast<size_t>(pl.nparts) * kPartFields * M * T);
@@ -224,9 +225,9 @@ Plan make_plan(const mls_problem* p, int pairs) {
   pl.off_epart = o;
   o = align_up(o + sizeof(float) * static_cast<size_t>(pl.eval_S) * kEvalFields * T);
   pl.off_eacc = o;
-  o = align_up(o + sizeof(double) * 2 * kMaxModels * kMaxModels * static_cast<size_t>(pl.merge_blocks + 1));
+  o = align_up(o + sizeof(double) * 2 * kMaxModels * kMaxModels * static_cast<size_t>(pl.eval_merge_blocks + 1));
   pl.off_ecnt = o;
-  o = align_up(o + sizeof(long long) * static_cast<size_t>(pl.merge_blocks + 1));
+  o = align_up(o + sizeof(long long) * static_cast<size_t>(pl.eval_merge_blocks + 1));
   pl.eval_bytes = o;
 
   pl.total = pl.fwd_bytes > pl.bwd_bytes ? pl.fwd_bytes : pl.bwd_bytes;
@@ -804,10 +805,10 @@ extern "C" int mls_head_pairwise(const mls_problem* p, const void* const* H, con
   mp.block_acc = reinterpret_cast<double*>(wsb + pl.off_eacc);
   mp.block_cnt = reinterpret_cast<long long*>(wsb + pl.off_ecnt);
   mp.status = dev->status;
-  if ((rc = timed("pairwise_merge", s, [&] { return launch_eval_merge(mp, pl.merge_blocks, s); })))
+  if ((rc = timed("pairwise_merge", s, [&] { return launch_eval_merge(mp, pl.eval_merge_blocks, s); })))
     return rc;
   return timed("pairwise_final", s, [&] {
-    return launch_eval_final(mp.block_acc, mp.block_cnt, pl.merge_blocks, p->M, pair_stats, s);
+    return launch_eval_final(mp.block_acc, mp.block_cnt, pl.eval_merge_blocks, p->M, pair_stats, s);
   });
 }
 

@@ -245,7 +245,8 @@ struct MergeParams {
   int* status;
 };
 
-constexpr int kMergeThreads = 128;
+constexpr int kMergeTokens = 8;        // tokens per merge block: one warp per token
+constexpr int kEvalMergeTokens = 128;  // tokens per evaluation-merge block: one thread per token
 
 // Launchers (return the cudaError_t of the launch).
 cudaError_t launch_head_fwd(const HeadParams& p, bool tf32, bool tau_one, cudaStream_t s);

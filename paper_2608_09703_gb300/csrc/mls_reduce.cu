@@ -1,7 +1,7 @@
 // Row reductions of the forward pass, the token count of the backward and an
 // fp32 transpose (used only for fp32 inputs, whose tf32 GEMMs read K-major copies).
 //
-// merge_kernel: one thread per token combines the partial row states that the
+// merge_kernel: one warp per token combines the partial row states that the
 // head kernel wrote per (CTA, half tile) into
 //   lse_m    = logsumexp(z_m)            CE_m = lse_m - z_m[y]
 //   lset_m   = logsumexp(z_m / tau)
@@ -35,17 +35,32 @@ __device__ __forceinline__ double block_sum_double(double v, double* sh) {
   return s;  // valid in thread 0
 }
 
-__global__ void __launch_bounds__(kMergeThreads) merge_kernel(const __grid_constant__ MergeParams p) {
-  __shared__ double sh[kMergeThreads / 32];
-  const long long t = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
+__device__ __forceinline__ float warp_max_f(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+__device__ __forceinline__ float warp_sum_f(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// One warp per token: lane k takes partials k, k + 32, ...; warp reductions
+// (butterflies, so every lane holds the same result and the order is fixed)
+// combine them, and lane 0 writes the token's outputs.
+__global__ void __launch_bounds__(kMergeTokens * 32) merge_kernel(const __grid_constant__ MergeParams p) {
+  __shared__ double sh_sum[kMergeTokens], sh_cnt[kMergeTokens];
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const long long t = static_cast<long long>(blockIdx.x) * kMergeTokens + w;
   double contrib = 0.0, cnt = 0.0;
-  if (t < p.T) {
+  if (t < p.T) {  // warp-uniform
     const long long T = p.T;
     const long long MT = static_cast<long long>(p.M) * T;
     const long long PS = kPartFields * MT;  // stride between partials
     const int y = p.y[t];
     const bool bad = y >= p.V;
-    if (bad) atomicOr(p.status, kStatusBadTarget);
+    if (bad && lane == 0) atomicOr(p.status, kStatusBadTarget);
     const bool valid = y >= 0 && !bad;
     const float invtau = 1.0f / p.tau;
     const int tc = p.teacher;
@@ -53,18 +68,19 @@ __global__ void __launch_bounds__(kMergeThreads) merge_kernel(const __grid_const
 
     // teacher: row maximum, sums at tau = 1 and tau, teacher-weighted sum B
     float mT = -INFINITY;
-    for (int k = 0; k < p.nparts; ++k) mT = fmaxf(mT, Pt[k * PS + kPartMax * MT]);
+    for (int k = lane; k < p.nparts; k += 32) mT = fmaxf(mT, Pt[k * PS + kPartMax * MT]);
+    mT = warp_max_f(mT);
     // The teacher's weighted sum is relative to its own maximum:
     // B_k = sum q~ (z - m_k) log2(e)/tau; moving it to the row maximum mT adds
     // (m_k - mT) log2(e)/tau per unit of weight before the weights are rescaled.
     float s1T = 0.f, stT = 0.f, bT = 0.f, zT = 0.f;
     int amT = INT_MAX;
-    for (int k = 0; k < p.nparts; ++k) {
+    for (int k = lane; k < p.nparts; k += 32) {
       const float* P = Pt + k * PS;
       const float mk = P[kPartMax * MT];
-      const float f1 = exp2f((mk - mT) * p.L1);
-      const float ft = exp2f((mk - mT) * p.Ltau);
       if (mk != -INFINITY) {
+        const float f1 = exp2f((mk - mT) * p.L1);
+        const float ft = exp2f((mk - mT) * p.Ltau);
         const float stk = P[kPartSumTau * MT];
         s1T += P[kPartSum1 * MT] * f1;
         stT += stk * ft;
@@ -73,6 +89,11 @@ __global__ void __launch_bounds__(kMergeThreads) merge_kernel(const __grid_const
       zT += P[kPartTarget * MT];
       if (mk == mT) amT = min(amT, __float_as_int(P[kPartArgmax * MT]));
     }
+    s1T = warp_sum_f(s1T);
+    stT = warp_sum_f(stT);
+    bT = warp_sum_f(bT);
+    zT = warp_sum_f(zT);
+    amT = __reduce_min_sync(0xffffffffu, amT);
     const float lseT = mT + logf(s1T);
     const float lsetT = mT * invtau + logf(stT);
     // H(q) = log S - E_q[(z - mT)/tau]; both terms are >= 0
@@ -92,10 +113,11 @@ __global__ void __launch_bounds__(kMergeThreads) merge_kernel(const __grid_const
       } else {
         const float* Pm = p.part + static_cast<long long>(m) * T + t;
         float mm = -INFINITY;
-        for (int k = 0; k < p.nparts; ++k) mm = fmaxf(mm, Pm[k * PS + kPartMax * MT]);
+        for (int k = lane; k < p.nparts; k += 32) mm = fmaxf(mm, Pm[k * PS + kPartMax * MT]);
+        mm = warp_max_f(mm);
         float s1 = 0.f, st = 0.f, A = 0.f, zy = 0.f;
         am = INT_MAX;
-        for (int k = 0; k < p.nparts; ++k) {
+        for (int k = lane; k < p.nparts; k += 32) {
           const float* P = Pm + k * PS;
           const float mk = P[kPartMax * MT];
           if (mk != -INFINITY) {
@@ -107,6 +129,11 @@ __global__ void __launch_bounds__(kMergeThreads) merge_kernel(const __grid_const
           zy += P[kPartTarget * MT];
           if (mk == mm) am = min(am, __float_as_int(P[kPartArgmax * MT]));
         }
+        s1 = warp_sum_f(s1);
+        st = warp_sum_f(st);
+        A = warp_sum_f(A);
+        zy = warp_sum_f(zy);
+        am = __reduce_min_sync(0xffffffffu, am);
         lse = mm + logf(s1);
         lset = mm * invtau + logf(st);
         ce = lse - zy;
@@ -115,23 +142,33 @@ __global__ void __launch_bounds__(kMergeThreads) merge_kernel(const __grid_const
         L = (1.f - p.alpha) * ce + p.alpha * ld;
       }
       if (!valid) ce = ld = kl = L = 0.f;
-      const long long o = static_cast<long long>(m) * T + t;
-      p.tok_loss[o] = L;
-      if (p.tok_diag) {
-        p.tok_diag[o] = ce;
-        p.tok_diag[MT + o] = ld;
-        p.tok_diag[2 * MT + o] = kl;
+      if (lane == 0) {
+        const long long o = static_cast<long long>(m) * T + t;
+        p.tok_loss[o] = L;
+        if (p.tok_diag) {
+          p.tok_diag[o] = ce;
+          p.tok_diag[MT + o] = ld;
+          p.tok_diag[2 * MT + o] = kl;
+        }
+        if (p.argmax) p.argmax[o] = am;
+        p.stats[o] = lse;
+        p.stats[MT + o] = lset;
       }
-      if (p.argmax) p.argmax[o] = am;
-      p.stats[o] = lse;
-      p.stats[MT + o] = lset;
       contrib += static_cast<double>(p.w[m]) * static_cast<double>(L);
     }
     cnt = valid ? 1.0 : 0.0;
   }
-  const double bs = block_sum_double(contrib, sh);
-  const double bc = block_sum_double(cnt, sh);
+  if (lane == 0) {
+    sh_sum[w] = contrib;
+    sh_cnt[w] = cnt;
+  }
+  __syncthreads();
   if (threadIdx.x == 0) {
+    double bs = 0.0, bc = 0.0;
+    for (int i = 0; i < kMergeTokens; ++i) {
+      bs += sh_sum[i];
+      bc += sh_cnt[i];
+    }
     p.block_sum[blockIdx.x] = bs;
     p.block_cnt[blockIdx.x] = static_cast<long long>(bc);
   }
@@ -202,7 +239,7 @@ cudaError_t launch_transpose(const float* in, long long rows, long long cols, lo
 
 cudaError_t launch_merge(const MergeParams& p, int blocks, cudaStream_t s) {
   if (blocks <= 0) return cudaSuccess;
-  merge_kernel<<<blocks, kMergeThreads, 0, s>>>(p);
+  merge_kernel<<<blocks, kMergeTokens * 32, 0, s>>>(p);
   return cudaGetLastError();
 }
 
