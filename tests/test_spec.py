@@ -328,3 +328,27 @@ def test_spec_argument_errors():
     with pytest.raises(B.MLSError) as ei:
         B.mls_spec_verify(p, h, w, h, w, t, u, o, o, ws[:1024])
     assert ei.value.code == B.MLS_ERR_WORKSPACE
+
+
+def test_spec_tiny_top_p_is_greedy_at_suite_shape():
+    """top_p -> 0 keeps only the most likely token (ties apart), so with drafts
+    equal to the draft model's argmax, nucleus verification must reproduce
+    greedy verification exactly: accept while the verifier's argmax agrees,
+    then emit it (the residual max(0, p - q) is one-hot there).  Checked on
+    the benchmark's shape, every sequence, against the greedy path itself."""
+    wl = synth.SPEC_WORKLOADS["spec_suite3"]
+    Hd, Wd, Hv, Wv = synth.make_spec_inputs(wl, 51, device="cuda")
+    u = synth.make_uniforms(wl.B, wl.gamma, 51, device="cuda")
+    zd = Hd.float() @ Wd.float().T
+    draft = zd.argmax(1).to(torch.int32).reshape(wl.B, wl.gamma)
+    # the verifier agrees on a prefix of varying length
+    n_g, nx_g = run_gpu(wl, Hd, Wd, Hv, Wv, draft, u, greedy=True)
+    n_s, nx_s = run_gpu(wl, Hd, Wd, Hv, Wv, draft, u, greedy=False, top_p=1e-6)
+    assert (n_s == n_g).all() and (nx_s == nx_g).all()
+    assert 0 < n_g.mean() < wl.gamma
+
+
+def test_spec_long_drafts():
+    wl = synth.SpecWorkload("long", B=6, gamma=16, V=1500, d_draft=64, d_verify=128, extra=0.05)
+    n, _, _ = check(wl, *inputs(wl, 52))
+    assert n.max() > 4
