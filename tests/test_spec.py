@@ -340,7 +340,7 @@ def test_spec_tiny_top_p_is_greedy_at_suite_shape():
     Hd, Wd, Hv, Wv = synth.make_spec_inputs(wl, 51, device="cuda")
     u = synth.make_uniforms(wl.B, wl.gamma, 51, device="cuda")
     zd = Hd.float() @ Wd.float().T
-    draft = zd.argmax(1).to(torch.int32).reshape(wl.B, wl.gamma)
+    draft = zd.argmax(1).to(torch.int32).reshape(wl.B, wl.gamma).cpu().numpy()
     # the verifier agrees on a prefix of varying length
     n_g, nx_g = run_gpu(wl, Hd, Wd, Hv, Wv, draft, u, greedy=True)
     n_s, nx_s = run_gpu(wl, Hd, Wd, Hv, Wv, draft, u, greedy=False, top_p=1e-6)
