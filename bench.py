@@ -165,44 +165,47 @@ def aggregate(ms_local: float, tokens_per_rank: int, world: int):
 
 
 # ------------------------------------------------------------------------- oracle timing
-def oracle_sample(wl, ntok: int, seed: int = 1234):
-    """The first `ntok` tokens of the workload's seeded inputs, as oracle arrays."""
+def oracle_sample(wl, ntok: int, seed: int = 1234, tensors=None):
+    """The first `ntok` tokens of the workload's seeded inputs (or of the given
+    (H, W, y) tensors), as oracle arrays."""
     import numpy as np
 
     from paper_2608_09703_gb300 import synth
 
-    H, W, y = synth.make_inputs(wl, seed=seed)
+    H, W, y = tensors if tensors is not None else synth.make_inputs(wl, seed=seed)
     Hs = synth.as_oracle_arrays([h[:ntok] for h in H])
     Ws = synth.as_oracle_arrays(W)
-    return Hs, Ws, y[:ntok].numpy().astype(np.int32)
+    return Hs, Ws, y[:ntok].cpu().numpy().astype(np.int32)
 
 
 def oracle_step(wl, Hs, Ws, ys):
     from oracle import oracle
 
     kw = dict(teacher=wl.teacher_index, tau=wl.tau, alpha=wl.alpha, w=wl.weights)
-    oracle.forward(Hs, Ws, ys, **kw)
+    fwd = oracle.forward(Hs, Ws, ys, **kw)
     oracle.backward(Hs, Ws, ys, **kw)
+    return fwd
 
 
-def oracle_rate(wl, budget_s: float, seed: int = 1234):
+def oracle_rate(wl, budget_s: float, seed: int = 1234, tensors=None):
     """Calibrates the sample size to ~budget_s of CPU work, then times one
-    forward+backward of the oracle on it.  Returns (tokens/s, tokens, seconds)."""
+    forward+backward of the oracle on it.  Returns (tokens/s, tokens,
+    seconds, the oracle's forward results on the sample)."""
     from oracle import oracle
 
     oracle.build()
     # the oracle runs one token per thread: calibrate with one token per thread
     ncal = max(2, oracle.threads())
-    Hs, Ws, ys = oracle_sample(wl, ncal, seed)
+    Hs, Ws, ys = oracle_sample(wl, ncal, seed, tensors)
     t0 = time.perf_counter()
     oracle_step(wl, Hs, Ws, ys)
     per_tok = (time.perf_counter() - t0) / ncal
     ntok = int(max(2, min(wl.T, budget_s / max(per_tok, 1e-6))))
-    Hs, Ws, ys = oracle_sample(wl, ntok, seed)
+    Hs, Ws, ys = oracle_sample(wl, ntok, seed, tensors)
     t0 = time.perf_counter()
-    oracle_step(wl, Hs, Ws, ys)
+    fwd = oracle_step(wl, Hs, Ws, ys)
     dt = time.perf_counter() - t0
-    return ntok / dt, ntok, dt
+    return ntok / dt, ntok, dt, fwd
 
 
 def reference_arm(args, rank, world):
@@ -278,9 +281,15 @@ def gpu_arm(args, rank, world, local):
     op = B.HeadLoss(wl.d, wl.T, wl.V, teacher=wl.teacher_index, tau=wl.tau, alpha=wl.alpha,
                     w=wl.weights, dtype=torch.bfloat16, device=dev, vocab_group=args.vocab_group)
 
+    nvtx = torch.cuda.nvtx
+
     def step():
+        nvtx.range_push("mls_head_loss_fwd")
         op.forward(H, W, y)
+        nvtx.range_pop()
+        nvtx.range_push("mls_head_loss_bwd")
         op.backward(H, W, y)
+        nvtx.range_pop()
 
     for _ in range(args.warmup):
         step()
@@ -298,10 +307,12 @@ def gpu_arm(args, rank, world, local):
     sampler.start()
     time.sleep(0.25)
     B.mls_profile_enable(True)
+    nvtx.range_push("timed_steps")
     e0.record(stream)
     for _ in range(args.steps):
         step()
     e1.record(stream)
+    nvtx.range_pop()
     torch.cuda.synchronize()
     kern = B.mls_profile_read()
     B.mls_profile_enable(False)
@@ -363,27 +374,47 @@ def gpu_arm(args, rank, world, local):
     # ---- inter-model junctions (Eq. 1) of the suite, forward + backward
     junction = None
     if not args.no_junction:
+        nvtx.range_push("junction")
         junction = junction_run(args, wl, dev, float(pk["hbm_gbs"]))
+        nvtx.range_pop()
 
     # ---- speculative-decoding verify step (draft 1024 / verifier 3072 of the suite)
     spec = None
     if not args.no_spec:
+        nvtx.range_push("spec_verify")
         spec = spec_run(args, dev, pk)
+        nvtx.range_pop()
 
     # ---- end to end through the C ABI with host buffers (pinned), copies timed
     e2e = None
     if not args.no_e2e:
+        nvtx.range_push("end_to_end")
         e2e = e2e_run(args, op, H, W, y, world, stream, wl)
+        nvtx.range_pop()
     if rank != 0:
         return
     cpu = None
+    parity = None
     if world == 1 and not args.no_cpu_baseline:
-        rate, ntok, secs = oracle_rate(wl, budget_s=15.0)
+        # the oracle on the first tokens of the very inputs the GPU ran
+        rate, ntok, secs, ref = oracle_rate(wl, budget_s=15.0, tensors=(H, W, y))
         from oracle import oracle
 
         cpu = {"value": rate, "unit": UNIT, "cores": oracle.threads(), "kind": "oracle",
                "sample": f"first {ntok} of {wl.T} tokens of {wl.name} (full V and widths), "
                          f"fp64 forward+backward, {secs:.1f} s"}
+        # parity of the timed GPU step's per-token outputs on that sample
+        import numpy as np
+
+        got = op.tok_loss[:, :ntok].double().cpu().numpy()
+        diag = op.tok_diag[:, :, :ntok].double().cpu().numpy()
+        rel = lambda a, b: float(np.max(np.abs(a - b) / np.maximum(np.abs(b), 1e-30)))
+        kl_err = float(np.max(np.abs(diag[2] - ref["kl"]) / np.maximum(1.0, ref["ld"])))
+        parity = {"tokens": ntok, "max_rel_err_tok_loss": rel(got, ref["tok_loss"]),
+                  "max_rel_err_ce": rel(diag[0], ref["ce"]), "max_rel_err_ld": rel(diag[1], ref["ld"]),
+                  "max_err_kl_vs_max1_ld": kl_err,
+                  "argmax_agree": float(np.mean(op.argmax[:, :ntok].cpu().numpy() == ref["argmax"])),
+                  "tolerance": "per-token losses 1e-3 relative; KL 1e-3 * max(1, Ld)"}
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True, "scaling": "weak",
@@ -394,7 +425,7 @@ def gpu_arm(args, rank, world, local):
         "tensor_frac_step_sustained": step_flops / (ms_max / 1e3) / 1e12 / peak,
         "roofline": roofline, "kernels": per_kernel, "gpu_launches": gpu_launches,
         "clocks": clocks, "e2e": e2e, "cpu_baseline": cpu, "pairwise_eval": pairwise,
-        "junction": junction, "spec_verify": spec,
+        "junction": junction, "spec_verify": spec, "parity_sample": parity,
     }
     print(json.dumps(line), flush=True)
 
