@@ -57,7 +57,8 @@ enum {
   MLS_ERR_CUDA = -5,         /* a CUDA runtime call or kernel launch failed */
   MLS_ERR_DEVICE = -6,       /* current device is not a compute-capability 10.3 GPU */
   MLS_STATUS_BAD_TARGET = 1, /* some target was >= V; that token was treated as ignored */
-  MLS_STATUS_TIMEOUT = 2     /* a pipeline wait exceeded its bound; outputs are invalid */
+  MLS_STATUS_TIMEOUT = 2,    /* a pipeline wait exceeded its bound; outputs are invalid */
+  MLS_STATUS_CHECK = 4       /* checked build only: an internal invariant failed */
 };
 
 /* Maximum number of sub-models per call. */

@@ -13,14 +13,17 @@ from typing import Optional, Sequence
 
 import torch
 
-_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libmls.so")
+# MLS_CHECKED=1 selects the checked build (invariant checks in the kernels).
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)),
+                         "libmls_checked.so" if os.environ.get("MLS_CHECKED") == "1"
+                         else "libmls.so")
 _lib = None
 
 MLS_BF16, MLS_FP32 = 0, 1
 MLS_OK = 0
 MLS_ERR_ARG, MLS_ERR_ALIGN, MLS_ERR_UNSUPPORTED = -1, -2, -3
 MLS_ERR_WORKSPACE, MLS_ERR_CUDA, MLS_ERR_DEVICE = -4, -5, -6
-MLS_STATUS_BAD_TARGET, MLS_STATUS_TIMEOUT = 1, 2
+MLS_STATUS_BAD_TARGET, MLS_STATUS_TIMEOUT, MLS_STATUS_CHECK = 1, 2, 4
 MLS_MAX_MODELS = 4
 
 
@@ -73,7 +76,8 @@ def lib():
     if _lib is None:
         if not os.path.exists(_LIB_PATH):
             raise RuntimeError(f"{_LIB_PATH} is missing: build it with "
-                               "`python -m paper_2608_09703_gb300.build`")
+                               "`python -m paper_2608_09703_gb300.build`"
+                               + (" --checked" if _LIB_PATH.endswith("_checked.so") else ""))
         L = ctypes.CDLL(_LIB_PATH)
         P = ctypes.POINTER(mls_problem)
         vp = ctypes.c_void_p

@@ -1,9 +1,12 @@
 """Builds the CUDA library libmls.so in-tree for sm_103a (GB300).
 
 Each translation unit under csrc/ is compiled by its own nvcc process (in
-parallel), then linked into paper_2608_09703_gb300/libmls.so.  Usage:
+parallel), then linked into paper_2608_09703_gb300/libmls.so.  With --checked
+the same sources are built with -DMLS_CHECKED into libmls_checked.so, whose
+kernels also check internal invariants and raise MLS_STATUS_CHECK when one
+fails (the binding loads it when MLS_CHECKED=1 is set).  Usage:
 
-    python -m paper_2608_09703_gb300.build [--verbose-ptxas] [--force]
+    python -m paper_2608_09703_gb300.build [--verbose-ptxas] [--force] [--checked]
 """
 from __future__ import annotations
 
@@ -19,6 +22,8 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libmls.so")
+BUILD_CHECKED = os.path.join(PKG, "_build_checked")
+LIB_CHECKED = os.path.join(PKG, "libmls_checked.so")
 SOURCES = ["mls_api.cu", "mls_head.cu", "mls_gemm.cu", "mls_reduce.cu", "mls_eval.cu",
            "mls_junction.cu", "mls_spec.cu"]
 HEADERS = ["mls_device.cuh", "mls_kernels.h"]
@@ -32,11 +37,13 @@ def nvcc() -> str:
     raise RuntimeError("nvcc not found")
 
 
-def _flags(verbose_ptxas: bool):
+def _flags(verbose_ptxas: bool, checked: bool = False):
     f = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-O2",
                 "-I", os.path.join(ROOT, "include"), "-I", CSRC]
     if verbose_ptxas:
         f += ["-Xptxas", "-v"]
+    if checked:
+        f += ["-DMLS_CHECKED"]
     return f
 
 
@@ -47,44 +54,47 @@ def _stale(target: str, deps) -> bool:
     return any(os.path.getmtime(d) > t for d in deps)
 
 
-def _compile(src: str, verbose_ptxas: bool, force: bool) -> tuple[str, str]:
-    obj = os.path.join(BUILD, os.path.splitext(src)[0] + ".o")
+def _compile(src: str, verbose_ptxas: bool, force: bool, checked: bool = False) -> tuple[str, str]:
+    obj = os.path.join(BUILD_CHECKED if checked else BUILD, os.path.splitext(src)[0] + ".o")
     deps = [os.path.join(CSRC, src)] + [os.path.join(CSRC, h) for h in HEADERS] + \
         [os.path.join(ROOT, "include", "mls.h")]
     if not force and not verbose_ptxas and not _stale(obj, deps):
         return obj, ""
-    cmd = [nvcc()] + _flags(verbose_ptxas) + ["-c", os.path.join(CSRC, src), "-o", obj]
+    cmd = [nvcc()] + _flags(verbose_ptxas, checked) + ["-c", os.path.join(CSRC, src), "-o", obj]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"nvcc failed for {src}:\n{r.stdout}\n{r.stderr}")
     return obj, r.stdout + r.stderr
 
 
-def build(verbose_ptxas: bool = False, force: bool = False, quiet: bool = True) -> str:
-    os.makedirs(BUILD, exist_ok=True)
+def build(verbose_ptxas: bool = False, force: bool = False, quiet: bool = True,
+          checked: bool = False) -> str:
+    lib = LIB_CHECKED if checked else LIB
+    os.makedirs(BUILD_CHECKED if checked else BUILD, exist_ok=True)
     with cf.ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
-        results = list(ex.map(lambda s: _compile(s, verbose_ptxas, force), SOURCES))
+        results = list(ex.map(lambda s: _compile(s, verbose_ptxas, force, checked), SOURCES))
     objs = [o for o, _ in results]
     if verbose_ptxas or not quiet:
         for o, log in results:
             if log:
                 sys.stdout.write(f"== {os.path.basename(o)}\n{log}")
-    if force or _stale(LIB, objs):
-        tmp = LIB + f".tmp{os.getpid()}"
+    if force or _stale(lib, objs):
+        tmp = lib + f".tmp{os.getpid()}"
         cmd = [nvcc()] + ARCH + ["-shared", "-o", tmp] + objs
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
             raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
-        os.replace(tmp, LIB)
-    return LIB
+        os.replace(tmp, lib)
+    return lib
 
 
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--verbose-ptxas", action="store_true")
     ap.add_argument("--force", action="store_true")
+    ap.add_argument("--checked", action="store_true")
     a = ap.parse_args()
-    print(build(verbose_ptxas=a.verbose_ptxas, force=a.force, quiet=False))
+    print(build(verbose_ptxas=a.verbose_ptxas, force=a.force, quiet=False, checked=a.checked))
 
 
 if __name__ == "__main__":

@@ -617,6 +617,7 @@ extern "C" const char* mls_strerror(int code) {
     case MLS_STATUS_BAD_TARGET: return "a target was >= V (token ignored)";
     case MLS_STATUS_TIMEOUT: return "a pipeline wait timed out; outputs are invalid";
     case MLS_STATUS_BAD_TARGET | MLS_STATUS_TIMEOUT: return "target >= V and a pipeline timeout";
+    case MLS_STATUS_CHECK: return "an internal invariant failed (checked build)";
     default: return "unknown code";
   }
 }
@@ -955,6 +956,7 @@ extern "C" int mls_spec_verify(const mls_spec_problem* p, const void* H_draft, c
   sp.state_d = at(pl.off_sd);
   sp.n_accepted = n_accepted;
   sp.next_token = next_token;
+  sp.status = dev->status;
 
   // Logits of the verify positions: one GEMM launch over the verifier's rows
   // and (sampling) the draft's, z = H W^T with both operands K-major; its

@@ -14,6 +14,21 @@ namespace mls {
 // Bits OR-ed into the library's device status word (see mls.h).
 constexpr int kStatusBadTarget = 1;
 constexpr int kStatusTimeout = 2;
+constexpr int kStatusCheck = 4;
+
+// Invariant checks of the checked build (-DMLS_CHECKED, libmls_checked.so):
+// a failed condition raises kStatusCheck in the status word and execution
+// continues; in the normal build they compile to nothing.
+#ifdef MLS_CHECKED
+#define MLS_CHECK(status, cond)                                  \
+  do {                                                           \
+    if (!(cond)) atomicOr((status), ::mls::kStatusCheck);        \
+  } while (0)
+#else
+#define MLS_CHECK(status, cond) \
+  do {                          \
+  } while (0)
+#endif
 
 // A pipeline wait gives up after this long (ns) and raises kStatusTimeout.
 // Legitimate waits in these kernels last microseconds.

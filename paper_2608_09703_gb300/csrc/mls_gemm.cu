@@ -110,6 +110,9 @@ __device__ __forceinline__ void gemm_producer(const GemmParams& p, uint32_t base
   for (int j = 0; ok && (t = pair_tile(p, pair, npairs, j)) >= 0; ++j) {
     const TileCoord tc = decode_tile(p, t);
     const GemmProblem& pr = p.prob[tc.prob];
+    MLS_CHECK(p.status, t < p.total_tiles && tc.prob < p.nprob && pr.a_map < kGemmMaxProblems &&
+                            static_cast<long long>(tc.tm) * kPairM < pr.Mrows &&
+                            static_cast<long long>(tc.tn) * kGemmBN < pr.Ncols);
     const bool amn = a_mn_of<kAMode>(pr);
     const CUtensorMap* ma = &p.mapA[pr.a_map];
     const CUtensorMap* mb = &p.mapB[pr.b_map];

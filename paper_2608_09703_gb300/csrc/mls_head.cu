@@ -84,6 +84,8 @@ __device__ __forceinline__ void head_producer(const HeadParams& p, uint32_t base
   for (int vt = p.vt_begin + split; ok && vt < p.vt_end; vt += p.S) {
     for (int u = 0; ok && u < p.M; ++u) {
       const int m = p.order[u];
+      MLS_CHECK(p.status, m >= 0 && m < p.M && split < p.S &&
+                              static_cast<long long>(vt) * kHeadBN < p.V + kHeadBN);
       for (int kb = 0; kb < p.nk[m]; ++kb) {
         if (!mbar_wait(HeadSmem::empty(base, stage), phase ^ 1u, abort_flag, p.status)) {
           ok = false;
@@ -420,6 +422,7 @@ __device__ __forceinline__ void fwd_epilogue(const HeadParams& p, uint32_t base,
   const float accT = (mT == -INFINITY ? 0.f : fat * (aT + (mT - mTm) * Lt * stT)) +
                      (mT1 == -INFINITY ? 0.f : fbt * (X(kPartAcc, 0) + (mT1 - mTm) * Lt * stT1));
   const long long MT = static_cast<long long>(p.M) * p.T;
+  MLS_CHECK(p.status, split < p.S && row < p.T);
   float* P = p.part + static_cast<long long>(split) * kPartFields * MT;
   {
     float* Pt = P + static_cast<long long>(p.order[0]) * p.T + row;

@@ -222,6 +222,7 @@ struct SpecParams {
   float* state_v;                // [B * (gamma + 1)][kSpecStateWords]
   int* n_accepted;               // [B]
   int* next_token;               // [B]
+  int* status;                   // checked build: invariant failures
 };
 cudaError_t setup_spec_kernels();
 cudaError_t launch_spec_rows(const SpecParams& p, cudaStream_t s);

@@ -357,7 +357,7 @@ __device__ __forceinline__ void first_pass(const float* et, const float* ftab, i
 // Writes the row's tokens with key in [lo, lo + w) to dst in warp order,
 // this warp from slot `run`, never past cnt.
 __device__ __forceinline__ void row_compact(const float* et, const float* ftab, int V, uint32_t lo,
-                                            uint32_t w, float* dst, int run, int cnt) {
+                                            uint32_t w, float* dst, int run, int cnt, int* status) {
   const int l = lane_id();
   constexpr int kStride = kWarps * kStep;
   for (int base = warp_id() * kStep; base < V; base += kUnroll * kStride) {
@@ -386,7 +386,10 @@ __device__ __forceinline__ void row_compact(const float* et, const float* ftab, 
       int at = run + incl - k;
 #pragma unroll
       for (int j = 0; j < 4; ++j)
-        if (keep[j] && at < cnt) dst[at++] = e[j];
+        if (keep[j]) {
+          MLS_CHECK(status, at < cnt);
+          if (at < cnt) dst[at++] = e[j];
+        }
       run += __shfl_sync(0xffffffffu, incl, 31);
     }
   }
@@ -497,7 +500,7 @@ __device__ void finish_exact(const float* L, int n, float target, float mass_hi,
 // Nucleus of one row (e_t, per-tile stats st); writes f_t to fg.
 __device__ RowNucleus nucleus(const float* et, const float* st, float* fg, long long V, int tiles,
                               float scale, float top_p, float* ftab, float* listA, float* listB,
-                              Shared& sh) {
+                              Shared& sh, int* status) {
   RowNucleus r;
   row_stats(st, tiles, scale, ftab, fg, r.m, r.S, sh);
   const float target = top_p * r.S;
@@ -607,7 +610,7 @@ __device__ RowNucleus nucleus(const float* et, const float* st, float* fg, long 
         warp_bases(side, sh);
         int run = sh.wbase[warp_id()];
         if (list == nullptr) {
-          row_compact(et, ftab, static_cast<int>(V), lo, hi - lo, dst, run, cnt);
+          row_compact(et, ftab, static_cast<int>(V), lo, hi - lo, dst, run, cnt, status);
         } else {
           for (int base = warp_id() * 32; base < n_list; base += kThreads) {
             const int i = base + lane_id();
@@ -619,6 +622,7 @@ __device__ RowNucleus nucleus(const float* et, const float* st, float* fg, long 
             }
             const unsigned bal = __ballot_sync(0xffffffffu, keep);
             const int at = run + __popc(bal & ((1u << lane_id()) - 1u));
+            if (keep) MLS_CHECK(status, at < cnt);
             if (keep && at < cnt) dst[at] = e;
             run += __popc(bal);
           }
@@ -632,6 +636,7 @@ __device__ RowNucleus nucleus(const float* et, const float* st, float* fg, long 
         resolved = true;
         break;
       }
+      MLS_CHECK(status, pass < 39);  // hi - lo at least halves each pass
     }
   }
   r.b = __uint_as_float(lo);
@@ -729,7 +734,7 @@ __global__ void __launch_bounds__(kThreads, 4) spec_row_kernel(const SpecParams 
   const float* et = (verifier ? p.ev : p.ed) + r * p.ldz;
   const RowNucleus n = nucleus(et, (verifier ? p.stats_v : p.stats_d) + r * sld,
                                (verifier ? p.f_v : p.f_d) + r * p.tiles, p.V, p.tiles, p.scale,
-                               p.top_p, ftab, listA, listB, sh);
+                               p.top_p, ftab, listA, listB, sh, p.status);
   if (threadIdx.x == 0) store_state((verifier ? p.state_v : p.state_d) + r * kSpecStateWords, n);
 }
 
@@ -845,7 +850,7 @@ __device__ void step_tie_bases(const float* et, const float* ftab, const RowNucl
 template <int NW>
 __device__ int sample(const float* ep, const float* fp, const RowNucleus& np, const float* eq,
                       const float* fq, const RowNucleus& nq, bool have_q, long long V, float u,
-                      float* cum, int* tp, int* tq, SharedT<NW>& sh) {
+                      float* cum, int* tp, int* tq, SharedT<NW>& sh, int* status) {
   const int nsteps = static_cast<int>((V + kStep - 1) / kStep);
   const int w = warp_id(), l = lane_id();
   const float ip = 1.f / np.kept, iq = have_q ? 1.f / nq.kept : 0.f;
@@ -905,6 +910,8 @@ __device__ int sample(const float* ep, const float* fp, const RowNucleus& np, co
       for (int st = nsteps - 1; st >= 0 && owner < 0; --st)
         if (cum[st] > (st > 0 ? cum[st - 1] : 0.f)) owner = st;
       before = -INFINITY;  // pick its last token with mass
+      MLS_CHECK(status, owner >= 0);
+      if (owner < 0) owner = 0;
     } else {
       before = owner > 0 ? cum[owner - 1] : 0.f;
     }
@@ -1028,10 +1035,10 @@ __global__ void __launch_bounds__(kSampleWarps * 32) spec_sample_kernel(const Sp
       const RowNucleus nq = load_state(p.state_d + pos_d * kSpecStateWords);
       for (int t = threadIdx.x; t < p.tiles; t += kSampleWarps * 32) fq[t] = p.f_d[pos_d * p.tiles + t];
       __syncthreads();
-      next = sample(ev, fp, np, p.ed + pos_d * p.ldz, fq, nq, true, p.V, u, cum, tp, tq, sh);
+      next = sample(ev, fp, np, p.ed + pos_d * p.ldz, fq, nq, true, p.V, u, cum, tp, tq, sh, p.status);
     }
     __syncthreads();
-    if (next < 0) next = sample(ev, fp, np, ev, fp, np, false, p.V, u, cum, tp, tq, sh);
+    if (next < 0) next = sample(ev, fp, np, ev, fp, np, false, p.V, u, cum, tp, tq, sh, p.status);
     if (next < 0) next = static_cast<int>(p.V - 1);  // unreachable: the maximum has e = 1
   }
   if (threadIdx.x == 0) {

@@ -124,3 +124,14 @@ def test_spec_verify_validation_without_gpu(lib):
     # sampling keeps a per-tile table in shared memory: V <= 4096 tiles of 256
     assert call(B.spec_problem(4, 2, 4096 * 256 + 1, 64, 64)) == B.MLS_ERR_UNSUPPORTED
     assert B.mls_spec_workspace_size(B.spec_problem(4, 2, 4096 * 256 + 1, 64, 64, greedy=True)) > 0
+
+
+def test_checked_build_compiles():
+    """The checked build (invariant checks compiled in) builds and exports the
+    same entry points as the normal one."""
+    path = mbuild.build(checked=True)
+    out = subprocess.run(["nm", "-D", "--defined-only", path], capture_output=True, text=True,
+                         check=True).stdout
+    exported = set(l.split()[-1] for l in out.splitlines() if l.strip())
+    for name in declared_functions():
+        assert name in exported, name
