@@ -25,8 +25,8 @@ namespace {
 struct EvalSmem {
   static constexpr uint32_t kA = 0;
   static constexpr uint32_t kB = kEvalStages * kEvalABytes;
-  static constexpr uint32_t kX = kB + kEvalStages * kEvalBBytes;  // half-merge exchange
-  static constexpr uint32_t kBar = kX + kEvalXchg;
+  static constexpr uint32_t kX = kA;  // half-merge exchange, after the main loop only
+  static constexpr uint32_t kBar = kB + kEvalStages * kEvalBBytes;
   static __device__ __forceinline__ uint32_t full(uint32_t b, int s) { return b + kBar + 8u * s; }
   static __device__ __forceinline__ uint32_t empty(uint32_t b, int s) {
     return b + kBar + 8u * (kEvalStages + s);

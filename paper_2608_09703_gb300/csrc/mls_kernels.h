@@ -143,13 +143,16 @@ struct GemmParams {
 // for every ordered pair (s, j), D_sj = sum_v exp(z_s[v] - max_s) (z_s[v] - z_j[v]).
 constexpr int kEvalBN = 128;     // vocabulary columns per tile
 constexpr int kEvalBHalf = 64;   // rows of W per CTA
-constexpr int kEvalStages = 8;
+constexpr int kEvalStages = 9;
 constexpr uint32_t kEvalABytes = kHeadBM * 128;
 constexpr uint32_t kEvalBBytes = kEvalBHalf * 128;
 // per token and split: max_s (4), sum_s (4), argmax_s (4), D_sj for j != s (4 x 3)
 constexpr int kEvalFields = 24;
 constexpr uint32_t kEvalXchg = kEvalFields * kHeadBM * 4;
-constexpr uint32_t kEvalSmem = kEvalStages * (kEvalABytes + kEvalBBytes) + kEvalXchg + 1024 + 1024;
+// The half-merge exchange is only used after the main loop, when the operand
+// stages are idle, so it shares their memory.
+constexpr uint32_t kEvalSmem = kEvalStages * (kEvalABytes + kEvalBBytes) + 1024 + 1024;
+static_assert(kEvalXchg <= kEvalStages * (kEvalABytes + kEvalBBytes), "exchange fits in the stages");
 
 struct EvalParams {
   CUtensorMap mapH[kMaxModels];  // H_m [T, d_m], box {128 B of K, kHeadBM rows}
