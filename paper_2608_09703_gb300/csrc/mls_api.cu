@@ -783,6 +783,16 @@ extern "C" int mls_head_pairwise(const mls_problem* p, const void* const* H, con
     ep.nk[m] = static_cast<int>(ceil_div(p->d[m], KE));
   }
   ep.M = p->M;
+  // units of a vocabulary tile, widest sub-model first (it overlaps the epilogue)
+  for (int i = 0; i < p->M; ++i) ep.order[i] = i;
+  for (int i = 0; i < p->M; ++i)
+    for (int k = i + 1; k < p->M; ++k)
+      if (p->d[ep.order[k]] > p->d[ep.order[i]]) {
+        const int t = ep.order[i];
+        ep.order[i] = ep.order[k];
+        ep.order[k] = t;
+      }
+  for (int i = 0; i < p->M; ++i) ep.pos[ep.order[i]] = i;
   ep.ntt = pl.ntt;
   ep.nvt = pl.eval_nvt;
   ep.S = pl.eval_S;

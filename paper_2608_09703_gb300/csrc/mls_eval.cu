@@ -11,9 +11,12 @@
 // accumulates, per sub-model s, the running max, sum_v exp(z_s - max_s) and
 // D_sj = sum_v exp(z_s - max_s) (z_s - z_j) for every j != s (the difference
 // is taken element by element, so nearly equal sub-models lose no precision).
-// The accumulators are single-buffered: the next tile's MMAs wait for the
-// epilogue.  Roles: warp 8 TMA producer, warp 9 MMA issuer (even CTA), warps
-// 0-7 epilogue (one thread per token and 64 columns).
+// TMEM is a ring of four 128-column slots: the u-th unit (one sub-model of one
+// vocabulary tile, widest sub-model first) goes to slot u mod 4 and waits only
+// for that slot's previous tile to be drained, so at M = 3 the next tile's
+// widest unit runs during the epilogue (M = 2: full double buffering; M = 4:
+// one tile at a time).  Roles: warp 8 TMA producer, warp 9 MMA issuer (even
+// CTA), warps 0-7 epilogue (one thread per token and 64 columns).
 #include <climits>
 
 #include "mls_device.cuh"
@@ -31,14 +34,17 @@ struct EvalSmem {
   static __device__ __forceinline__ uint32_t empty(uint32_t b, int s) {
     return b + kBar + 8u * (kEvalStages + s);
   }
-  static __device__ __forceinline__ uint32_t accf(uint32_t b) { return b + kBar + 8u * (2 * kEvalStages); }
-  static __device__ __forceinline__ uint32_t acce(uint32_t b) {
-    return b + kBar + 8u * (2 * kEvalStages + 1);
+  // tile j's accumulators are complete: accf(j mod 4); slot s drained: slote(s)
+  static __device__ __forceinline__ uint32_t accf(uint32_t b, int j) {
+    return b + kBar + 8u * (2 * kEvalStages + (j & 3));
+  }
+  static __device__ __forceinline__ uint32_t slote(uint32_t b, int s) {
+    return b + kBar + 8u * (2 * kEvalStages + 4 + s);
   }
   static __device__ __forceinline__ uint32_t drain(uint32_t b) {
-    return b + kBar + 8u * (2 * kEvalStages + 2);
+    return b + kBar + 8u * (2 * kEvalStages + 8);
   }
-  static constexpr uint32_t kTmemSlot = kBar + 8u * (2 * kEvalStages + 3);
+  static constexpr uint32_t kTmemSlot = kBar + 8u * (2 * kEvalStages + 9);
   static constexpr uint32_t kAbort = kTmemSlot + 4;
   static constexpr uint32_t kEnd = kAbort + 4;
 };
@@ -60,7 +66,8 @@ __device__ __forceinline__ void eval_producer(const EvalParams& p, uint32_t base
   uint32_t phase = 0, filled = 0, lastpar = 0;
   bool ok = true;
   for (int vt = split; ok && vt < p.nvt; vt += p.S) {
-    for (int m = 0; ok && m < p.M; ++m) {
+    for (int i = 0; ok && i < p.M; ++i) {
+      const int m = p.order[i];
       for (int kb = 0; kb < p.nk[m]; ++kb) {
         if (!mbar_wait(EvalSmem::empty(base, stage), phase ^ 1u, abort_flag, p.status)) {
           ok = false;
@@ -95,13 +102,24 @@ __device__ __forceinline__ void eval_mma(const EvalParams& p, uint32_t base, uin
                                          int split, volatile int* abort_flag) {
   constexpr uint32_t kIdesc = make_idesc(2 * kHeadBM, kEvalBN, kTF32, false, false);
   int stage = 0;
-  uint32_t phase = 0, par = 0;
+  uint32_t phase = 0;
+  int uses[4] = {0, 0, 0, 0};  // times each TMEM slot has been handed out
   bool ok = true;
-  for (int vt = split; ok && vt < p.nvt; vt += p.S) {
-    if (!mbar_wait(EvalSmem::acce(base), par ^ 1u, abort_flag, p.status)) break;
-    tc_fence_after();
-    for (int m = 0; ok && m < p.M; ++m) {
-      const uint32_t d = tmem + static_cast<uint32_t>(m) * kEvalBN;
+  int j = 0;
+  for (int vt = split; ok && vt < p.nvt; vt += p.S, ++j) {
+    for (int i = 0; ok && i < p.M; ++i) {
+      const int m = p.order[i];
+      const int slot = (j * p.M + i) & 3;
+      // the n-th use of a slot waits for its (n-1)-th drain
+      if (uses[slot] > 0 &&
+          !mbar_wait(EvalSmem::slote(base, slot), static_cast<uint32_t>(uses[slot] - 1) & 1u,
+                     abort_flag, p.status)) {
+        ok = false;
+        break;
+      }
+      ++uses[slot];
+      tc_fence_after();
+      const uint32_t d = tmem + static_cast<uint32_t>(slot) * kEvalBN;
       for (int kb = 0; kb < p.nk[m]; ++kb) {
         if (!mbar_wait(EvalSmem::full(base, stage), phase, abort_flag, p.status)) {
           ok = false;
@@ -121,8 +139,7 @@ __device__ __forceinline__ void eval_mma(const EvalParams& p, uint32_t base, uin
       }
     }
     if (!ok) break;
-    mma_commit_pair(EvalSmem::accf(base), 0x3);
-    par ^= 1u;
+    mma_commit_pair(EvalSmem::accf(base, j), 0x3);
   }
   mma_commit_pair(EvalSmem::drain(base), 0x1);
   mbar_wait_drain(EvalSmem::drain(base), 0, kDrainNs);
@@ -194,10 +211,11 @@ __device__ __forceinline__ void eval_epilogue(const EvalParams& p, uint32_t base
 #pragma unroll
     for (int j = 0; j < kMaxModels; ++j) st.d[s][j] = 0.f;
   }
-  uint32_t par = 0;
   float z[kMaxModels][32];
-  for (int vt = split; vt < p.nvt; vt += p.S) {
-    const bool ok = mbar_wait(EvalSmem::accf(base), par, abort_flag, p.status);
+  int j = 0;
+  for (int vt = split; vt < p.nvt; vt += p.S, ++j) {
+    const bool ok = mbar_wait(EvalSmem::accf(base, j), static_cast<uint32_t>(j >> 2) & 1u,
+                              abort_flag, p.status);
     if (!__all_sync(0xffffffffu, ok)) break;
     tc_fence_after();
 #pragma unroll
@@ -207,7 +225,10 @@ __device__ __forceinline__ void eval_epilogue(const EvalParams& p, uint32_t base
       if (nvalid == 0) continue;  // warp-uniform
 #pragma unroll
       for (int s = 0; s < kMaxModels; ++s)
-        if (s < M) tmem_ld32(tl + static_cast<uint32_t>(s * kEvalBN + c * 32), z[s]);
+        if (s < M) {
+          const uint32_t slot = static_cast<uint32_t>(j * M + p.pos[s]) & 3u;
+          tmem_ld32(tl + slot * kEvalBN + static_cast<uint32_t>(c * 32), z[s]);
+        }
       if (nvalid == 32)
         eval_chunk<false>(z, M, 32, col0, L1, st);
       else
@@ -215,8 +236,9 @@ __device__ __forceinline__ void eval_epilogue(const EvalParams& p, uint32_t base
     }
     tc_fence_before();
     __syncwarp();
-    if (lane == 0) mbar_arrive_remote(map_to_rank(EvalSmem::acce(base), 0));
-    par ^= 1u;
+    if (lane == 0)
+      for (int i = 0; i < M; ++i)
+        mbar_arrive_remote(map_to_rank(EvalSmem::slote(base, (j * M + i) & 3), 0));
   }
 
   // the two column halves of a token combine through shared memory
@@ -271,8 +293,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kHeadThreads, 1)
       mbar_init(EvalSmem::full(base, s), 1);
       mbar_init(EvalSmem::empty(base, s), 1);
     }
-    mbar_init(EvalSmem::accf(base), 1);
-    mbar_init(EvalSmem::acce(base), 2 * kHeadEpiWarps);
+    for (int q = 0; q < 4; ++q) {
+      mbar_init(EvalSmem::accf(base, q), 1);
+      mbar_init(EvalSmem::slote(base, q), 2 * kHeadEpiWarps);
+    }
     mbar_init(EvalSmem::drain(base), 1);
     fence_barrier_init();
   }

@@ -158,6 +158,8 @@ struct EvalParams {
   CUtensorMap mapH[kMaxModels];  // H_m [T, d_m], box {128 B of K, kHeadBM rows}
   CUtensorMap mapW[kMaxModels];  // W_m [V, d_m], box {128 B of K, kEvalBHalf rows}
   int M;
+  int order[kMaxModels];         // units of a vocabulary tile, widest sub-model first
+  int pos[kMaxModels];           // pos[order[i]] = i
   int nk[kMaxModels];
   int ntt;                       // token tiles of 256 (one per CTA pair)
   int nvt;                       // vocabulary tiles of kEvalBN
