@@ -216,62 +216,111 @@ __device__ __forceinline__ void gemm_mma(const GemmParams& p, uint32_t base, uin
   mbar_wait_drain(GemmSmem::drain(base), 0, kDrainNs);
 }
 
+// Largest of 32 values, as a tree (depth 5, not a 32-step chain).
+__device__ __forceinline__ float max32(const float (&v)[32]) {
+  float m[16];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) m[i] = fmaxf(v[i], v[i + 16]);
+#pragma unroll
+  for (int w = 8; w > 0; w >>= 1)
+#pragma unroll
+    for (int i = 0; i < w; ++i) m[i] = fmaxf(m[i], m[i + w]);
+  return m[0];
+}
+
 // Row statistics epilogues (kEpiSoftmax, kEpiArgmax) of one 128 x kGemmBN
-// accumulator tile: each lane owns one row.  The maximum (and its first
-// column) come from one read of the row's accumulators; kEpiSoftmax reads
-// them again to store 2^((z - m_t) scale) and sum it in column order.
+// accumulator tile: each lane owns one row, and `ncols` of its columns lie
+// inside C.  kEpiArgmax reads the row's accumulators once for the maximum and
+// its first column.  kEpiSoftmax reads them once for the maximum m_t and again
+// to store e = 2^((z - m_t) scale) and sum it.
+// Each epilogue warp runs alone on its SM sub-partition, so latency is not
+// hidden by other warps; the softmax passes avoid long dependent chains (the
+// maximum is a tree, the sum four interleaved partial sums).  Its cost must
+// stay under the MMAs of the next tile, ~8.4k cycles for a K = 1024 tile; with
+// 32-step chains it took ~16k cycles.
 __device__ __noinline__ void epilogue_stats(const GemmProblem& pr, const CUtensorMap* mapC,
                                             uint32_t stage, uint32_t& count, uint32_t tacc,
                                             int tn, long long row, bool row_ok, int row0,
                                             int lane) {
   float v[32];
   float mt = -INFINITY;
-  int mi = tn * kGemmBN;
-#pragma unroll 1
-  for (int c = 0; c < kGemmBN / 32; ++c) {
-    tmem_ld32(tacc + c * 32, v);
-    const int col = tn * kGemmBN + c * 32;
-#pragma unroll
-    for (int i = 0; i < 32; ++i)
-      if (col + i < pr.Ncols && v[i] > mt) {
-        mt = v[i];
-        mi = col + i;
-      }
-  }
+  const int col0 = tn * kGemmBN;
+  const int ncols = pr.Ncols - col0;  // >= 1: a tile starts inside C
   float* srow = pr.stats + (row_ok ? row : 0) * pr.stats_ld + 2 * tn;
   if (pr.epi == kEpiArgmax) {
+    int mi = col0;
+#pragma unroll 1
+    for (int c = 0; c < kGemmBN / 32; ++c) {
+      tmem_ld32(tacc + c * 32, v);
+#pragma unroll
+      for (int i = 0; i < 32; ++i)
+        if (c * 32 + i < ncols && v[i] > mt) {
+          mt = v[i];
+          mi = col0 + c * 32 + i;
+        }
+    }
     if (row_ok) {
       srow[0] = mt;
       srow[1] = __int_as_float(mi);
     }
     return;
   }
+  const int nchunks = ncols < kGemmBN ? (ncols + 31) / 32 : kGemmBN / 32;
+#pragma unroll 1
+  for (int c = 0; c < nchunks; ++c) {
+    tmem_ld32(tacc + c * 32, v);
+    if (c * 32 + 32 > ncols) {
+#pragma unroll
+      for (int i = 0; i < 32; ++i)
+        if (c * 32 + i >= ncols) v[i] = -INFINITY;
+    }
+    mt = fmaxf(mt, max32(v));
+  }
+  // Two chunks (both staging buffers) per round: one proxy fence and one
+  // bulk group for 32 rows x 64 columns.
   float st = 0.f;
 #pragma unroll 1
-  for (int c = 0; c < kGemmBN / 32; ++c) {
-    tmem_ld32(tacc + c * 32, v);
-    const int col = tn * kGemmBN + c * 32;
+  for (int c = 0; c < nchunks; c += 2) {
+    float w[2][32];
+    tmem_ld32(tacc + c * 32, w[0]);
+    if (c + 1 < nchunks) tmem_ld32(tacc + c * 32 + 32, w[1]);
+    float s4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-    for (int i = 0; i < 32; ++i) {
-      v[i] = col + i < pr.Ncols ? fast_exp2((v[i] - mt) * pr.epi_scale) : 0.f;
-      st += v[i];
+    for (int h = 0; h < 2; ++h) {
+      const int cc = (c + h) * 32;
+      if (cc + 32 <= ncols) {
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          w[h][i] = fast_exp2((w[h][i] - mt) * pr.epi_scale);
+          s4[i & 3] += w[h][i];
+        }
+      } else {
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          w[h][i] = cc + i < ncols ? fast_exp2((w[h][i] - mt) * pr.epi_scale) : 0.f;
+          s4[i & 3] += w[h][i];
+        }
+      }
     }
-    if (col >= pr.Ncols) continue;  // warp-uniform
-    // 32 rows x 32 columns through shared memory; the TMA store drops rows
-    // and columns outside C.
-    const uint32_t buf = stage + (count & 1u) * GemmSmem::kChunk;
-    if (lane == 0) bulk_wait_read<1>();  // the store that last used this buffer has read it
+    st += (s4[0] + s4[1]) + (s4[2] + s4[3]);
+    // 32 rows x 32 columns per buffer through shared memory; the TMA store
+    // drops rows and columns outside C.
+    if (lane == 0) bulk_wait_read<0>();  // the previous round's stores have read both buffers
     __syncwarp();
-    const uint32_t rowaddr = buf + lane * 128;
 #pragma unroll
-    for (int j = 0; j < 8; ++j)
-      st_shared_v4(rowaddr + ((j ^ (lane & 7)) << 4), __float_as_uint(v[4 * j]),
-                   __float_as_uint(v[4 * j + 1]), __float_as_uint(v[4 * j + 2]),
-                   __float_as_uint(v[4 * j + 3]));
+    for (int h = 0; h < 2; ++h) {
+      const uint32_t rowaddr = stage + h * GemmSmem::kChunk + lane * 128;
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        st_shared_v4(rowaddr + ((j ^ (lane & 7)) << 4), __float_as_uint(w[h][4 * j]),
+                     __float_as_uint(w[h][4 * j + 1]), __float_as_uint(w[h][4 * j + 2]),
+                     __float_as_uint(w[h][4 * j + 3]));
+    }
     fence_proxy_async_smem();
     __syncwarp();
     if (lane == 0) {
-      tma_store_2d(mapC, buf, col, row0);
+      tma_store_2d(mapC, stage, col0 + c * 32, row0);
+      if (c + 1 < nchunks) tma_store_2d(mapC, stage + GemmSmem::kChunk, col0 + c * 32 + 32, row0);
       bulk_commit();
     }
     ++count;
