@@ -259,11 +259,17 @@ def workload(args):
 
 
 def workload_config(wl, world):
-    return {"workload": f"{wl.name}: 3-level Matryoshka suite head+CE+distillation, T={wl.T} tokens "
-                        f"(4x2048), d={list(wl.d)}, V={wl.V}, bf16, tau={wl.tau}, alpha={wl.alpha}",
+    elt = 2 if wl.dtype == "bf16" else 4
+    w_mb = wl.V * sum(wl.d) * elt / 1e6
+    seqs = f"{wl.T // 2048}x2048" if wl.T % 2048 == 0 else f"{wl.T}"
+    l2 = (f"inputs larger than L2 (W {w_mb:.0f} MB {wl.dtype}), no flush" if w_mb > 129
+          else f"inputs smaller than L2 (W {w_mb:.1f} MB {wl.dtype}), no flush")
+    return {"workload": f"{wl.name}: {len(wl.d)}-level Matryoshka suite head+CE+distillation, "
+                        f"T={wl.T} tokens ({seqs}), d={list(wl.d)}, V={wl.V}, {wl.dtype}, "
+                        f"tau={wl.tau}, alpha={wl.alpha}",
             "T": wl.T, "d": list(wl.d), "V": wl.V, "tau": wl.tau, "alpha": wl.alpha,
             "global_batch": wl.T * world, "seq_len": 2048, "parallelism": f"dp{world}",
-            "l2": "inputs larger than L2 (W 618 MB bf16), no flush"}
+            "l2": l2}
 
 
 # ------------------------------------------------------------------------- GPU arm
@@ -418,11 +424,16 @@ def gpu_arm(args, rank, world, local):
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded N(0,1) hidden states, "
-        "N(0,0.02^2) heads, uniform targets; FineWeb-Edu not available)",
+        "vs_baseline": None, "dtype": "bf16" if wl.dtype == "bf16" else "tf32",
+        "data": f"synthetic (seeded N(0,1) hidden states, N(0,{wl.w_sigma}^2) heads"
+        + (f" with the teacher's x{wl.teacher_scale:g}" if wl.teacher_scale != 1.0 else "")
+        + f", {wl.targets} targets; FineWeb-Edu not available)",
         "config": workload_config(wl, world),
         "tensor_frac_step": step_flops / (ms_max / 1e3) / 1e12 / burst,
         "tensor_frac_step_sustained": step_flops / (ms_max / 1e3) / 1e12 / peak,
+        # the model-FLOPs convention 6*T*V*sum(d), which leaves out the
+        # backward's recompute of the logits
+        "tensor_frac_step_6tvd": 0.75 * step_flops / (ms_max / 1e3) / 1e12 / burst,
         "roofline": roofline, "kernels": per_kernel, "gpu_launches": gpu_launches,
         "clocks": clocks, "e2e": e2e, "cpu_baseline": cpu, "pairwise_eval": pairwise,
         "junction": junction, "spec_verify": spec, "parity_sample": parity,

@@ -64,6 +64,10 @@ WORKLOADS = {
     "suite4": Workload("suite4", T=16384, d=(2048, 4096, 6144, 8192), V=128256, w_sigma=0.01),
     "stress": Workload("stress", T=32768, d=(1024, 2048, 4096), V=256000, tau=0.5,
                        teacher_scale=8.0, targets="zipf"),
+    # The paper's own 3B Matryoshka suite (Sec. 3.1, Table 1): widths
+    # 1024 / 2304 / 4352 and the 49,152-token vocabulary, at the same four
+    # packed 2048-token sequences as suite3.
+    "suite3_paper": Workload("suite3_paper", T=8192, d=(1024, 2304, 4352), V=49152),
 }
 
 

@@ -45,7 +45,7 @@ def test_small_ragged_bf16_teacher_not_last():
 
 
 @pytest.mark.parametrize("name,T", [("suite3", 136), ("suite3_big", 136), ("suite4", 24),
-                                    ("stress", 24)])
+                                    ("stress", 24), ("suite3_paper", 136)])
 def test_reduced_tokens_full_vocab(name, T):
     """Each benchmark workload at its full V, widths, tau and value
     distribution, with fewer tokens (ragged last token tile)."""
@@ -192,6 +192,6 @@ def _full_size(name, nsample, seed=21):
     return op
 
 
-@pytest.mark.parametrize("name", ["suite3", "suite3_big", "suite4", "stress"])
+@pytest.mark.parametrize("name", ["suite3", "suite3_big", "suite4", "stress", "suite3_paper"])
 def test_full_size_sampled(name):
     _full_size(name, nsample=10)
