@@ -5,24 +5,30 @@
 // Backward with g = dL/dx, s = ||e|| / ||o||:
 //   dL/do = s (g_o - o (g_o . o) / ||o||^2)
 //   dL/de = g_e + s (g_o . o) e / ||e||^2
-// Both are row reductions plus an elementwise pass, bound by HBM: one warp per
-// token, 16-byte vector accesses, fp32 sums; the second pass re-reads the row
-// from L1/L2.
+// Both are row reductions followed by an elementwise pass, bound by HBM.  One
+// warp owns a token.  It issues every 16-byte load of its row at once (o and
+// e, and g in the backward), keeps them packed in registers for the
+// elementwise pass, and so reads each input byte from HBM once with many loads
+// in flight: one row costs one memory latency.  A row segment (o, or e) needs
+// ceil(length / (32 * elements per 16 bytes)) vectors per lane; the kernels
+// are instantiated for 1, 2, 4, 8 and 12, and wider rows take a streaming
+// path that reads the row twice (the second time from L2).  Sums are fp32,
+// accumulated per lane in column order, then across the warp, in both paths.
 #include "mls_device.cuh"
 #include "mls_kernels.h"
 
 namespace mls {
 namespace {
 
-constexpr int kRowsPerBlock = 8;
+constexpr int kRowsPerBlock = 4;
 
+// 16 bytes of E <-> N fp32 values.
 template <typename E>
 struct Vec;
 template <>
 struct Vec<__nv_bfloat16> {
   static constexpr int N = 8;
-  static __device__ __forceinline__ void load(const void* p, float (&f)[8]) {
-    const uint4 u = *reinterpret_cast<const uint4*>(p);
+  static __device__ __forceinline__ void unpack(const uint4& u, float (&f)[8]) {
     const uint32_t w[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
@@ -32,30 +38,41 @@ struct Vec<__nv_bfloat16> {
       f[2 * i + 1] = v.y;
     }
   }
-  static __device__ __forceinline__ void store(void* p, const float (&f)[8]) {
+  static __device__ __forceinline__ uint4 pack(const float (&f)[8]) {
     uint32_t w[4];
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       __nv_bfloat162 h = __floats2bfloat162_rn(f[2 * i], f[2 * i + 1]);
       w[i] = *reinterpret_cast<uint32_t*>(&h);
     }
-    *reinterpret_cast<uint4*>(p) = make_uint4(w[0], w[1], w[2], w[3]);
+    return make_uint4(w[0], w[1], w[2], w[3]);
   }
 };
 template <>
 struct Vec<float> {
   static constexpr int N = 4;
-  static __device__ __forceinline__ void load(const void* p, float (&f)[4]) {
-    const float4 v = *reinterpret_cast<const float4*>(p);
-    f[0] = v.x;
-    f[1] = v.y;
-    f[2] = v.z;
-    f[3] = v.w;
+  static __device__ __forceinline__ void unpack(const uint4& u, float (&f)[4]) {
+    f[0] = __uint_as_float(u.x);
+    f[1] = __uint_as_float(u.y);
+    f[2] = __uint_as_float(u.z);
+    f[3] = __uint_as_float(u.w);
   }
-  static __device__ __forceinline__ void store(void* p, const float (&f)[4]) {
-    *reinterpret_cast<float4*>(p) = make_float4(f[0], f[1], f[2], f[3]);
+  static __device__ __forceinline__ uint4 pack(const float (&f)[4]) {
+    return make_uint4(__float_as_uint(f[0]), __float_as_uint(f[1]), __float_as_uint(f[2]),
+                      __float_as_uint(f[3]));
   }
 };
+
+__device__ __forceinline__ uint4 ld16(const void* p) { return *reinterpret_cast<const uint4*>(p); }
+__device__ __forceinline__ void st16(void* p, const uint4& v) { *reinterpret_cast<uint4*>(p) = v; }
+
+// Tells the compiler the cached vectors may have changed, so it re-unpacks
+// them after the reductions instead of keeping 8 floats per vector alive.
+template <int R>
+__device__ __forceinline__ void keep_packed(uint4 (&v)[R]) {
+#pragma unroll
+  for (int j = 0; j < R; ++j) asm volatile("" : "+r"(v[j].x), "+r"(v[j].y), "+r"(v[j].z), "+r"(v[j].w));
+}
 
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
@@ -63,52 +80,109 @@ __device__ __forceinline__ float warp_sum(float v) {
   return v;
 }
 
+// Lane `lane`'s vectors of a row segment of n elements: vector j holds
+// elements (32 j + lane) N ... + N - 1; those past n read as zeros.
+template <typename E, int R>
+__device__ __forceinline__ void load_seg(const E* row, int n, int lane, uint4 (&v)[R]) {
+  constexpr int N = Vec<E>::N;
+#pragma unroll
+  for (int j = 0; j < R; ++j) {
+    const int k = (j * 32 + lane) * N;
+    v[j] = k < n ? ld16(row + k) : make_uint4(0u, 0u, 0u, 0u);
+  }
+}
+
+template <typename E, int R>
+__device__ __forceinline__ float sumsq_cached(const uint4 (&v)[R]) {
+  constexpr int N = Vec<E>::N;
+  float acc = 0.f;
+#pragma unroll
+  for (int j = 0; j < R; ++j) {
+    float f[N];
+    Vec<E>::unpack(v[j], f);
+#pragma unroll
+    for (int i = 0; i < N; ++i) acc = fmaf(f[i], f[i], acc);
+  }
+  return acc;
+}
+
 template <typename E>
-__device__ __forceinline__ float sumsq(const E* row, int n, int lane) {
+__device__ __forceinline__ float sumsq_stream(const E* row, int n, int lane) {
   constexpr int N = Vec<E>::N;
   float acc = 0.f;
   for (int k = lane * N; k < n; k += 32 * N) {
     float f[N];
-    Vec<E>::load(row + k, f);
+    Vec<E>::unpack(ld16(row + k), f);
 #pragma unroll
     for (int i = 0; i < N; ++i) acc = fmaf(f[i], f[i], acc);
   }
-  return warp_sum(acc);
+  return acc;
 }
 
+struct FwdRow {
+  long long t;
+  int de;
+  const void *o, *e;
+  void *xo, *xe;
+};
+
 template <typename E>
-__global__ void __launch_bounds__(32 * kRowsPerBlock)
-    junction_fwd_kernel(const JunctionParams p) {
+__device__ __forceinline__ FwdRow fwd_row(const JunctionParams& p, long long t) {
+  const int de = p.d_next - p.d_prev;
+  E* x = static_cast<E*>(p.x) + t * p.d_next;
+  return {t, de, static_cast<const E*>(p.o) + t * p.d_prev, static_cast<const E*>(p.e) + t * de,
+          x + (p.embed_first ? de : 0), x + (p.embed_first ? 0 : p.d_prev)};
+}
+
+// kR > 0: both segments fit kR cached vectors per lane; kR == 0: streaming.
+template <typename E, int kR>
+__global__ void __launch_bounds__(32 * kRowsPerBlock) junction_fwd_kernel(const JunctionParams p) {
   constexpr int N = Vec<E>::N;
   const long long t = static_cast<long long>(blockIdx.x) * kRowsPerBlock + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (t >= p.T) return;
-  const int de = p.d_next - p.d_prev;
-  const E* o = static_cast<const E*>(p.o) + t * p.d_prev;
-  const E* e = static_cast<const E*>(p.e) + t * de;
-  E* x = static_cast<E*>(p.x) + t * p.d_next;
-  const float no = sqrtf(sumsq(o, p.d_prev, lane));
-  const float ne = sqrtf(sumsq(e, de, lane));
-  const float s = no > 0.f ? ne / no : 0.f;
-  E* xo = x + (p.embed_first ? de : 0);
-  E* xe = x + (p.embed_first ? 0 : p.d_prev);
-  for (int k = lane * N; k < p.d_prev; k += 32 * N) {
-    float f[N];
-    Vec<E>::load(o + k, f);
+  const FwdRow r = fwd_row<E>(p, t);
+  const E* o = static_cast<const E*>(r.o);
+  const E* e = static_cast<const E*>(r.e);
+  E* xo = static_cast<E*>(r.xo);
+  E* xe = static_cast<E*>(r.xe);
+  if constexpr (kR > 0) {
+    uint4 vo[kR], ve[kR];
+    load_seg<E, kR>(o, p.d_prev, lane, vo);
+    load_seg<E, kR>(e, r.de, lane, ve);
+    const float no = sqrtf(warp_sum(sumsq_cached<E, kR>(vo)));
+    const float ne = sqrtf(warp_sum(sumsq_cached<E, kR>(ve)));
+    const float s = no > 0.f ? ne / no : 0.f;
+    keep_packed(vo);
 #pragma unroll
-    for (int i = 0; i < N; ++i) f[i] *= s;
-    Vec<E>::store(xo + k, f);
-  }
-  for (int k = lane * N; k < de; k += 32 * N) {
-    float f[N];
-    Vec<E>::load(e + k, f);
-    Vec<E>::store(xe + k, f);
+    for (int j = 0; j < kR; ++j) {
+      const int k = (j * 32 + lane) * N;
+      if (k < p.d_prev) {
+        float f[N];
+        Vec<E>::unpack(vo[j], f);
+#pragma unroll
+        for (int i = 0; i < N; ++i) f[i] *= s;
+        st16(xo + k, Vec<E>::pack(f));
+      }
+      if (k < r.de) st16(xe + k, ve[j]);
+    }
+  } else {
+    const float no = sqrtf(warp_sum(sumsq_stream(o, p.d_prev, lane)));
+    const float ne = sqrtf(warp_sum(sumsq_stream(e, r.de, lane)));
+    const float s = no > 0.f ? ne / no : 0.f;
+    for (int k = lane * N; k < p.d_prev; k += 32 * N) {
+      float f[N];
+      Vec<E>::unpack(ld16(o + k), f);
+#pragma unroll
+      for (int i = 0; i < N; ++i) f[i] *= s;
+      st16(xo + k, Vec<E>::pack(f));
+    }
+    for (int k = lane * N; k < r.de; k += 32 * N) st16(xe + k, ld16(e + k));
   }
 }
 
-template <typename E>
-__global__ void __launch_bounds__(32 * kRowsPerBlock)
-    junction_bwd_kernel(const JunctionParams p) {
+template <typename E, int kR>
+__global__ void __launch_bounds__(32 * kRowsPerBlock) junction_bwd_kernel(const JunctionParams p) {
   constexpr int N = Vec<E>::N;
   const long long t = static_cast<long long>(blockIdx.x) * kRowsPerBlock + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
@@ -121,40 +195,131 @@ __global__ void __launch_bounds__(32 * kRowsPerBlock)
   const E* ge = g + (p.embed_first ? 0 : p.d_prev);
   E* d_o = static_cast<E*>(p.d_o) + t * p.d_prev;
   E* d_e = static_cast<E*>(p.d_e) + t * de;
-  float oo = 0.f, dot = 0.f;
-  for (int k = lane * N; k < p.d_prev; k += 32 * N) {
-    float fo[N], fg[N];
-    Vec<E>::load(o + k, fo);
-    Vec<E>::load(go + k, fg);
+  float oo = 0.f, dot = 0.f, ee;
+  if constexpr (kR > 0) {
+    // Every input vector of the row is loaded at once and stays in registers.
+    uint4 vo[kR], vg[kR], ve[kR], vge[kR];
+    load_seg<E, kR>(o, p.d_prev, lane, vo);
+    load_seg<E, kR>(go, p.d_prev, lane, vg);
+    load_seg<E, kR>(e, de, lane, ve);
+    load_seg<E, kR>(ge, de, lane, vge);
 #pragma unroll
-    for (int i = 0; i < N; ++i) {
-      oo = fmaf(fo[i], fo[i], oo);
-      dot = fmaf(fg[i], fo[i], dot);
+    for (int j = 0; j < kR; ++j) {
+      float fo[N], fg[N];
+      Vec<E>::unpack(vo[j], fo);
+      Vec<E>::unpack(vg[j], fg);
+#pragma unroll
+      for (int i = 0; i < N; ++i) {
+        oo = fmaf(fo[i], fo[i], oo);
+        dot = fmaf(fg[i], fo[i], dot);
+      }
+    }
+    oo = warp_sum(oo);
+    dot = warp_sum(dot);
+    ee = warp_sum(sumsq_cached<E, kR>(ve));
+    const float no = sqrtf(oo), ne = sqrtf(ee);
+    const float s = no > 0.f ? ne / no : 0.f;
+    const float co = no > 0.f ? dot / oo : 0.f;                    // (g_o . o) / ||o||^2
+    const float ce = (no > 0.f && ee > 0.f) ? s * dot / ee : 0.f;  // s (g_o . o) / ||e||^2
+    keep_packed(vo);
+    keep_packed(vg);
+    keep_packed(ve);
+#pragma unroll
+    for (int j = 0; j < kR; ++j) {
+      const int k = (j * 32 + lane) * N;
+      if (k < p.d_prev) {
+        float fo[N], fg[N], r[N];
+        Vec<E>::unpack(vo[j], fo);
+        Vec<E>::unpack(vg[j], fg);
+#pragma unroll
+        for (int i = 0; i < N; ++i) r[i] = s * fmaf(-fo[i], co, fg[i]);
+        st16(d_o + k, Vec<E>::pack(r));
+      }
+      if (k < de) {
+        float fe[N], fg[N], r[N];
+        Vec<E>::unpack(ve[j], fe);
+        Vec<E>::unpack(vge[j], fg);
+#pragma unroll
+        for (int i = 0; i < N; ++i) r[i] = fmaf(ce, fe[i], fg[i]);
+        st16(d_e + k, Vec<E>::pack(r));
+      }
+    }
+  } else {
+    for (int k = lane * N; k < p.d_prev; k += 32 * N) {
+      float fo[N], fg[N];
+      Vec<E>::unpack(ld16(o + k), fo);
+      Vec<E>::unpack(ld16(go + k), fg);
+#pragma unroll
+      for (int i = 0; i < N; ++i) {
+        oo = fmaf(fo[i], fo[i], oo);
+        dot = fmaf(fg[i], fo[i], dot);
+      }
+    }
+    oo = warp_sum(oo);
+    dot = warp_sum(dot);
+    ee = warp_sum(sumsq_stream(e, de, lane));
+    const float no = sqrtf(oo), ne = sqrtf(ee);
+    const float s = no > 0.f ? ne / no : 0.f;
+    const float co = no > 0.f ? dot / oo : 0.f;
+    const float ce = (no > 0.f && ee > 0.f) ? s * dot / ee : 0.f;
+    for (int k = lane * N; k < p.d_prev; k += 32 * N) {
+      float fo[N], fg[N], r[N];
+      Vec<E>::unpack(ld16(o + k), fo);
+      Vec<E>::unpack(ld16(go + k), fg);
+#pragma unroll
+      for (int i = 0; i < N; ++i) r[i] = s * fmaf(-fo[i], co, fg[i]);
+      st16(d_o + k, Vec<E>::pack(r));
+    }
+    for (int k = lane * N; k < de; k += 32 * N) {
+      float fe[N], fg[N], r[N];
+      Vec<E>::unpack(ld16(e + k), fe);
+      Vec<E>::unpack(ld16(ge + k), fg);
+#pragma unroll
+      for (int i = 0; i < N; ++i) r[i] = fmaf(ce, fe[i], fg[i]);
+      st16(d_e + k, Vec<E>::pack(r));
     }
   }
-  oo = warp_sum(oo);
-  dot = warp_sum(dot);
-  const float ee = sumsq(e, de, lane);
-  const float no = sqrtf(oo), ne = sqrtf(ee);
-  const float s = no > 0.f ? ne / no : 0.f;
-  const float co = no > 0.f ? dot / oo : 0.f;             // (g_o . o) / ||o||^2
-  const float ce = (no > 0.f && ee > 0.f) ? s * dot / ee : 0.f;  // s (g_o . o) / ||e||^2
-  for (int k = lane * N; k < p.d_prev; k += 32 * N) {
-    float fo[N], fg[N], r[N];
-    Vec<E>::load(o + k, fo);
-    Vec<E>::load(go + k, fg);
-#pragma unroll
-    for (int i = 0; i < N; ++i) r[i] = s * fmaf(-fo[i], co, fg[i]);
-    Vec<E>::store(d_o + k, r);
+}
+
+// Cached vectors per lane for a row whose segments are d_prev and d_next -
+// d_prev elements of `elt` bytes: the smallest of 1, 2, 4, 8, 12 that holds both,
+// or 0 (streaming) when a segment needs more than 12 (the backward then holds
+// 48 vectors, 192 registers, per lane).
+int cache_vectors(int d_prev, int d_next, int elt) {
+  const int per = 32 * (16 / elt);  // elements per cached vector across the warp
+  const int need_o = (d_prev + per - 1) / per, need_e = (d_next - d_prev + per - 1) / per;
+  const int need = need_o > need_e ? need_o : need_e;
+  for (const int r : {1, 2, 4, 8, 12})
+    if (need <= r) return r;
+  return 0;
+}
+
+template <typename E>
+cudaError_t fwd_launch(const JunctionParams& p, int r, unsigned blocks, cudaStream_t s) {
+  const dim3 b(32 * kRowsPerBlock);
+  switch (r) {
+    case 1: junction_fwd_kernel<E, 1><<<blocks, b, 0, s>>>(p); break;
+    case 2: junction_fwd_kernel<E, 2><<<blocks, b, 0, s>>>(p); break;
+    case 4: junction_fwd_kernel<E, 4><<<blocks, b, 0, s>>>(p); break;
+    case 8: junction_fwd_kernel<E, 8><<<blocks, b, 0, s>>>(p); break;
+    case 12: junction_fwd_kernel<E, 12><<<blocks, b, 0, s>>>(p); break;
+    default: junction_fwd_kernel<E, 0><<<blocks, b, 0, s>>>(p); break;
   }
-  for (int k = lane * N; k < de; k += 32 * N) {
-    float fe[N], fg[N], r[N];
-    Vec<E>::load(e + k, fe);
-    Vec<E>::load(ge + k, fg);
-#pragma unroll
-    for (int i = 0; i < N; ++i) r[i] = fmaf(ce, fe[i], fg[i]);
-    Vec<E>::store(d_e + k, r);
+  return cudaGetLastError();
+}
+
+template <typename E>
+cudaError_t bwd_launch(const JunctionParams& p, int r, unsigned blocks, cudaStream_t s) {
+  const dim3 b(32 * kRowsPerBlock);
+  switch (r) {
+    case 1: junction_bwd_kernel<E, 1><<<blocks, b, 0, s>>>(p); break;
+    case 2: junction_bwd_kernel<E, 2><<<blocks, b, 0, s>>>(p); break;
+    case 4: junction_bwd_kernel<E, 4><<<blocks, b, 0, s>>>(p); break;
+    case 8: junction_bwd_kernel<E, 8><<<blocks, b, 0, s>>>(p); break;
+    case 12: junction_bwd_kernel<E, 12><<<blocks, b, 0, s>>>(p); break;
+    default: junction_bwd_kernel<E, 0><<<blocks, b, 0, s>>>(p); break;
   }
+  return cudaGetLastError();
 }
 
 }  // namespace
@@ -162,21 +327,17 @@ __global__ void __launch_bounds__(32 * kRowsPerBlock)
 cudaError_t launch_junction_fwd(const JunctionParams& p, bool fp32, cudaStream_t s) {
   const long long blocks = (p.T + kRowsPerBlock - 1) / kRowsPerBlock;
   if (blocks <= 0) return cudaSuccess;
-  if (fp32)
-    junction_fwd_kernel<float><<<static_cast<unsigned>(blocks), 32 * kRowsPerBlock, 0, s>>>(p);
-  else
-    junction_fwd_kernel<__nv_bfloat16><<<static_cast<unsigned>(blocks), 32 * kRowsPerBlock, 0, s>>>(p);
-  return cudaGetLastError();
+  const int r = cache_vectors(p.d_prev, p.d_next, fp32 ? 4 : 2);
+  return fp32 ? fwd_launch<float>(p, r, static_cast<unsigned>(blocks), s)
+              : fwd_launch<__nv_bfloat16>(p, r, static_cast<unsigned>(blocks), s);
 }
 
 cudaError_t launch_junction_bwd(const JunctionParams& p, bool fp32, cudaStream_t s) {
   const long long blocks = (p.T + kRowsPerBlock - 1) / kRowsPerBlock;
   if (blocks <= 0) return cudaSuccess;
-  if (fp32)
-    junction_bwd_kernel<float><<<static_cast<unsigned>(blocks), 32 * kRowsPerBlock, 0, s>>>(p);
-  else
-    junction_bwd_kernel<__nv_bfloat16><<<static_cast<unsigned>(blocks), 32 * kRowsPerBlock, 0, s>>>(p);
-  return cudaGetLastError();
+  const int r = cache_vectors(p.d_prev, p.d_next, fp32 ? 4 : 2);
+  return fp32 ? bwd_launch<float>(p, r, static_cast<unsigned>(blocks), s)
+              : bwd_launch<__nv_bfloat16>(p, r, static_cast<unsigned>(blocks), s);
 }
 
 }  // namespace mls

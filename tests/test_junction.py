@@ -65,3 +65,33 @@ def test_junction_suite3_shapes_full_size(dp, dn):
     e = (torch.randn(T, dn - dp, generator=g) * 0.02).to(torch.bfloat16)
     gr = (torch.randn(T, dn, generator=g) * 1e-3).to(torch.bfloat16)
     compare(o, e, gr, False, tol_x=4e-3, tol_g=1e-2)
+
+
+# Each register-cache size of the kernels (16-byte vectors per lane per row
+# segment: 1, 2, 4, 8, 12) and the streaming path for wider segments, with
+# segments that end part-way through a vector round and a ragged last block.
+@pytest.mark.parametrize("dtype,dp,de", [
+    (torch.bfloat16, 72, 40),      # 1 vector
+    (torch.bfloat16, 264, 8),      # 2
+    (torch.bfloat16, 520, 1000),   # 4
+    (torch.bfloat16, 1800, 200),   # 8
+    (torch.bfloat16, 3072, 1024),  # 12
+    (torch.bfloat16, 3080, 16),    # o past 12: streaming
+    (torch.bfloat16, 64, 4096),    # e past 12: streaming
+    (torch.float32, 1536, 512),    # 12
+    (torch.float32, 1540, 4),      # streaming
+])
+def test_junction_cache_sizes(dtype, dp, de):
+    g = torch.Generator().manual_seed(44 + dp + de)
+    T = 37
+    o = (torch.randn(T, dp, generator=g) * 3).to(dtype)
+    e = (torch.randn(T, de, generator=g) * 0.1).to(dtype)
+    gr = torch.randn(T, dp + de, generator=g).to(dtype)
+    o[5] = 0   # ||o|| = 0: o~ = 0, dL/do = 0, dL/de = g_e
+    e[11] = 0  # ||e|| = 0: o~ = 0, dL/do = 0
+    bf = dtype == torch.bfloat16
+    for embed_first in (False, True):
+        x, d_o, d_e = compare(o, e, gr, embed_first, tol_x=4e-3 if bf else 1e-5,
+                              tol_g=1e-2 if bf else 1e-5)
+        assert np.abs(d_o[5]).max() == 0.0 and np.abs(d_o[11]).max() == 0.0
+        np.testing.assert_array_equal(d_e[5], gr[5, (0 if embed_first else dp):][:de].double().numpy())
