@@ -299,56 +299,98 @@ __device__ __forceinline__ void row_pass(const float* et, const float* ftab, int
   }
 }
 
+// The column tiles that can hold an e >= 2^-8 (f_t >= 2^-8, since every e of
+// tile t is at most f_t), in tile order, into kept[]; returns their number.
+// Needs ftab published; the trailing barrier publishes kept[].
+__device__ int kept_tiles(const float* ftab, int tiles, int* kept, Shared& sh) {
+  int nk = 0;
+  for (int c0 = 0; c0 < tiles; c0 += kThreads) {
+    const int t = c0 + static_cast<int>(threadIdx.x);
+    const bool keep = t < tiles && __float_as_uint(ftab[t]) >= kFirstMid;
+    const unsigned bal = __ballot_sync(0xffffffffu, keep);
+    if (lane_id() == 0) sh.wcnt[warp_id()] = __popc(bal);
+    __syncthreads();
+    int at = nk, total = 0;
+    for (int w = 0; w < kWarps; ++w) {
+      const int c = sh.wcnt[w];
+      if (w < warp_id()) at += c;
+      total += c;
+    }
+    if (keep) kept[at + __popc(bal & ((1u << lane_id()) - 1u))] = t;
+    nk += total;
+    __syncthreads();  // sh.wcnt is rewritten next
+  }
+  return nk;
+}
+
 // The first bisection pass over a row: the split at 2^-8 of the maximum.
-// Every e of column tile t is at most f_t, so only tiles with f_t >= 2^-8 are
-// read.  Mass and count of the upper side; its few tokens are also appended,
-// in this warp's visiting order, to its own region of kSpecListCap / kWarps
-// slots of `regions` (wrun counts them, also past the region's end).
+// Only the kept tiles are read.  Warp w takes kept[w], kept[w + kWarps], ...,
+// kFirstTiles of them per round with all their loads in flight, so a peaked
+// row (a few dozen kept tiles spread over the vocabulary) costs about one
+// memory latency.  Mass and count of the upper side; its few tokens are also
+// appended, in this warp's visiting order, to its own region of
+// kSpecListCap / kWarps slots of `regions` (wrun counts them, also past the
+// region's end).
 constexpr int kRegion = kSpecListCap / kWarps;
-__device__ __forceinline__ void first_pass(const float* et, const float* ftab, int V, float* regions,
-                                           PassStats& ps, int& wrun) {
+constexpr int kFirstTiles = 3;
+static_assert(kGemmBN == 2 * kStep, "a column tile is two 128-element steps");
+__device__ __forceinline__ void first_pass(const float* et, const float* ftab, const int* kept,
+                                           int nk, int V, float* regions, PassStats& ps,
+                                           int& wrun) {
   const int l = lane_id();
-  constexpr int kStride = kWarps * kStep;
   float* reg = regions + warp_id() * kRegion;
   wrun = 0;
-  for (int base = warp_id() * kStep; base < V; base += kUnroll * kStride) {
-    float4 v[kUnroll];
-    float fm[kUnroll];
+  for (int j0 = warp_id(); j0 < nk; j0 += kFirstTiles * kWarps) {
+    float4 v[kFirstTiles][2];
+    float fm[kFirstTiles];
+    int i0s[kFirstTiles];
 #pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      const int s0 = base + u * kStride, i0 = s0 + l * 4;
-      fm[u] = s0 < V ? ftab[static_cast<unsigned>(s0) / kGemmBN] : 0.f;  // warp-uniform
-      v[u] = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (__float_as_uint(fm[u]) >= kFirstMid && i0 < V)
-        v[u] = __ldg(reinterpret_cast<const float4*>(et + i0));
+    for (int u = 0; u < kFirstTiles; ++u) {
+      const int j = j0 + u * kWarps;
+      fm[u] = 0.f;
+      i0s[u] = V;
+      v[u][0] = v[u][1] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (j < nk) {  // warp-uniform
+        const int t = kept[j];
+        fm[u] = ftab[t];
+        i0s[u] = t * kGemmBN + l * 4;
+#pragma unroll
+        for (int h = 0; h < 2; ++h)
+          if (i0s[u] + h * kStep < V)
+            v[u][h] = __ldg(reinterpret_cast<const float4*>(et + i0s[u] + h * kStep));
+      }
     }
 #pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      if (__float_as_uint(fm[u]) < kFirstMid) continue;  // warp-uniform: nothing reaches 2^-8
-      const int i0 = base + u * kStride + l * 4;
-      const int nv = min(max(V - i0, 0), 4);
-      const float e[4] = {v[u].x * fm[u], v[u].y * fm[u], v[u].z * fm[u], v[u].w * fm[u]};
-      bool ge[4];
-      int k = 0;
+    for (int u = 0; u < kFirstTiles; ++u) {
+      if (j0 + u * kWarps >= nk) break;  // warp-uniform
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        ge[j] = j < nv && __float_as_uint(e[j]) >= kFirstMid;
-        if (ge[j]) {
-          ps.mass_ge += e[j];
-          ++k;
-        }
-      }
-      ps.cnt_ge += k;
-      if (__any_sync(0xffffffffu, k > 0)) {
-        const int incl = warp_incl_scan(k);
-        int at = wrun + incl - k;
+      for (int h = 0; h < 2; ++h) {
+        const int i0 = i0s[u] + h * kStep;
+        const int nv = min(max(V - i0, 0), 4);
+        const float e[4] = {v[u][h].x * fm[u], v[u][h].y * fm[u], v[u][h].z * fm[u],
+                            v[u][h].w * fm[u]};
+        bool ge[4];
+        int k = 0;
 #pragma unroll
-        for (int j = 0; j < 4; ++j)
+        for (int j = 0; j < 4; ++j) {
+          ge[j] = j < nv && __float_as_uint(e[j]) >= kFirstMid;
           if (ge[j]) {
-            if (at < kRegion) reg[at] = e[j];
-            ++at;
+            ps.mass_ge += e[j];
+            ++k;
           }
-        wrun += __shfl_sync(0xffffffffu, incl, 31);
+        }
+        ps.cnt_ge += k;
+        if (__any_sync(0xffffffffu, k > 0)) {
+          const int incl = warp_incl_scan(k);
+          int at = wrun + incl - k;
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            if (ge[j]) {
+              if (at < kRegion) reg[at] = e[j];
+              ++at;
+            }
+          wrun += __shfl_sync(0xffffffffu, incl, 31);
+        }
       }
     }
   }
@@ -518,7 +560,10 @@ __device__ RowNucleus nucleus(const float* et, const float* st, float* fg, long 
     {
       PassStats ps;
       int wrun = 0;
-      first_pass(et, ftab, static_cast<int>(V), listA, ps, wrun);
+      // The kept-tile list lives in listB until the upper side is copied there.
+      int* kept = reinterpret_cast<int*>(listB);
+      const int nk = kept_tiles(ftab, tiles, kept, sh);
+      first_pass(et, ftab, kept, nk, static_cast<int>(V), listA, ps, wrun);
       if (lane_id() == 0) sh.wcnt[warp_id()] = wrun;
       reduce_pass(ps, sh);  // its barriers also publish wcnt
       int cnt;
