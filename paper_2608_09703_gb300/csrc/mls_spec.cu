@@ -299,19 +299,22 @@ __device__ __forceinline__ void row_pass(const float* et, const float* ftab, int
   }
 }
 
-// The column tiles that can hold an e >= 2^-8 (f_t >= 2^-8, since every e of
-// tile t is at most f_t), in tile order, into kept[]; returns their number.
-// Needs ftab published; the trailing barrier publishes kept[].
-__device__ int kept_tiles(const float* ftab, int tiles, int* kept, Shared& sh) {
+// The column tiles whose factor f_t has a key of at least min_key (so the
+// only tiles that can hold an e >= that value, since every e of tile t is at
+// most f_t), in tile order, into kept[]; returns their number.  Needs ftab
+// published; the trailing barrier publishes kept[].
+template <int NW>
+__device__ int kept_tiles(const float* ftab, int tiles, uint32_t min_key, int* kept,
+                          SharedT<NW>& sh) {
   int nk = 0;
-  for (int c0 = 0; c0 < tiles; c0 += kThreads) {
+  for (int c0 = 0; c0 < tiles; c0 += NW * 32) {
     const int t = c0 + static_cast<int>(threadIdx.x);
-    const bool keep = t < tiles && __float_as_uint(ftab[t]) >= kFirstMid;
+    const bool keep = t < tiles && __float_as_uint(ftab[t]) >= min_key;
     const unsigned bal = __ballot_sync(0xffffffffu, keep);
     if (lane_id() == 0) sh.wcnt[warp_id()] = __popc(bal);
     __syncthreads();
     int at = nk, total = 0;
-    for (int w = 0; w < kWarps; ++w) {
+    for (int w = 0; w < NW; ++w) {
       const int c = sh.wcnt[w];
       if (w < warp_id()) at += c;
       total += c;
@@ -562,7 +565,7 @@ __device__ RowNucleus nucleus(const float* et, const float* st, float* fg, long 
       int wrun = 0;
       // The kept-tile list lives in listB until the upper side is copied there.
       int* kept = reinterpret_cast<int*>(listB);
-      const int nk = kept_tiles(ftab, tiles, kept, sh);
+      const int nk = kept_tiles(ftab, tiles, kFirstMid, kept, sh);
       first_pass(et, ftab, kept, nk, static_cast<int>(V), listA, ps, wrun);
       if (lane_id() == 0) sh.wcnt[warp_id()] = wrun;
       reduce_pass(ps, sh);  // its barriers also publish wcnt
@@ -891,46 +894,45 @@ __device__ void step_tie_bases(const float* et, const float* ftab, const RowNucl
 }
 
 // sample(r, u) over r_v = max(0, p_v - q_v) (have_q) or r_v = p_v; -1 when r
-// is all zero.  cum: nsteps floats; tp/tq: nsteps ints each.
+// is all zero.  cum: nsteps floats; tp/tq: nsteps ints each; live: one int
+// per column tile.
 template <int NW>
 __device__ int sample(const float* ep, const float* fp, const RowNucleus& np, const float* eq,
                       const float* fq, const RowNucleus& nq, bool have_q, long long V, float u,
-                      float* cum, int* tp, int* tq, SharedT<NW>& sh, int* status) {
+                      float* cum, int* tp, int* tq, int* live, SharedT<NW>& sh, int* status) {
   const int nsteps = static_cast<int>((V + kStep - 1) / kStep);
   const int w = warp_id(), l = lane_id();
   const float ip = 1.f / np.kept, iq = have_q ? 1.f / nq.kept : 0.f;
   const bool part_p = np.c < np.eq, part_q = have_q && nq.c < nq.eq;
   if (part_p) step_tie_bases<NW>(ep, fp, np, V, nsteps, tp);
   if (part_q) step_tie_bases<NW>(eq, fq, nq, V, nsteps, tq);
-  // mass of every step; p is 0 where e < b, so a step of a tile whose maximum
-  // f_t lies below b has none (and is not read)
-  constexpr int kU = 2;
-  for (int s0 = w; s0 < nsteps; s0 += kU * NW) {
-    float4 vp[kU], vq[kU];
-    bool live[kU];
+  // Mass of every step.  p is 0 where e < b, so only the tiles whose maximum
+  // f_t reaches b (listed in tile order) are read; warp w takes live tiles w,
+  // w + NW, ..., one tile (two steps, p and q) per round with all four loads
+  // in flight.  The other steps' masses are 0.
+  for (int st = threadIdx.x; st < nsteps; st += NW * 32) cum[st] = 0.f;
+  const int nlive = kept_tiles(fp, (nsteps * kStep + kGemmBN - 1) / kGemmBN,
+                               __float_as_uint(np.b), live, sh);  // its barriers publish cum
+  for (int j = w; j < nlive; j += NW) {
+    const int t = live[j];
+    float4 vp[2], vq[2];
 #pragma unroll
-    for (int k = 0; k < kU; ++k) {
-      const int st = s0 + k * NW;
-      const long long i0 = static_cast<long long>(st) * kStep + l * 4;
-      live[k] = st < nsteps && fp[static_cast<long long>(st) * kStep / kGemmBN] >= np.b;
-      vp[k] = live[k] ? load_e(ep, fp, i0, V) : make_float4(0.f, 0.f, 0.f, 0.f);
-      vq[k] = live[k] && have_q ? load_e(eq, fq, i0, V) : make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int h = 0; h < 2; ++h) {
+      const long long i0 = static_cast<long long>(t) * kGemmBN + h * kStep + l * 4;
+      vp[h] = load_e(ep, fp, i0, V);
+      vq[h] = have_q ? load_e(eq, fq, i0, V) : make_float4(0.f, 0.f, 0.f, 0.f);
     }
 #pragma unroll
-    for (int k = 0; k < kU; ++k) {
-      const int st = s0 + k * NW;
-      if (st >= nsteps) break;
-      if (!live[k]) {  // warp-uniform
-        if (l == 0) cum[st] = 0.f;
-        continue;
-      }
+    for (int h = 0; h < 2; ++h) {
+      const int st = t * (kGemmBN / kStep) + h;
+      if (st >= nsteps) break;  // warp-uniform
       const long long i0 = static_cast<long long>(st) * kStep + l * 4;
       float a[4], c[4] = {0.f, 0.f, 0.f, 0.f};
-      probs4(vp[k], i0, V, np, ip, part_p ? tp[st] : 0, a);
-      if (have_q) probs4(vq[k], i0, V, nq, iq, part_q ? tq[st] : 0, c);
+      probs4(vp[h], i0, V, np, ip, part_p ? tp[st] : 0, a);
+      if (have_q) probs4(vq[h], i0, V, nq, iq, part_q ? tq[st] : 0, c);
       float m = 0.f;
 #pragma unroll
-      for (int j = 0; j < 4; ++j) m += fmaxf(0.f, a[j] - c[j]);
+      for (int j2 = 0; j2 < 4; ++j2) m += fmaxf(0.f, a[j2] - c[j2]);
       m = warp_sum(m);
       if (l == 0) cum[st] = m;
     }
@@ -1026,7 +1028,8 @@ __global__ void __launch_bounds__(kSampleWarps * 32) spec_sample_kernel(const Sp
     float* cum = fq + p.tiles;
     int* tp = reinterpret_cast<int*>(cum + nsteps);
     int* tq = tp + nsteps;
-    int* acc = tq + nsteps;  // per drafted position: 1 accepted, 0 rejected, 2 undecided
+    int* live = tq + nsteps;  // the sampler's live tiles
+    int* acc = live + p.tiles;  // per drafted position: 1 accepted, 0 rejected, 2 undecided
     // Acceptance of every drafted token, in parallel: q(x) and p(x) from the
     // rows' nucleus states; a token tied at a boundary of which only some
     // ties are kept needs its rank among them (a pass over the row, below).
@@ -1080,10 +1083,11 @@ __global__ void __launch_bounds__(kSampleWarps * 32) spec_sample_kernel(const Sp
       const RowNucleus nq = load_state(p.state_d + pos_d * kSpecStateWords);
       for (int t = threadIdx.x; t < p.tiles; t += kSampleWarps * 32) fq[t] = p.f_d[pos_d * p.tiles + t];
       __syncthreads();
-      next = sample(ev, fp, np, p.ed + pos_d * p.ldz, fq, nq, true, p.V, u, cum, tp, tq, sh, p.status);
+      next = sample(ev, fp, np, p.ed + pos_d * p.ldz, fq, nq, true, p.V, u, cum, tp, tq, live, sh,
+                    p.status);
     }
     __syncthreads();
-    if (next < 0) next = sample(ev, fp, np, ev, fp, np, false, p.V, u, cum, tp, tq, sh, p.status);
+    if (next < 0) next = sample(ev, fp, np, ev, fp, np, false, p.V, u, cum, tp, tq, live, sh, p.status);
     if (next < 0) next = static_cast<int>(p.V - 1);  // unreachable: the maximum has e = 1
   }
   if (threadIdx.x == 0) {
@@ -1094,7 +1098,7 @@ __global__ void __launch_bounds__(kSampleWarps * 32) spec_sample_kernel(const Sp
 
 size_t sample_smem(long long V, int tiles, int gamma) {
   const long long nsteps = (V + kStep - 1) / kStep;
-  return sizeof(float) * (2 * static_cast<size_t>(tiles) + 3 * static_cast<size_t>(nsteps) +
+  return sizeof(float) * (3 * static_cast<size_t>(tiles) + 3 * static_cast<size_t>(nsteps) +
                           static_cast<size_t>(gamma));
 }
 
