@@ -87,7 +87,7 @@ size_t mls_workspace_size(const mls_problem* p);
 
 /*
  * Forward (Eq. 2, Eq. 3, weighted sum over sub-models).
- *   H[m]      device, [T, d_m] in_dtype      hidden states of sub-model m
+ *   H[m]      device, [T, d_m] in_dtype      hidden states of sub-model m (may be NULL when T = 0)
  *   W[m]      device, [V, d_m] in_dtype      LM head of sub-model m
  *   targets   device, int32 [T]; < 0 = ignored token
  *   loss      device, fp32 [1]               the scalar objective
@@ -107,7 +107,8 @@ int mls_head_loss_fwd(const mls_problem* p, const void* const* H, const void* co
  * Backward: gradients of grad_scale * loss.
  *   stats     device, fp32 [2, M, T] as written by mls_head_loss_fwd for the same inputs
  *   dH[m]     device, fp32 [T, d_m]    overwritten with d(loss)/dH_m
- *   dW[m]     device, fp32 [V, d_m]    overwritten with d(loss)/dW_m
+ *   dW[m]     device, fp32 [V, d_m]    overwritten with d(loss)/dW_m (zeros when T = 0
+ *                                      or no token counts; H[m], dH[m] may be NULL when T = 0)
  * The teacher's parameters get only the gradient of w_t * mean CE_t: Eq. 2 stops
  * the gradient through q.  The logits are recomputed, never read from memory.
  */

@@ -355,7 +355,7 @@ extern "C" int mls_head_loss_fwd(const mls_problem* p, const void* const* H, con
   if (rc) return rc;
   if (!H || !W || !loss || (p->T > 0 && (!targets || !tok_loss || !stats))) return MLS_ERR_ARG;
   for (int m = 0; m < p->M; ++m) {
-    if (!H[m] || !W[m]) return MLS_ERR_ARG;
+    if ((p->T > 0 && !H[m]) || !W[m]) return MLS_ERR_ARG;  // no rows to read when T = 0
     if (!aligned16(H[m]) || !aligned16(W[m])) return MLS_ERR_ALIGN;
   }
   DeviceState* dev = nullptr;
@@ -430,7 +430,7 @@ extern "C" int mls_head_loss_bwd(const mls_problem* p, const void* const* H, con
   if (!H || !W || !dH || !dW || (p->T > 0 && (!targets || !stats))) return MLS_ERR_ARG;
   if (!std::isfinite(grad_scale)) return MLS_ERR_ARG;
   for (int m = 0; m < p->M; ++m) {
-    if (!H[m] || !W[m] || !dW[m] || (p->T > 0 && !dH[m])) return MLS_ERR_ARG;
+    if ((p->T > 0 && (!H[m] || !dH[m])) || !W[m] || !dW[m]) return MLS_ERR_ARG;
     if (!aligned16(H[m]) || !aligned16(W[m]) || !aligned16(dW[m]) || !aligned16(dH[m]))
       return MLS_ERR_ALIGN;
   }
@@ -700,7 +700,7 @@ extern "C" int mls_head_loss_fwd_noalloc(const mls_problem* p, const void* const
   if (rc) return rc;
   if (!H || !W || !loss || (p->T > 0 && (!targets || !tok_loss || !stats))) return MLS_ERR_ARG;
   for (int m = 0; m < p->M; ++m) {
-    if (!H[m] || !W[m]) return MLS_ERR_ARG;
+    if ((p->T > 0 && !H[m]) || !W[m]) return MLS_ERR_ARG;  // no rows to read when T = 0
     if (!aligned16(H[m]) || !aligned16(W[m])) return MLS_ERR_ALIGN;
   }
   DeviceState* dev = nullptr;
@@ -761,7 +761,7 @@ extern "C" int mls_head_pairwise(const mls_problem* p, const void* const* H, con
   if (rc) return rc;
   if (!H || !W || !pair_stats || (p->T > 0 && !tok_kl)) return MLS_ERR_ARG;
   for (int m = 0; m < p->M; ++m) {
-    if (!H[m] || !W[m]) return MLS_ERR_ARG;
+    if ((p->T > 0 && !H[m]) || !W[m]) return MLS_ERR_ARG;  // no rows to read when T = 0
     if (!aligned16(H[m]) || !aligned16(W[m])) return MLS_ERR_ALIGN;
   }
   DeviceState* dev = nullptr;

@@ -195,3 +195,32 @@ def _full_size(name, nsample, seed=21):
 @pytest.mark.parametrize("name", ["suite3", "suite3_big", "suite4", "stress", "suite3_paper"])
 def test_full_size_sampled(name):
     _full_size(name, nsample=10)
+
+
+def test_empty_token_batch():
+    """T = 0 (null hidden states are allowed then): the loss is 0, dW is
+    overwritten with zeros, the pairwise means are 0 and the junction does
+    nothing; nothing raises a status bit."""
+    dev = torch.device("cuda")
+    B.mls_get_status()  # clear bits an earlier test may have left
+    d, V = (64, 128), 300
+    op = B.HeadLoss(d, 0, V, device=dev)
+    H = [torch.empty(0, dm, dtype=torch.bfloat16, device=dev) for dm in d]
+    W = [torch.randn(V, dm, device=dev).to(torch.bfloat16) for dm in d]
+    y = torch.empty(0, dtype=torch.int32, device=dev)
+    op.loss.fill_(float("nan"))
+    for t in op.dW:
+        t.fill_(float("nan"))
+    op.forward(H, W, y)
+    op.backward(H, W, y)
+    _, _, ps = op.pairwise(H, W)
+    o = torch.empty(0, 64, dtype=torch.bfloat16, device=dev)
+    e = torch.empty(0, 64, dtype=torch.bfloat16, device=dev)
+    x = torch.empty(0, 128, dtype=torch.bfloat16, device=dev)
+    B.mls_junction_fwd(o, e, x)
+    B.mls_junction_bwd(o, e, x, torch.empty_like(o), torch.empty_like(e))
+    torch.cuda.synchronize()
+    assert op.loss.item() == 0.0
+    assert all(bool((t == 0).all()) for t in op.dW)
+    assert bool((ps == 0).all())
+    assert B.mls_get_status() == 0
