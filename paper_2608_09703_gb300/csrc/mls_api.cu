@@ -1008,7 +1008,7 @@ extern "C" int mls_spec_verify(const mls_spec_problem* p, const void* H_draft, c
   g.total_tiles = tiles;
   g.status = dev->status;
   const int grid = 2 * (tiles < dev->gemm_pairs ? tiles : dev->gemm_pairs);
-  if ((rc = timed("spec_logits", s, [&] { return launch_gemm_kk(g, tf32, grid, s); }))) return rc;
+  if ((rc = timed("spec_logits", s, [&] { return launch_gemm_stats(g, tf32, grid, s); }))) return rc;
   if (!p->greedy && (rc = timed("spec_rows", s, [&] { return launch_spec_rows(sp, s); })))
     return rc;
   return timed("spec_sample", s, [&] { return launch_spec_sample(sp, s); });

@@ -331,6 +331,10 @@ __device__ __noinline__ void epilogue_stats(const GemmProblem& pr, const CUtenso
   }
 }
 
+// kStats: the launch may hold problems with a statistics epilogue (only the
+// verify step's logits GEMM); without it epilogue_stats is not in the kernel,
+// which keeps the training GEMMs at 64 registers instead of 119.
+template <bool kStats>
 __device__ __forceinline__ void gemm_epilogue(const GemmParams& p, uint32_t base, uint32_t tmem,
                                               uint32_t rank, int warp, int lane,
                                               volatile int* abort_flag) {
@@ -348,7 +352,7 @@ __device__ __forceinline__ void gemm_epilogue(const GemmParams& p, uint32_t base
     const long long row = static_cast<long long>(tc.tm) * kPairM + rank * kGemmBM + warp * 32 + lane;
     const bool row_ok = row < pr.Mrows;
     float v[32];
-    if (pr.epi != kEpiPlain) {
+    if (kStats && pr.epi != kEpiPlain) {
       const int row0 = tc.tm * kPairM + static_cast<int>(rank) * kGemmBM + warp * 32;
       epilogue_stats(pr, &p.mapC[tc.prob], stage, stores, tl + acc * kGemmBN, tc.tn, row, row_ok,
                      row0, lane);
@@ -391,7 +395,7 @@ __device__ __forceinline__ void gemm_epilogue(const GemmParams& p, uint32_t base
   if (stores && lane == 0) bulk_wait_all();  // staging must outlive the stores reading it
 }
 
-template <bool kTF32, int kAMode, bool kBMN>
+template <bool kTF32, int kAMode, bool kBMN, bool kStats>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     gemm_kernel(const __grid_constant__ GemmParams p) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -437,7 +441,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     if (lane == 0 && rank == 0) gemm_mma<kTF32, kAMode, kBMN>(p, base, tmem, abort_flag);
     __syncwarp();
   } else {
-    gemm_epilogue(p, base, tmem, rank, warp, lane, abort_flag);
+    gemm_epilogue<kStats>(p, base, tmem, rank, warp, lane, abort_flag);
   }
 
   tc_fence_before();
@@ -448,30 +452,27 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
   }
 }
 
-template <int kAMode, bool kBMN>
+template <int kAMode, bool kBMN, bool kStats>
 cudaError_t launch(const GemmParams& p, bool tf32, int grid, cudaStream_t s) {
   if (p.total_tiles <= 0 || grid <= 0) return cudaSuccess;
   if (tf32)
-    gemm_kernel<true, kAMode, kBMN><<<grid, kGemmThreads, kGemmSmem, s>>>(p);
+    gemm_kernel<true, kAMode, kBMN, kStats><<<grid, kGemmThreads, kGemmSmem, s>>>(p);
   else
-    gemm_kernel<false, kAMode, kBMN><<<grid, kGemmThreads, kGemmSmem, s>>>(p);
+    gemm_kernel<false, kAMode, kBMN, kStats><<<grid, kGemmThreads, kGemmSmem, s>>>(p);
   return cudaGetLastError();
 }
 
 }  // namespace
 
-cudaError_t launch_gemm_dw(const GemmParams& p, bool tf32, int grid, cudaStream_t s) {
-  return launch<1, true>(p, tf32, grid, s);
-}
-cudaError_t launch_gemm_dh(const GemmParams& p, bool tf32, int grid, cudaStream_t s) {
-  return launch<0, true>(p, tf32, grid, s);
-}
 cudaError_t launch_gemm_kk(const GemmParams& p, bool tf32, int grid, cudaStream_t s) {
-  return launch<0, false>(p, tf32, grid, s);
+  return launch<0, false, false>(p, tf32, grid, s);
+}
+cudaError_t launch_gemm_stats(const GemmParams& p, bool tf32, int grid, cudaStream_t s) {
+  return launch<0, false, true>(p, tf32, grid, s);
 }
 cudaError_t launch_gemm_mixed(const GemmParams& p, int grid, cudaStream_t s) {
   if (p.total_tiles <= 0 || grid <= 0) return cudaSuccess;
-  gemm_kernel<false, 2, true><<<grid, kGemmThreads, kGemmSmem, s>>>(p);
+  gemm_kernel<false, 2, true, false><<<grid, kGemmThreads, kGemmSmem, s>>>(p);
   return cudaGetLastError();
 }
 
@@ -483,7 +484,7 @@ int gemm_max_active_pairs() {
   cfg.blockDim = dim3(kGemmThreads);
   cfg.dynamicSmemBytes = kGemmSmem;
   int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, gemm_kernel<false, 1, true>, &cfg) != cudaSuccess) {
+  if (cudaOccupancyMaxActiveClusters(&n, gemm_kernel<false, 2, true, false>, &cfg) != cudaSuccess) {
     cudaGetLastError();
     return 0;
   }
@@ -492,23 +493,21 @@ int gemm_max_active_pairs() {
 
 cudaError_t setup_gemm_kernels() {
   cudaError_t e;
-#define MLS_SET(TF, AM, BM)                                                                     \
-  e = cudaFuncSetAttribute(gemm_kernel<TF, AM, BM>, cudaFuncAttributeMaxDynamicSharedMemorySize, \
-                           kGemmSmem);                                                          \
+#define MLS_SET(TF, AM, BM, ST)                                                                 \
+  e = cudaFuncSetAttribute(gemm_kernel<TF, AM, BM, ST>,                                         \
+                           cudaFuncAttributeMaxDynamicSharedMemorySize, kGemmSmem);             \
   if (e != cudaSuccess) return e;                                                               \
   {                                                                                             \
     cudaFuncAttributes fa;                                                                      \
-    e = cudaFuncGetAttributes(&fa, gemm_kernel<TF, AM, BM>);                                    \
+    e = cudaFuncGetAttributes(&fa, gemm_kernel<TF, AM, BM, ST>);                                \
     if (e != cudaSuccess) return e;                                                             \
     if (fa.maxThreadsPerBlock < kGemmThreads) return cudaErrorLaunchOutOfResources;             \
   }
-  MLS_SET(true, 1, true)
-  MLS_SET(false, 1, true)
-  MLS_SET(true, 0, true)
-  MLS_SET(false, 0, true)
-  MLS_SET(true, 0, false)
-  MLS_SET(false, 0, false)
-  MLS_SET(false, 2, true)
+  MLS_SET(true, 0, false, false)
+  MLS_SET(false, 0, false, false)
+  MLS_SET(true, 0, false, true)
+  MLS_SET(false, 0, false, true)
+  MLS_SET(false, 2, true, false)
 #undef MLS_SET
   return cudaSuccess;
 }

@@ -257,12 +257,13 @@ constexpr int kEvalMergeTokens = 128;  // tokens per evaluation-merge block: one
 // Launchers (return the cudaError_t of the launch).
 cudaError_t launch_head_fwd(const HeadParams& p, bool tf32, bool tau_one, cudaStream_t s);
 cudaError_t launch_head_bwd(const HeadParams& p, bool tf32, bool tau_one, cudaStream_t s);
-cudaError_t launch_gemm_dw(const GemmParams& p, bool tf32, int grid, cudaStream_t s);
-cudaError_t launch_gemm_dh(const GemmParams& p, bool tf32, int grid, cudaStream_t s);
 // bf16, B MN-major, A's layout per problem (GemmProblem::a_mn): dW and dH in one launch.
 cudaError_t launch_gemm_mixed(const GemmParams& p, int grid, cudaStream_t s);
-// Both operands K-major (tf32 path: fp32 inputs with transposed copies).
+// Both operands K-major (tf32 path: fp32 inputs with transposed copies);
+// plain epilogues only.
 cudaError_t launch_gemm_kk(const GemmParams& p, bool tf32, int grid, cudaStream_t s);
+// Both operands K-major, with the statistics epilogues (GemmProblem::epi).
+cudaError_t launch_gemm_stats(const GemmParams& p, bool tf32, int grid, cudaStream_t s);
 cudaError_t launch_transpose(const float* in, long long rows, long long cols, long long ld_in,
                              float* out, long long ld_out, cudaStream_t s);
 cudaError_t launch_merge(const MergeParams& p, int blocks, cudaStream_t s);
