@@ -77,6 +77,17 @@ def test_alpha_zero_and_one():
         full_parity(wl, H, W, y)
 
 
+@pytest.mark.parametrize("alpha,tau", [(0.3, 1.0), (0.7, 1.0), (0.5, 0.1), (0.5, 10.0)])
+def test_paper_alphas_and_extreme_temperatures(alpha, tau):
+    """The paper's alpha sweep values besides 0, 0.5 and 1, and temperatures far
+    from 1 (a nearly one-hot q at 0.1, a nearly uniform one at 10), with the
+    normalised per-size weights of App. G (1/3 each) and a 3-level suite."""
+    wl = synth.Workload("alpha_tau", T=70, d=(64, 128, 192), V=900, alpha=alpha, tau=tau,
+                        w_sigma=0.1, weights=(1 / 3, 1 / 3, 1 / 3))
+    H, W, y = synth.make_inputs(wl, seed=6)
+    full_parity(wl, H, W, y)
+
+
 def test_all_targets_ignored():
     wl = synth.Workload("ign", T=96, d=(64, 64), V=300, w_sigma=0.05)
     H, W, y = synth.make_inputs(wl, seed=6)

@@ -245,6 +245,16 @@ def test_spec_top_p_one_and_gamma_zero():
     assert (n == 0).all()
 
 
+@pytest.mark.parametrize("temperature,top_p", [(1.0, 0.5), (0.7, 0.95), (0.2, 0.99)])
+def test_spec_other_temperatures_and_nucleus_sizes(temperature, top_p):
+    """Temperatures and nucleus sizes other than the paper's 0.4 / 0.9: a
+    small nucleus of a softer distribution, a wide one, and a sharp one."""
+    wl = synth.SpecWorkload("tp", B=24, gamma=4, V=1500, d_draft=64, d_verify=128,
+                            temperature=temperature, top_p=top_p)
+    # a wide nucleus of a soft distribution has more tokens near its cut
+    check(wl, *inputs(wl, 60 + int(100 * temperature)), min_checked=0.6)
+
+
 def test_spec_identical_models_accept_every_draft():
     """Draft == verifier: p == q exactly on both sides, so every drafted token
     inside the nucleus is accepted and the bonus token is sampled from p."""
