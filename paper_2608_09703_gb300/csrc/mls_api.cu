@@ -70,6 +70,8 @@ int device_state(DeviceState** out) {
       s.err = fail(MLS_ERR_CUDA, "eval kernel attributes", e);
     } else if ((e = setup_spec_kernels()) != cudaSuccess) {
       s.err = fail(MLS_ERR_CUDA, "spec kernel attributes", e);
+    } else if ((e = setup_junction_kernels()) != cudaSuccess) {
+      s.err = fail(MLS_ERR_CUDA, "junction kernel attributes", e);
     } else if ((s.gemm_pairs = gemm_max_active_pairs()) <= 0) {
       s.err = fail(MLS_ERR_CUDA, "gemm cluster occupancy");
     } else if ((s.head_pairs = head_max_active_pairs()) <= 0) {
@@ -846,7 +848,8 @@ extern "C" int mls_junction_fwd(int64_t T, int32_t d_prev, int32_t d_next, int32
   if (rc) return rc;
   DeviceState* dev = nullptr;
   if ((rc = device_state(&dev))) return rc;
-  JunctionParams jp{T, d_prev, d_next, embed_first ? 1 : 0, o, e, x, nullptr, nullptr, nullptr};
+  JunctionParams jp{T, d_prev, d_next, embed_first ? 1 : 0, o, e, x, nullptr, nullptr, nullptr,
+                    dev->status, dev->sms};
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   return timed("junction_fwd", s, [&] { return launch_junction_fwd(jp, in_dtype == MLS_FP32, s); });
 }
@@ -859,7 +862,8 @@ extern "C" int mls_junction_bwd(int64_t T, int32_t d_prev, int32_t d_next, int32
   if (rc) return rc;
   DeviceState* dev = nullptr;
   if ((rc = device_state(&dev))) return rc;
-  JunctionParams jp{T, d_prev, d_next, embed_first ? 1 : 0, o, e, nullptr, g, d_o, d_e};
+  JunctionParams jp{T, d_prev, d_next, embed_first ? 1 : 0, o, e, nullptr, g, d_o, d_e, dev->status,
+                    dev->sms};
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   return timed("junction_bwd", s, [&] { return launch_junction_bwd(jp, in_dtype == MLS_FP32, s); });
 }

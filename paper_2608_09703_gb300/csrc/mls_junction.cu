@@ -6,14 +6,17 @@
 //   dL/do = s (g_o - o (g_o . o) / ||o||^2)
 //   dL/de = g_e + s (g_o . o) e / ||e||^2
 // Both are row reductions followed by an elementwise pass, bound by HBM.  One
-// warp owns a token.  It issues every 16-byte load of its row at once (o and
-// e, and g in the backward), keeps them packed in registers for the
-// elementwise pass, and so reads each input byte from HBM once with many loads
-// in flight: one row costs one memory latency.  A row segment (o, or e) needs
-// ceil(length / (32 * elements per 16 bytes)) vectors per lane; the kernels
-// are instantiated for 1, 2, 4, 8 and 12, and wider rows take a streaming
-// path that reads the row twice (the second time from L2).  Sums are fp32,
-// accumulated per lane in column order, then across the warp, in both paths.
+// warp owns a token, and each input byte is read from HBM once.  Three paths:
+//   - register cache (rows whose segments need at most 8 vectors of 16 bytes
+//     per lane): the warp issues every load of its row at once (o and e, and g
+//     in the backward) and keeps them packed in registers, so a row costs one
+//     memory latency;
+//   - TMA ring (wider rows): persistent warps fetch whole rows into shared
+//     memory with 1-D bulk copies, several rows ahead;
+//   - streaming (rows too wide for two ring buffers): the row is read twice,
+//     the second time from L2.
+// Sums are fp32, accumulated per lane in column order, then across the warp,
+// in every path, so all three give identical results.
 #include "mls_device.cuh"
 #include "mls_kernels.h"
 
@@ -281,15 +284,202 @@ __global__ void __launch_bounds__(32 * kRowsPerBlock) junction_bwd_kernel(const 
   }
 }
 
+// ---------------------------------------------------------------- TMA ring
+// The main path.  Persistent CTAs of `warps` warps; each warp owns a ring of
+// `stages` row buffers in shared memory and the rows gw, gw + GW, ... (gw its
+// global warp index, GW the warps of the grid).  Its lane 0 fetches whole rows
+// (o and e, and g in the backward) with 1-D bulk copies that complete on the
+// buffer's mbarrier, `stages` rows ahead, so every SM keeps tens of rows
+// of HBM reads in flight whatever T is.  The warp computes a row from shared
+// memory, in the same lane and column order as the kernels above, and stores
+// its outputs with coalesced 16-byte stores.
+constexpr int kRingWarps = 4;
+constexpr int kRingStages = 4;
+constexpr uint32_t kRingSmem = 220 * 1024;  // dynamic shared memory a CTA may use
+constexpr uint64_t kDrainNs = 100000000ull;
+
+template <typename E>
+__device__ __forceinline__ uint4 ld16s(const E* p) { return *reinterpret_cast<const uint4*>(p); }
+
+template <typename E, bool kBwd>
+__global__ void __launch_bounds__(32 * kRingWarps)
+    junction_ring_kernel(const JunctionParams p, int stages, uint32_t stage_bytes) {
+  constexpr int N = Vec<E>::N;
+  extern __shared__ __align__(128) uint8_t ring_smem[];
+  __shared__ __align__(8) uint64_t bars[kRingWarps * kRingStages];
+  __shared__ int abort_flag;
+  const int nw = static_cast<int>(blockDim.x >> 5), w = static_cast<int>(threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  const long long GW = static_cast<long long>(gridDim.x) * nw;
+  const long long gw = static_cast<long long>(blockIdx.x) * nw + w;
+  const int de = p.d_next - p.d_prev;
+  const uint32_t ob = p.d_prev * sizeof(E), eb = de * sizeof(E);
+  const uint32_t gb = kBwd ? p.d_next * sizeof(E) : 0u;
+  uint8_t* ring = ring_smem + static_cast<size_t>(w) * stages * stage_bytes;
+  const uint32_t ring_s = smem_u32(ring), bar0 = smem_u32(&bars[w * kRingStages]);
+  if (threadIdx.x == 0) abort_flag = 0;
+  if (lane == 0)
+    for (int st = 0; st < stages; ++st) mbar_init(bar0 + 8u * st, 1);
+  fence_barrier_init();
+  __syncthreads();
+  const E* o = static_cast<const E*>(p.o);
+  const E* e = static_cast<const E*>(p.e);
+  const E* g = static_cast<const E*>(p.g);
+  auto fetch = [&](long long r, int st) {
+    const uint32_t dst = ring_s + static_cast<uint32_t>(st) * stage_bytes, bar = bar0 + 8u * st;
+    mbar_arrive_expect_tx(bar, ob + eb + gb);
+    bulk_load_1d(dst, o + r * p.d_prev, ob, bar);
+    bulk_load_1d(dst + ob, e + r * de, eb, bar);
+    if (kBwd) bulk_load_1d(dst + ob + eb, g + r * p.d_next, gb, bar);
+  };
+  if (lane == 0)
+    for (int st = 0; st < stages; ++st)
+      if (gw + st * GW < p.T) fetch(gw + st * GW, st);
+  long long i = 0;
+  bool ok = true;
+  for (long long r = gw; r < p.T; r += GW, ++i) {
+    const int st = static_cast<int>(i % stages);
+    if (!mbar_wait(bar0 + 8u * st, static_cast<uint32_t>((i / stages) & 1), &abort_flag, p.status)) {
+      ok = false;
+      break;
+    }
+    const E* os = reinterpret_cast<const E*>(ring + static_cast<size_t>(st) * stage_bytes);
+    const E* es = os + p.d_prev;
+    if constexpr (!kBwd) {
+      float so = 0.f, se = 0.f;
+      for (int k = lane * N; k < p.d_prev; k += 32 * N) {
+        float f[N];
+        Vec<E>::unpack(ld16s(os + k), f);
+#pragma unroll
+        for (int q = 0; q < N; ++q) so = fmaf(f[q], f[q], so);
+      }
+      for (int k = lane * N; k < de; k += 32 * N) {
+        float f[N];
+        Vec<E>::unpack(ld16s(es + k), f);
+#pragma unroll
+        for (int q = 0; q < N; ++q) se = fmaf(f[q], f[q], se);
+      }
+      const float no = sqrtf(warp_sum(so)), ne = sqrtf(warp_sum(se));
+      const float sc = no > 0.f ? ne / no : 0.f;
+      E* x = static_cast<E*>(p.x) + r * p.d_next;
+      E* xo = x + (p.embed_first ? de : 0);
+      E* xe = x + (p.embed_first ? 0 : p.d_prev);
+      for (int k = lane * N; k < p.d_prev; k += 32 * N) {
+        float f[N];
+        Vec<E>::unpack(ld16s(os + k), f);
+#pragma unroll
+        for (int q = 0; q < N; ++q) f[q] *= sc;
+        st16(xo + k, Vec<E>::pack(f));
+      }
+      for (int k = lane * N; k < de; k += 32 * N) st16(xe + k, ld16s(es + k));
+    } else {
+      const E* gs = es + de;
+      const E* gos = gs + (p.embed_first ? de : 0);
+      const E* ges = gs + (p.embed_first ? 0 : p.d_prev);
+      float oo = 0.f, dot = 0.f, ee = 0.f;
+      for (int k = lane * N; k < p.d_prev; k += 32 * N) {
+        float fo[N], fg[N];
+        Vec<E>::unpack(ld16s(os + k), fo);
+        Vec<E>::unpack(ld16s(gos + k), fg);
+#pragma unroll
+        for (int q = 0; q < N; ++q) {
+          oo = fmaf(fo[q], fo[q], oo);
+          dot = fmaf(fg[q], fo[q], dot);
+        }
+      }
+      for (int k = lane * N; k < de; k += 32 * N) {
+        float f[N];
+        Vec<E>::unpack(ld16s(es + k), f);
+#pragma unroll
+        for (int q = 0; q < N; ++q) ee = fmaf(f[q], f[q], ee);
+      }
+      oo = warp_sum(oo);
+      dot = warp_sum(dot);
+      ee = warp_sum(ee);
+      const float no = sqrtf(oo), ne = sqrtf(ee);
+      const float sc = no > 0.f ? ne / no : 0.f;
+      const float co = no > 0.f ? dot / oo : 0.f;                     // (g_o . o) / ||o||^2
+      const float ce = (no > 0.f && ee > 0.f) ? sc * dot / ee : 0.f;  // s (g_o . o) / ||e||^2
+      E* d_o = static_cast<E*>(p.d_o) + r * p.d_prev;
+      E* d_e = static_cast<E*>(p.d_e) + r * de;
+      for (int k = lane * N; k < p.d_prev; k += 32 * N) {
+        float fo[N], fg[N], y[N];
+        Vec<E>::unpack(ld16s(os + k), fo);
+        Vec<E>::unpack(ld16s(gos + k), fg);
+#pragma unroll
+        for (int q = 0; q < N; ++q) y[q] = sc * fmaf(-fo[q], co, fg[q]);
+        st16(d_o + k, Vec<E>::pack(y));
+      }
+      for (int k = lane * N; k < de; k += 32 * N) {
+        float fe[N], fg[N], y[N];
+        Vec<E>::unpack(ld16s(es + k), fe);
+        Vec<E>::unpack(ld16s(ges + k), fg);
+#pragma unroll
+        for (int q = 0; q < N; ++q) y[q] = fmaf(ce, fe[q], fg[q]);
+        st16(d_e + k, Vec<E>::pack(y));
+      }
+    }
+    // Every lane's reads of this buffer precede the copy that refills it.
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0 && r + stages * GW < p.T) fetch(r + stages * GW, st);
+  }
+  if (!ok && lane == 0) {
+    // The copies already issued (iterations i .. i + stages - 1) must land
+    // before this CTA's shared memory goes away.
+    for (long long k = i; k < i + stages; ++k)
+      if (gw + k * GW < p.T)
+        mbar_wait_drain(bar0 + 8u * static_cast<uint32_t>(k % stages),
+                        static_cast<uint32_t>((k / stages) & 1), kDrainNs);
+  }
+}
+
+// Ring shape for a row of `row_bytes`: 4 warps per CTA with 2 to 4 buffers
+// each, two CTAs per SM when they fit, else one.  Returns false for rows too
+// wide for that (over 27.5 KB), which stream instead: fewer than four warps
+// per SM cannot keep HBM busy.  (Eight warps per CTA measured no faster.)
+bool ring_shape(uint32_t row_bytes, int& warps, int& stages) {
+  for (const int ctas : {2, 1}) {
+    const long long st = kRingSmem / (static_cast<long long>(ctas) * kRingWarps * row_bytes);
+    if (st >= 2) {
+      warps = kRingWarps;
+      stages = st > kRingStages ? kRingStages : static_cast<int>(st);
+      return true;
+    }
+  }
+  return false;
+}
+
+template <typename E, bool kBwd>
+cudaError_t ring_launch(const JunctionParams& p, cudaStream_t s, bool& launched) {
+  launched = false;
+  const uint32_t elt = sizeof(E);
+  const uint32_t row = (static_cast<uint32_t>(p.d_next) + (kBwd ? p.d_next : 0)) * elt;
+  int warps = 0, stages = 0;
+  if (!ring_shape(row, warps, stages)) return cudaSuccess;
+  const size_t smem = static_cast<size_t>(warps) * stages * row;
+  int per_sm = 0;
+  cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+      &per_sm, junction_ring_kernel<E, kBwd>, 32 * warps, smem);
+  if (e != cudaSuccess) return e;
+  if (per_sm < 1) return cudaSuccess;
+  const long long need = (p.T + warps - 1) / warps;
+  const long long most = static_cast<long long>(p.sms > 0 ? p.sms : 1) * per_sm;
+  const unsigned blocks = static_cast<unsigned>(need < most ? need : most);
+  junction_ring_kernel<E, kBwd><<<blocks, 32 * warps, smem, s>>>(p, stages, row);
+  launched = true;
+  return cudaGetLastError();
+}
+
 // Cached vectors per lane for a row whose segments are d_prev and d_next -
-// d_prev elements of `elt` bytes: the smallest of 1, 2, 4, 8, 12 that holds both,
-// or 0 (streaming) when a segment needs more than 12 (the backward then holds
-// 48 vectors, 192 registers, per lane).
+// d_prev elements of `elt` bytes: the smallest of 1, 2, 4, 8 that holds both,
+// or 0 when a segment needs more.  At 12 vectors the backward needed 254
+// registers and ran ~10% slower than the TMA ring.
 int cache_vectors(int d_prev, int d_next, int elt) {
   const int per = 32 * (16 / elt);  // elements per cached vector across the warp
   const int need_o = (d_prev + per - 1) / per, need_e = (d_next - d_prev + per - 1) / per;
   const int need = need_o > need_e ? need_o : need_e;
-  for (const int r : {1, 2, 4, 8, 12})
+  for (const int r : {1, 2, 4, 8})
     if (need <= r) return r;
   return 0;
 }
@@ -302,7 +492,6 @@ cudaError_t fwd_launch(const JunctionParams& p, int r, unsigned blocks, cudaStre
     case 2: junction_fwd_kernel<E, 2><<<blocks, b, 0, s>>>(p); break;
     case 4: junction_fwd_kernel<E, 4><<<blocks, b, 0, s>>>(p); break;
     case 8: junction_fwd_kernel<E, 8><<<blocks, b, 0, s>>>(p); break;
-    case 12: junction_fwd_kernel<E, 12><<<blocks, b, 0, s>>>(p); break;
     default: junction_fwd_kernel<E, 0><<<blocks, b, 0, s>>>(p); break;
   }
   return cudaGetLastError();
@@ -316,7 +505,6 @@ cudaError_t bwd_launch(const JunctionParams& p, int r, unsigned blocks, cudaStre
     case 2: junction_bwd_kernel<E, 2><<<blocks, b, 0, s>>>(p); break;
     case 4: junction_bwd_kernel<E, 4><<<blocks, b, 0, s>>>(p); break;
     case 8: junction_bwd_kernel<E, 8><<<blocks, b, 0, s>>>(p); break;
-    case 12: junction_bwd_kernel<E, 12><<<blocks, b, 0, s>>>(p); break;
     default: junction_bwd_kernel<E, 0><<<blocks, b, 0, s>>>(p); break;
   }
   return cudaGetLastError();
@@ -324,10 +512,18 @@ cudaError_t bwd_launch(const JunctionParams& p, int r, unsigned blocks, cudaStre
 
 }  // namespace
 
+// Register cache when a row fits 8 vectors per lane, else the TMA ring, else
+// (rows too wide for two ring buffers) the streaming kernel.
 cudaError_t launch_junction_fwd(const JunctionParams& p, bool fp32, cudaStream_t s) {
   const long long blocks = (p.T + kRowsPerBlock - 1) / kRowsPerBlock;
   if (blocks <= 0) return cudaSuccess;
   const int r = cache_vectors(p.d_prev, p.d_next, fp32 ? 4 : 2);
+  if (r == 0) {
+    bool launched = false;
+    const cudaError_t e = fp32 ? ring_launch<float, false>(p, s, launched)
+                               : ring_launch<__nv_bfloat16, false>(p, s, launched);
+    if (e != cudaSuccess || launched) return e;
+  }
   return fp32 ? fwd_launch<float>(p, r, static_cast<unsigned>(blocks), s)
               : fwd_launch<__nv_bfloat16>(p, r, static_cast<unsigned>(blocks), s);
 }
@@ -336,8 +532,28 @@ cudaError_t launch_junction_bwd(const JunctionParams& p, bool fp32, cudaStream_t
   const long long blocks = (p.T + kRowsPerBlock - 1) / kRowsPerBlock;
   if (blocks <= 0) return cudaSuccess;
   const int r = cache_vectors(p.d_prev, p.d_next, fp32 ? 4 : 2);
+  if (r == 0) {
+    bool launched = false;
+    const cudaError_t e = fp32 ? ring_launch<float, true>(p, s, launched)
+                               : ring_launch<__nv_bfloat16, true>(p, s, launched);
+    if (e != cudaSuccess || launched) return e;
+  }
   return fp32 ? bwd_launch<float>(p, r, static_cast<unsigned>(blocks), s)
               : bwd_launch<__nv_bfloat16>(p, r, static_cast<unsigned>(blocks), s);
+}
+
+cudaError_t setup_junction_kernels() {
+  cudaError_t e;
+#define MLS_SET(E, B)                                                                        \
+  e = cudaFuncSetAttribute(junction_ring_kernel<E, B>,                                       \
+                           cudaFuncAttributeMaxDynamicSharedMemorySize, kRingSmem);          \
+  if (e != cudaSuccess) return e;
+  MLS_SET(float, false)
+  MLS_SET(float, true)
+  MLS_SET(__nv_bfloat16, false)
+  MLS_SET(__nv_bfloat16, true)
+#undef MLS_SET
+  return cudaSuccess;
 }
 
 }  // namespace mls

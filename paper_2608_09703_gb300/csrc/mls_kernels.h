@@ -193,9 +193,12 @@ struct JunctionParams {
   const void* g;                 // [T, D_{m+1}] (backward)
   void* d_o;                     // [T, D_m] (backward)
   void* d_e;                     // [T, D_{m+1} - D_m] (backward)
+  int* status;                   // device status word (pipeline-wait timeouts)
+  int sms;                       // SMs of the device
 };
 cudaError_t launch_junction_fwd(const JunctionParams& p, bool fp32, cudaStream_t s);
 cudaError_t launch_junction_bwd(const JunctionParams& p, bool fp32, cudaStream_t s);
+cudaError_t setup_junction_kernels();
 
 // ------------------------------------------------------------------ speculative verify
 // Per position of a sequence: the verifier's logits row (and the draft's for

@@ -68,18 +68,20 @@ def test_junction_suite3_shapes_full_size(dp, dn):
 
 
 # Each register-cache size of the kernels (16-byte vectors per lane per row
-# segment: 1, 2, 4, 8, 12) and the streaming path for wider segments, with
-# segments that end part-way through a vector round and a ragged last block.
+# segment: 1, 2, 4, 8), the TMA ring for wider rows and the streaming path for
+# rows too wide for two ring buffers, with segments that end part-way through
+# a vector round and a ragged last block.
 @pytest.mark.parametrize("dtype,dp,de", [
     (torch.bfloat16, 72, 40),      # 1 vector
     (torch.bfloat16, 264, 8),      # 2
     (torch.bfloat16, 520, 1000),   # 4
     (torch.bfloat16, 1800, 200),   # 8
-    (torch.bfloat16, 3072, 1024),  # 12
-    (torch.bfloat16, 3080, 16),    # o past 12: streaming
-    (torch.bfloat16, 64, 4096),    # e past 12: streaming
-    (torch.float32, 1536, 512),    # 12
-    (torch.float32, 1540, 4),      # streaming
+    (torch.bfloat16, 3072, 1024),  # 12: TMA ring
+    (torch.bfloat16, 3080, 16),    # o past 12: ring
+    (torch.bfloat16, 64, 4096),    # e past 12: ring
+    (torch.float32, 1536, 512),    # ring
+    (torch.float32, 1540, 4),      # ring
+    (torch.float32, 28608, 64),    # a 112 KB row: streaming
 ])
 def test_junction_cache_sizes(dtype, dp, de):
     g = torch.Generator().manual_seed(44 + dp + de)
