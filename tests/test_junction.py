@@ -97,3 +97,16 @@ def test_junction_cache_sizes(dtype, dp, de):
                               tol_g=1e-2 if bf else 1e-5)
         assert np.abs(d_o[5]).max() == 0.0 and np.abs(d_o[11]).max() == 0.0
         np.testing.assert_array_equal(d_e[5], gr[5, (0 if embed_first else dp):][:de].double().numpy())
+
+
+def test_junction_ring_many_rows_per_warp():
+    """The TMA ring at a size where every warp takes many rows, so each of its
+    buffers is refilled several times (3072 -> 4096, bf16, T = 16384)."""
+    g = torch.Generator().manual_seed(45)
+    T, dp, de = 16384, 3072, 1024
+    o = (torch.randn(T, dp, generator=g) * 2).to(torch.bfloat16)
+    e = (torch.randn(T, de, generator=g) * 0.05).to(torch.bfloat16)
+    gr = (torch.randn(T, dp + de, generator=g) * 1e-2).to(torch.bfloat16)
+    o[T - 1] = 0
+    for embed_first in (False, True):
+        compare(o, e, gr, embed_first, tol_x=4e-3, tol_g=1e-2)
