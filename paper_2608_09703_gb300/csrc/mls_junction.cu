@@ -288,12 +288,11 @@ __global__ void __launch_bounds__(32 * kRowsPerBlock) junction_bwd_kernel(const 
 // Rows wider than the register cache.  Persistent CTAs of `warps` warps; each
 // warp owns a ring of `stages` row buffers in shared memory and the rows gw,
 // gw + GW, ... (gw its global warp index, GW the warps of the grid).  Its lane
-// 0 fetches whole rows
-// (o and e, and g in the backward) with 1-D bulk copies that complete on the
-// buffer's mbarrier, `stages` rows ahead, so every SM keeps tens of rows
-// of HBM reads in flight whatever T is.  The warp computes a row from shared
-// memory, in the same lane and column order as the kernels above, and stores
-// its outputs with coalesced 16-byte stores.
+// 0 fetches whole rows (o and e, and g in the backward) with 1-D bulk copies
+// that complete on the buffer's mbarrier, `stages` rows ahead, so every SM
+// keeps several rows of HBM reads in flight whatever T is.  The warp computes
+// a row from shared memory, in the same lane and column order as the kernels
+// above, and stores its outputs with coalesced 16-byte stores.
 constexpr int kRingWarps = 4;
 constexpr int kRingStages = 4;
 constexpr uint32_t kRingSmem = 220 * 1024;  // dynamic shared memory a CTA may use
