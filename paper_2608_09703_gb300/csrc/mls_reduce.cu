@@ -1,8 +1,8 @@
 // Row reductions of the forward pass, the token count of the backward and an
 // fp32 transpose (used only for fp32 inputs, whose tf32 GEMMs read K-major copies).
 //
-// merge_kernel: one warp per token combines the partial row states that the
-// head kernel wrote per (CTA, half tile) into
+// merge_kernel: a block of 8 warps combines, for 8 tokens, the partial row
+// states that the head kernel wrote per (CTA, half tile) into
 //   lse_m    = logsumexp(z_m)            CE_m = lse_m - z_m[y]
 //   lset_m   = logsumexp(z_m / tau)
 //   E_q[z_m] = sum_v q_v z_m[v]          from A_m / S_t (q = softmax(z_t / tau))
@@ -35,73 +35,164 @@ __device__ __forceinline__ double block_sum_double(double v, double* sh) {
   return s;  // valid in thread 0
 }
 
-__device__ __forceinline__ float warp_max_f(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
-  return v;
-}
-__device__ __forceinline__ float warp_sum_f(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  return v;
-}
+// A block of 8 warps merges kMergeTokens = 8 consecutive tokens.  Lane l of
+// warp w takes token t0 + (l mod 8) and the partials k = 4 w + l / 8,
+// k + 32, ...: the 8 lanes of a group read 32 consecutive bytes (one sector)
+// of each (partial, field, sub-model).  Round 1 takes every sub-model's row
+// maximum, round 2 its sums.  The partials of a token are combined in a fixed
+// order (within a lane, across the 4 lane groups by butterflies, across the 8
+// warps in warp order), so results are deterministic.
+constexpr int kMergeWarps = 8;
+static_assert(kMergeTokens == 8, "a lane group covers 8 tokens");
 
-// One warp per token: lane k takes partials k, k + 32, ...; warp reductions
-// (butterflies, so every lane holds the same result and the order is fixed)
-// combine them, and lane 0 writes the token's outputs.
-__global__ void __launch_bounds__(kMergeTokens * 32) merge_kernel(const __grid_constant__ MergeParams p) {
-  __shared__ double sh_sum[kMergeTokens], sh_cnt[kMergeTokens];
+__global__ void __launch_bounds__(kMergeWarps * 32, 4) merge_kernel(const __grid_constant__ MergeParams p) {
+  __shared__ float sh_f[4][kMergeWarps][kMaxModels][kMergeTokens];  // max, then s1, st, acc, zy
+  __shared__ int sh_am[kMergeWarps][kMaxModels][kMergeTokens];
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const long long t = static_cast<long long>(blockIdx.x) * kMergeTokens + w;
+  const int j = lane & 7, grp = lane >> 3;  // token within the block, partial group
+  const long long T = p.T;
+  const long long t = static_cast<long long>(blockIdx.x) * kMergeTokens + j;
+  const bool live = t < T;
+  const long long MT = static_cast<long long>(p.M) * T;
+  const long long PS = kPartFields * MT;  // stride between partials
+  const int tc = p.teacher;
+  const int k0 = 4 * w + grp;
+
+  // ---- round 1: row maxima of every sub-model
+  float mx[kMaxModels];
+#pragma unroll
+  for (int m = 0; m < kMaxModels; ++m) mx[m] = -INFINITY;
+  if (live)
+    for (int k = k0; k < p.nparts; k += 32) {
+#pragma unroll
+      for (int m = 0; m < kMaxModels; ++m)
+        if (m < p.M) mx[m] = fmaxf(mx[m], p.part[k * PS + kPartMax * MT + m * T + t]);
+    }
+#pragma unroll
+  for (int m = 0; m < kMaxModels; ++m) {
+    mx[m] = fmaxf(mx[m], __shfl_xor_sync(0xffffffffu, mx[m], 8));
+    mx[m] = fmaxf(mx[m], __shfl_xor_sync(0xffffffffu, mx[m], 16));
+    if (grp == 0) sh_f[0][w][m][j] = mx[m];
+  }
+  __syncthreads();
+#pragma unroll
+  for (int m = 0; m < kMaxModels; ++m) {
+    float v = -INFINITY;
+    for (int ww = 0; ww < kMergeWarps; ++ww) v = fmaxf(v, sh_f[0][ww][m][j]);
+    mx[m] = v;
+  }
+  float mT = -INFINITY;
+#pragma unroll
+  for (int m = 0; m < kMaxModels; ++m)
+    if (m == tc) mT = mx[m];
+  __syncthreads();  // sh_f[0] is reused below
+
+  // ---- round 2: sums.  The teacher's weighted sum is relative to its own
+  // maximum: B_k = sum q~ (z - m_k) log2(e)/tau; moving it to the row maximum
+  // mT adds (m_k - mT) log2(e)/tau per unit of weight before the weights are
+  // rescaled.  A student's A_k is relative to the teacher's maximum of the
+  // same partial.
+  float s1[kMaxModels], st[kMaxModels], acc[kMaxModels], zy[kMaxModels];
+  int am[kMaxModels];
+#pragma unroll
+  for (int m = 0; m < kMaxModels; ++m) {
+    s1[m] = st[m] = acc[m] = zy[m] = 0.f;
+    am[m] = INT_MAX;
+  }
+  if (live)
+    for (int k = k0; k < p.nparts; k += 32) {
+      const float mtk = p.part[k * PS + kPartMax * MT + static_cast<long long>(tc) * T + t];
+#pragma unroll
+      for (int m = 0; m < kMaxModels; ++m) {
+        if (m >= p.M) continue;
+        const float* P = p.part + k * PS + static_cast<long long>(m) * T + t;
+        const float mk = P[kPartMax * MT];
+        if (m == tc) {
+          if (mk != -INFINITY) {
+            const float f1 = exp2f((mk - mT) * p.L1);
+            const float ft = exp2f((mk - mT) * p.Ltau);
+            const float stk = P[kPartSumTau * MT];
+            s1[m] += P[kPartSum1 * MT] * f1;
+            st[m] += stk * ft;
+            acc[m] += (P[kPartAcc * MT] + (mk - mT) * p.Ltau * stk) * ft;
+          }
+        } else {
+          if (mk != -INFINITY) {
+            s1[m] += P[kPartSum1 * MT] * exp2f((mk - mx[m]) * p.L1);
+            st[m] += P[kPartSumTau * MT] * exp2f((mk - mx[m]) * p.Ltau);
+          }
+          if (mtk != -INFINITY) acc[m] += P[kPartAcc * MT] * exp2f((mtk - mT) * p.Ltau);
+        }
+        zy[m] += P[kPartTarget * MT];
+        if (mk == mx[m]) am[m] = min(am[m], __float_as_int(P[kPartArgmax * MT]));
+      }
+    }
+#pragma unroll
+  for (int m = 0; m < kMaxModels; ++m) {
+#pragma unroll
+    for (int o = 8; o <= 16; o <<= 1) {
+      s1[m] += __shfl_xor_sync(0xffffffffu, s1[m], o);
+      st[m] += __shfl_xor_sync(0xffffffffu, st[m], o);
+      acc[m] += __shfl_xor_sync(0xffffffffu, acc[m], o);
+      zy[m] += __shfl_xor_sync(0xffffffffu, zy[m], o);
+      am[m] = min(am[m], __shfl_xor_sync(0xffffffffu, am[m], o));
+    }
+    if (grp == 0) {
+      sh_f[0][w][m][j] = s1[m];
+      sh_f[1][w][m][j] = st[m];
+      sh_f[2][w][m][j] = acc[m];
+      sh_f[3][w][m][j] = zy[m];
+      sh_am[w][m][j] = am[m];
+    }
+  }
+  __syncthreads();
+  if (w != 0) return;
+
+  // ---- warp 0, lanes 0-7: one token each
   double contrib = 0.0, cnt = 0.0;
-  if (t < p.T) {  // warp-uniform
-    const long long T = p.T;
-    const long long MT = static_cast<long long>(p.M) * T;
-    const long long PS = kPartFields * MT;  // stride between partials
+  if (lane < kMergeTokens && live) {
+#pragma unroll
+    for (int m = 0; m < kMaxModels; ++m) {
+      float a = 0.f, b = 0.f, c = 0.f, d = 0.f;
+      int e = INT_MAX;
+      for (int ww = 0; ww < kMergeWarps; ++ww) {
+        a += sh_f[0][ww][m][j];
+        b += sh_f[1][ww][m][j];
+        c += sh_f[2][ww][m][j];
+        d += sh_f[3][ww][m][j];
+        e = min(e, sh_am[ww][m][j]);
+      }
+      s1[m] = a;
+      st[m] = b;
+      acc[m] = c;
+      zy[m] = d;
+      am[m] = e;
+    }
     const int y = p.y[t];
     const bool bad = y >= p.V;
-    if (bad && lane == 0) atomicOr(p.status, kStatusBadTarget);
+    if (bad) atomicOr(p.status, kStatusBadTarget);
     const bool valid = y >= 0 && !bad;
     const float invtau = 1.0f / p.tau;
-    const int tc = p.teacher;
-    const float* Pt = p.part + static_cast<long long>(tc) * T + t;
-
-    // teacher: row maximum, sums at tau = 1 and tau, teacher-weighted sum B
-    float mT = -INFINITY;
-    for (int k = lane; k < p.nparts; k += 32) mT = fmaxf(mT, Pt[k * PS + kPartMax * MT]);
-    mT = warp_max_f(mT);
-    // The teacher's weighted sum is relative to its own maximum:
-    // B_k = sum q~ (z - m_k) log2(e)/tau; moving it to the row maximum mT adds
-    // (m_k - mT) log2(e)/tau per unit of weight before the weights are rescaled.
     float s1T = 0.f, stT = 0.f, bT = 0.f, zT = 0.f;
     int amT = INT_MAX;
-    for (int k = lane; k < p.nparts; k += 32) {
-      const float* P = Pt + k * PS;
-      const float mk = P[kPartMax * MT];
-      if (mk != -INFINITY) {
-        const float f1 = exp2f((mk - mT) * p.L1);
-        const float ft = exp2f((mk - mT) * p.Ltau);
-        const float stk = P[kPartSumTau * MT];
-        s1T += P[kPartSum1 * MT] * f1;
-        stT += stk * ft;
-        bT += (P[kPartAcc * MT] + (mk - mT) * p.Ltau * stk) * ft;
+#pragma unroll
+    for (int m = 0; m < kMaxModels; ++m)
+      if (m == tc) {
+        s1T = s1[m];
+        stT = st[m];
+        bT = acc[m];
+        zT = zy[m];
+        amT = am[m];
       }
-      zT += P[kPartTarget * MT];
-      if (mk == mT) amT = min(amT, __float_as_int(P[kPartArgmax * MT]));
-    }
-    s1T = warp_sum_f(s1T);
-    stT = warp_sum_f(stT);
-    bT = warp_sum_f(bT);
-    zT = warp_sum_f(zT);
-    amT = __reduce_min_sync(0xffffffffu, amT);
     const float lseT = mT + logf(s1T);
     const float lsetT = mT * invtau + logf(stT);
     // H(q) = log S - E_q[(z - mT)/tau]; both terms are >= 0
     const float HqT = logf(stT) - bT / (stT * p.L1);
-
-    for (int m = 0; m < p.M; ++m) {
+#pragma unroll
+    for (int m = 0; m < kMaxModels; ++m) {
+      if (m >= p.M) continue;
       float lse, lset, ce, ld, kl, L;
-      int am;
+      int amm;
       if (m == tc) {
         lse = lseT;
         lset = lsetT;
@@ -109,68 +200,40 @@ __global__ void __launch_bounds__(kMergeTokens * 32) merge_kernel(const __grid_c
         ld = HqT;
         kl = 0.f;
         L = ce;
-        am = amT;
+        amm = amT;
       } else {
-        const float* Pm = p.part + static_cast<long long>(m) * T + t;
-        float mm = -INFINITY;
-        for (int k = lane; k < p.nparts; k += 32) mm = fmaxf(mm, Pm[k * PS + kPartMax * MT]);
-        mm = warp_max_f(mm);
-        float s1 = 0.f, st = 0.f, A = 0.f, zy = 0.f;
-        am = INT_MAX;
-        for (int k = lane; k < p.nparts; k += 32) {
-          const float* P = Pm + k * PS;
-          const float mk = P[kPartMax * MT];
-          if (mk != -INFINITY) {
-            s1 += P[kPartSum1 * MT] * exp2f((mk - mm) * p.L1);
-            st += P[kPartSumTau * MT] * exp2f((mk - mm) * p.Ltau);
-          }
-          const float mtk = Pt[k * PS + kPartMax * MT];  // the teacher max this A is relative to
-          if (mtk != -INFINITY) A += P[kPartAcc * MT] * exp2f((mtk - mT) * p.Ltau);
-          zy += P[kPartTarget * MT];
-          if (mk == mm) am = min(am, __float_as_int(P[kPartArgmax * MT]));
-        }
-        s1 = warp_sum_f(s1);
-        st = warp_sum_f(st);
-        A = warp_sum_f(A);
-        zy = warp_sum_f(zy);
-        am = __reduce_min_sync(0xffffffffu, am);
-        lse = mm + logf(s1);
-        lset = mm * invtau + logf(st);
-        ce = lse - zy;
-        ld = lset - (A / stT) * invtau;
+        lse = mx[m] + logf(s1[m]);
+        lset = mx[m] * invtau + logf(st[m]);
+        ce = lse - zy[m];
+        ld = lset - (acc[m] / stT) * invtau;
         kl = ld - HqT;
         L = (1.f - p.alpha) * ce + p.alpha * ld;
+        amm = am[m];
       }
       if (!valid) ce = ld = kl = L = 0.f;
-      if (lane == 0) {
-        const long long o = static_cast<long long>(m) * T + t;
-        p.tok_loss[o] = L;
-        if (p.tok_diag) {
-          p.tok_diag[o] = ce;
-          p.tok_diag[MT + o] = ld;
-          p.tok_diag[2 * MT + o] = kl;
-        }
-        if (p.argmax) p.argmax[o] = am;
-        p.stats[o] = lse;
-        p.stats[MT + o] = lset;
+      const long long o = static_cast<long long>(m) * T + t;
+      p.tok_loss[o] = L;
+      if (p.tok_diag) {
+        p.tok_diag[o] = ce;
+        p.tok_diag[MT + o] = ld;
+        p.tok_diag[2 * MT + o] = kl;
       }
+      if (p.argmax) p.argmax[o] = amm;
+      p.stats[o] = lse;
+      p.stats[MT + o] = lset;
       contrib += static_cast<double>(p.w[m]) * static_cast<double>(L);
     }
     cnt = valid ? 1.0 : 0.0;
   }
-  if (lane == 0) {
-    sh_sum[w] = contrib;
-    sh_cnt[w] = cnt;
+  // the block's share, over its tokens in a fixed order
+#pragma unroll
+  for (int o = 4; o > 0; o >>= 1) {
+    contrib += __shfl_down_sync(0xffffffffu, contrib, o);
+    cnt += __shfl_down_sync(0xffffffffu, cnt, o);
   }
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    double bs = 0.0, bc = 0.0;
-    for (int i = 0; i < kMergeTokens; ++i) {
-      bs += sh_sum[i];
-      bc += sh_cnt[i];
-    }
-    p.block_sum[blockIdx.x] = bs;
-    p.block_cnt[blockIdx.x] = static_cast<long long>(bc);
+  if (lane == 0) {
+    p.block_sum[blockIdx.x] = contrib;
+    p.block_cnt[blockIdx.x] = static_cast<long long>(cnt);
   }
 }
 
@@ -239,7 +302,7 @@ cudaError_t launch_transpose(const float* in, long long rows, long long cols, lo
 
 cudaError_t launch_merge(const MergeParams& p, int blocks, cudaStream_t s) {
   if (blocks <= 0) return cudaSuccess;
-  merge_kernel<<<blocks, kMergeTokens * 32, 0, s>>>(p);
+  merge_kernel<<<blocks, kMergeWarps * 32, 0, s>>>(p);
   return cudaGetLastError();
 }
 
