@@ -23,6 +23,7 @@ import argparse
 import hashlib
 import json
 import os
+import re
 import statistics
 import subprocess
 import sys
@@ -50,20 +51,30 @@ def peaks():
         return dict(FALLBACK_PEAKS), "fallback"
 
 
+def source_hash(names) -> str:
+    """Hash of the code of C/CUDA source files, blind to comments and layout:
+    // and /* */ comments are dropped and whitespace runs collapsed, so only a
+    change that can change the compiled kernel changes the hash."""
+    h = hashlib.sha256()
+    for name in names:
+        with open(os.path.join(ROOT, name), encoding="utf-8") as fh:
+            text = fh.read()
+        text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+        text = re.sub(r"//[^\n]*", " ", text)
+        h.update(" ".join(text.split()).encode())
+    return h.hexdigest()[:16]
+
+
 def traffic_for(kernel: str):
     """DRAM bytes per launch from the committed ncu summary, if it was taken
-    on the current sources of that kernel (the files it lists); else None."""
+    on the current code of that kernel (the files it lists); else None."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as fh:
             e = json.load(fh).get(kernel)
-        h = hashlib.sha256()
-        for name in e["sources"]:
-            with open(os.path.join(ROOT, name), "rb") as fh:
-                h.update(fh.read())
+        if e.get("source_hash") != source_hash(e["sources"]):
+            return None
     except Exception:
-        return None
-    if e.get("source_hash") != h.hexdigest()[:16]:
         return None
     return e.get("traffic_bytes_per_launch")
 

@@ -254,7 +254,7 @@ struct MergeParams {
   int* status;
 };
 
-constexpr int kMergeTokens = 8;        // tokens per merge block: one warp per token
+constexpr int kMergeTokens = 8;        // tokens per merge block (8 warps share them)
 constexpr int kEvalMergeTokens = 128;  // tokens per evaluation-merge block: one thread per token
 
 // Launchers (return the cudaError_t of the launch).
