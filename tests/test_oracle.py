@@ -521,3 +521,64 @@ def test_spec_verify_output_follows_the_verifier():
     first = np.where(n == 1, draft[:, 0], nxt)
     freq = np.bincount(first, minlength=V) / N
     assert np.abs(freq - p).max() < 4.5 * np.sqrt(p * (1 - p) / N).max()
+
+
+def test_spec_verify_nucleus_hand_worked_top_p_09():
+    """A nucleus cut strictly inside (0, 1), worked out by hand (V = 4, top_p = 0.9,
+    temperature 1, logits = log-probabilities so softmax returns them exactly).
+    The two nuclei keep different masses, so each renormalisation shows.
+
+    draft    q = (0.50, 0.30, 0.15, 0.05): cumulative 0.50, 0.80, 0.95 >= 0.9, so
+             tokens {0, 1, 2} are kept and q' = (0.50, 0.30, 0.15, 0) / 0.95.
+    verifier p = (0.08, 0.22, 0.30, 0.40): sorted 0.40, 0.30, 0.22 -> 0.92, so
+             tokens {3, 2, 1} are kept and p' = (0, 0.22, 0.30, 0.40) / 0.92.
+    Drafted x = 1: accept iff u q'(1) < p'(1), i.e. u < (0.22 / 0.92) / (0.30 / 0.95)
+    = 0.75725.  Without renormalising the cut would be 0.73333; renormalising
+    only p gives 0.79710, only q 0.69667.
+    Residual max(0, p' - q') = (0, 0, 0.30/0.92 - 0.15/0.95, 0.40/0.92) =
+    (0, 0, 0.16819, 0.43478): token 2 iff u < 0.16819 / 0.60297 = 0.27894
+    (0.27273 without renormalising).
+    Bonus position, verifier p = (0.60, 0.25, 0.10, 0.05): kept {0, 1, 2},
+    CDF 0.63158, 0.89474, 1: u = 0.88 gives token 1 (keeping token 3 would give 2)."""
+    q = np.array([0.50, 0.30, 0.15, 0.05])
+    p0 = np.array([0.08, 0.22, 0.30, 0.40])
+    p1 = np.array([0.60, 0.25, 0.10, 0.05])
+    Wd = np.log(q)[:, None]
+    Wv = np.stack([np.log(p0), np.log(p1)], axis=1)
+    Hd, Hv = np.ones((1, 1)), np.eye(2)
+
+    def run(x, u_acc, u_res, u_bonus=0.5):
+        u = np.array([[[u_acc, u_res], [0.0, u_bonus]]])
+        n, nxt = orc.spec_verify(Hd, Wd, Hv, Wv, [[x]], u, temperature=1.0, top_p=0.9)
+        return int(n[0]), int(nxt[0])
+
+    # acceptance threshold 0.75725, between the unrenormalised 0.73333 and the
+    # p-only 0.79710
+    assert run(1, 0.745, 0.1, u_bonus=0.88) == (1, 1)   # accepted, bonus token 1
+    assert run(1, 0.77, 0.1) == (0, 2)                  # rejected, residual token 2
+    # the residual's cut between tokens 2 and 3 at 0.27894
+    assert run(1, 0.99, 0.276) == (0, 2)
+    assert run(1, 0.99, 0.282) == (0, 3)
+    # token 0 lies outside the verifier's nucleus (p' = 0): always rejected
+    assert run(0, 0.0, 0.276) == (0, 2)
+    # token 3 lies outside the draft's nucleus (q' = 0): rejected as well
+    assert run(3, 0.0, 0.5) == (0, 3)
+    # bonus CDF 0.63158, 0.89474: the nucleus drops token 3 before sampling
+    assert run(1, 0.5, 0.0, u_bonus=0.62) == (1, 0)
+    assert run(1, 0.5, 0.0, u_bonus=0.90) == (1, 2)
+
+
+def test_spec_verify_temperature_applies_before_the_nucleus():
+    """At temperature 0.5 the draft's q = (0.50, 0.30, 0.15, 0.05) sharpens to
+    q^2 / sum q^2 = (0.6849, 0.2466, 0.0616, 0.0068), whose cumulative passes 0.9
+    at the second token: only {0, 1} are kept, so a drafted token 2 (inside the
+    untempered nucleus) is now rejected."""
+    q = np.array([0.50, 0.30, 0.15, 0.05])
+    p = np.array([0.25, 0.25, 0.25, 0.25])
+    Wd, Wv = np.log(q)[:, None], np.stack([np.log(p), np.log(p)], axis=1)
+    Hd, Hv = np.ones((1, 1)), np.eye(2)
+    u = np.array([[[0.0, 0.5], [0.0, 0.5]]])
+    n, _ = orc.spec_verify(Hd, Wd, Hv, Wv, [[2]], u, temperature=0.5, top_p=0.9)
+    assert n[0] == 0
+    n, _ = orc.spec_verify(Hd, Wd, Hv, Wv, [[2]], u, temperature=1.0, top_p=0.9)
+    assert n[0] == 1
