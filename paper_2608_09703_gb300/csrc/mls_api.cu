@@ -109,6 +109,7 @@ long long ceil_div(long long a, long long b) { return (a + b - 1) / b; }
 struct Plan {
   int elt = 2;
   int ntt = 0, nvt = 0;
+  int band = 1;  // token tiles per band of the head and evaluation kernels' launch order
   // forward
   int S = 1, nparts = 0, merge_blocks = 0, eval_merge_blocks = 0;
   size_t off_part = 0, off_bsum = 0, off_bcnt = 0, fwd_bytes = 0;
@@ -148,6 +149,23 @@ int choose_splits(int ntt, long long tiles, int pairs) {
   return static_cast<int>(best);
 }
 
+// Token tiles per band of the head kernels' launch order (band_unit): the
+// pairs resident at one time re-read the hidden states of every sub-model for
+// the band's tokens once per vocabulary tile, so a band's H is kept within a
+// share of L2 that stays resident while W streams past it.  Fewer token tiles
+// per band mean more passes over W (one per band); the bands are made equal.
+#ifndef MLS_HEAD_BAND_BYTES
+#define MLS_HEAD_BAND_BYTES (48ll << 20)
+#endif
+int choose_band(int ntt, long long h_bytes_per_tile) {
+  if (ntt < 1) return 1;
+  long long band = MLS_HEAD_BAND_BYTES / (h_bytes_per_tile > 0 ? h_bytes_per_tile : 1);
+  if (band < 1) band = 1;
+  if (band >= ntt) return ntt;
+  const long long nbands = (ntt + band - 1) / band;
+  return static_cast<int>((ntt + nbands - 1) / nbands);
+}
+
 int validate(const mls_problem* p) {
   if (!p || p->M < 1 || p->M > MLS_MAX_MODELS || p->T < 0 || p->V < 1 || p->V > INT_MAX ||
       p->T > INT_MAX || !p->d)
@@ -176,6 +194,9 @@ Plan make_plan(const mls_problem* p, int pairs) {
   pl.nvt = static_cast<int>(ceil_div(V, kHeadBN));
   pl.S = choose_splits(pl.ntt, pl.nvt, pairs);
   pl.nparts = pl.S;
+  long long sum_d = 0;
+  for (int m = 0; m < p->M; ++m) sum_d += p->d[m];
+  pl.band = choose_band(pl.ntt, 2LL * kHeadBM * sum_d * pl.elt);
   pl.merge_blocks = static_cast<int>(ceil_div(T, kMergeTokens));
   pl.eval_merge_blocks = static_cast<int>(ceil_div(T, kEvalMergeTokens));
   size_t o = 0;
@@ -375,6 +396,7 @@ extern "C" int mls_head_loss_fwd(const mls_problem* p, const void* const* H, con
   hp.vt_begin = 0;
   hp.vt_end = pl.nvt;
   hp.S = pl.S;
+  hp.band = pl.band;
   hp.part = reinterpret_cast<float*>(wsb + pl.off_part);
   if ((rc = timed("head_fwd", s, [&] { return launch_head_fwd(hp, pl.elt == 4, p->tau == 1.0f, s); }))) return rc;
 
@@ -512,6 +534,7 @@ extern "C" int mls_head_loss_bwd(const mls_problem* p, const void* const* H, con
     hp.vt_begin = static_cast<int>(g * tiles_per_group);
     hp.vt_end = static_cast<int>(ceil_div(c0 + gc, kHeadBN));
     hp.S = choose_splits(pl.ntt, hp.vt_end - hp.vt_begin, dev->head_pairs);
+    hp.band = pl.band;
     hp.g_col0 = c0;
     if ((rc = timed("head_bwd", s, [&] { return launch_head_bwd(hp, tf32, p->tau == 1.0f, s); }))) return rc;
     if (tf32)
@@ -620,7 +643,11 @@ extern "C" const char* mls_strerror(int code) {
     case MLS_STATUS_TIMEOUT: return "a pipeline wait timed out; outputs are invalid";
     case MLS_STATUS_BAD_TARGET | MLS_STATUS_TIMEOUT: return "target >= V and a pipeline timeout";
     case MLS_STATUS_CHECK: return "an internal invariant failed (checked build)";
-    default: return "unknown code";
+    case MLS_STATUS_DRAIN:
+    case MLS_STATUS_TIMEOUT | MLS_STATUS_DRAIN:
+      return "a pipeline timeout, and a shutdown wait ran out: the CUDA context is unreliable";
+    default:
+      return code > 0 && code < 16 ? "several status bits are set (MLS_STATUS_* in mls.h)" : "unknown code";
   }
 }
 
@@ -725,6 +752,7 @@ extern "C" int mls_head_loss_fwd_noalloc(const mls_problem* p, const void* const
   hp.vt_begin = 0;
   hp.vt_end = pl.nvt;
   hp.S = pl.S;
+  hp.band = pl.band;
   hp.part = reinterpret_cast<float*>(wsb + pl.off_part);
   if ((rc = timed("head_fwd", s, [&] { return launch_head_fwd(hp, pl.elt == 4, p->tau == 1.0f, s); })))
     return rc;
@@ -798,6 +826,7 @@ extern "C" int mls_head_pairwise(const mls_problem* p, const void* const* H, con
   ep.ntt = pl.ntt;
   ep.nvt = pl.eval_nvt;
   ep.S = pl.eval_S;
+  ep.band = pl.band;
   ep.T = p->T;
   ep.V = p->V;
   ep.L1 = 1.4426950408889634f;

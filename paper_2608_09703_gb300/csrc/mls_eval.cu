@@ -90,7 +90,7 @@ __device__ __forceinline__ void eval_producer(const EvalParams& p, uint32_t base
   if (!ok && filled) {
     if (rank == 0) {
       for (int s = 0; s < kEvalStages; ++s)
-        if ((filled >> s) & 1u) mbar_wait_drain(EvalSmem::full(base, s), (lastpar >> s) & 1u, kDrainNs);
+        if ((filled >> s) & 1u) mbar_wait_drain(EvalSmem::full(base, s), (lastpar >> s) & 1u, kDrainNs, p.status);
     } else {
       spin_ns(kDrainNs);
     }
@@ -142,7 +142,7 @@ __device__ __forceinline__ void eval_mma(const EvalParams& p, uint32_t base, uin
     mma_commit_pair(EvalSmem::accf(base, j), 0x3);
   }
   mma_commit_pair(EvalSmem::drain(base), 0x1);
-  mbar_wait_drain(EvalSmem::drain(base), 0, kDrainNs);
+  mbar_wait_drain(EvalSmem::drain(base), 0, kDrainNs, p.status);
 }
 
 struct EvalState {
@@ -283,8 +283,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kHeadThreads, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + EvalSmem::kTmemSlot);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = cluster_ctarank();
-  const int pair = blockIdx.x >> 1;
-  const int tt = pair % p.ntt, split = pair / p.ntt;
+  int tt, split;
+  band_unit(static_cast<int>(blockIdx.x >> 1), p.ntt, p.S, p.band, tt, split);
   const int row_base = tt * 2 * kHeadBM + static_cast<int>(rank) * kHeadBM;
 
   if (threadIdx.x == 0) {

@@ -120,7 +120,7 @@ __device__ __forceinline__ void head_producer(const HeadParams& p, uint32_t base
     // the even CTA's barriers, so it waits out a bound no TMA load approaches.
     if (rank == 0) {
       for (int s = 0; s < kHeadStages; ++s)
-        if ((filled >> s) & 1u) mbar_wait_drain(HeadSmem::full(base, s), (lastpar >> s) & 1u, kDrainNs);
+        if ((filled >> s) & 1u) mbar_wait_drain(HeadSmem::full(base, s), (lastpar >> s) & 1u, kDrainNs, p.status);
     } else {
       spin_ns(kDrainNs);
     }
@@ -170,7 +170,7 @@ __device__ __forceinline__ void head_mma(const HeadParams& p, uint32_t base, uin
   }
   // Every MMA this thread issued has finished before TMEM is released.
   mma_commit_pair(HeadSmem::drain(base), 0x1);
-  mbar_wait_drain(HeadSmem::drain(base), 0, kDrainNs);
+  mbar_wait_drain(HeadSmem::drain(base), 0, kDrainNs, p.status);
 }
 
 // Waits for accumulator `acc` to be full; warp-uniform result.
@@ -678,9 +678,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kHeadThreads, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = cluster_ctarank();
-  const int pair = blockIdx.x >> 1;
-  const int tt = pair % p.ntt;
-  const int split = pair / p.ntt;
+  int tt, split;
+  band_unit(static_cast<int>(blockIdx.x >> 1), p.ntt, p.S, p.band, tt, split);
   const int row_base = tt * 2 * kHeadBM + static_cast<int>(rank) * kHeadBM;  // this CTA's tokens
 
   if (threadIdx.x == 0) {

@@ -38,6 +38,25 @@ constexpr uint32_t kHeadStageChunk = 32 * 64;
 constexpr uint32_t kHeadStaging = kHeadEpiWarps * 2 * kHeadStageChunk;
 constexpr uint32_t kHeadSmem = kHeadStages * (kHeadABytes + kHeadBBytes) + kHeadStaging + 1024 + 1024;
 
+// Token tile and vocabulary split of CTA pair `pair` in a head or evaluation
+// launch of ntt x S pairs.  Pairs are numbered band by band: a band is `band`
+// consecutive token tiles (the last one may be shorter) and all S splits of
+// them, token tile fastest.  The hardware starts clusters roughly in index
+// order, so the pairs resident at one time cover the token tiles of one band
+// and a few consecutive splits: the hidden states they re-read for every
+// vocabulary tile are the band's, and each vocabulary tile is fetched by all
+// the band's token tiles at about the same time.  band >= ntt gives the plain
+// token-fastest order over all token tiles.
+__host__ __device__ inline void band_unit(int pair, int ntt, int S, int band, int& tt, int& split) {
+  if (band < 1 || band > ntt) band = ntt;
+  const int per_band = band * S;
+  const int b = pair / per_band;
+  const int i = pair - b * per_band;
+  const int nb = ntt - b * band < band ? ntt - b * band : band;
+  tt = b * band + i % nb;
+  split = i / nb;
+}
+
 // Partial row state written by the forward head kernel, per (partial, field, model, token).
 // kPartAcc holds, for a student, sum_v q~_v z_m[v] with q~ relative to the
 // teacher's running maximum of the same partial; for the teacher,
@@ -53,6 +72,7 @@ struct HeadParams {
   int ntt;                       // token tiles of 2 * kHeadBM (one per CTA pair)
   int vt_begin, vt_end;          // vocabulary tiles handled by this launch
   int S;                         // CTAs per token tile (vocabulary splits)
+  int band;                      // token tiles per band of the launch order (band_unit)
   long long T, V;
   float L1;                      // log2(e)
   float Ltau;                    // log2(e) / tau
@@ -164,6 +184,7 @@ struct EvalParams {
   int ntt;                       // token tiles of 256 (one per CTA pair)
   int nvt;                       // vocabulary tiles of kEvalBN
   int S;                         // CTA pairs per token tile
+  int band;                      // token tiles per band of the launch order (band_unit)
   long long T, V;
   float L1;
   int* status;
