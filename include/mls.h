@@ -58,7 +58,10 @@ enum {
   MLS_ERR_DEVICE = -6,       /* current device is not a compute-capability 10.3 GPU */
   MLS_STATUS_BAD_TARGET = 1, /* some target was >= V; that token was treated as ignored */
   MLS_STATUS_TIMEOUT = 2,    /* a pipeline wait exceeded its bound; outputs are invalid */
-  MLS_STATUS_CHECK = 4       /* checked build only: an internal invariant failed */
+  MLS_STATUS_CHECK = 4,      /* checked build only: an internal invariant failed */
+  MLS_STATUS_DRAIN = 8       /* after a timeout, a kernel's bounded shutdown wait for its own
+                                copies or MMAs also ran out: some may still have been in flight
+                                when it exited, so the CUDA context should not be trusted */
 };
 
 /* Maximum number of sub-models per call. */

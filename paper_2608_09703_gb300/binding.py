@@ -23,7 +23,7 @@ MLS_BF16, MLS_FP32 = 0, 1
 MLS_OK = 0
 MLS_ERR_ARG, MLS_ERR_ALIGN, MLS_ERR_UNSUPPORTED = -1, -2, -3
 MLS_ERR_WORKSPACE, MLS_ERR_CUDA, MLS_ERR_DEVICE = -4, -5, -6
-MLS_STATUS_BAD_TARGET, MLS_STATUS_TIMEOUT, MLS_STATUS_CHECK = 1, 2, 4
+MLS_STATUS_BAD_TARGET, MLS_STATUS_TIMEOUT, MLS_STATUS_CHECK, MLS_STATUS_DRAIN = 1, 2, 4, 8
 MLS_MAX_MODELS = 4
 
 

@@ -15,6 +15,7 @@ namespace mls {
 constexpr int kStatusBadTarget = 1;
 constexpr int kStatusTimeout = 2;
 constexpr int kStatusCheck = 4;
+constexpr int kStatusDrain = 8;
 
 // Invariant checks of the checked build (-DMLS_CHECKED, libmls_checked.so):
 // a failed condition raises kStatusCheck in the status word and execution
@@ -143,11 +144,17 @@ __device__ __forceinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity,
   }
 }
 
-// Bounded wait used only while shutting down after an abort.
-__device__ __forceinline__ bool mbar_wait_drain(uint32_t bar, uint32_t parity, uint64_t limit_ns) {
+// Bounded wait used only while shutting down after an abort.  If it runs out,
+// copies or MMAs this CTA issued may still be in flight when it exits; that is
+// recorded as kStatusDrain, which tells the caller not to trust the context.
+__device__ __forceinline__ bool mbar_wait_drain(uint32_t bar, uint32_t parity, uint64_t limit_ns,
+                                                int* status) {
   const uint64_t t0 = global_timer_ns();
   while (!mbar_try_wait(bar, parity)) {
-    if (global_timer_ns() - t0 > limit_ns) return false;
+    if (global_timer_ns() - t0 > limit_ns) {
+      atomicOr(status, kStatusDrain);
+      return false;
+    }
   }
   return true;
 }

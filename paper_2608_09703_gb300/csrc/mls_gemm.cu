@@ -156,7 +156,7 @@ __device__ __forceinline__ void gemm_producer(const GemmParams& p, uint32_t base
     // the even CTA's barriers, so it waits out a bound no TMA load approaches.
     if (rank == 0) {
       for (int s = 0; s < kGemmStages; ++s)
-        if ((filled >> s) & 1u) mbar_wait_drain(GemmSmem::full(base, s), (lastpar >> s) & 1u, kDrainNs);
+        if ((filled >> s) & 1u) mbar_wait_drain(GemmSmem::full(base, s), (lastpar >> s) & 1u, kDrainNs, p.status);
     } else {
       spin_ns(kDrainNs);
     }
@@ -213,7 +213,7 @@ __device__ __forceinline__ void gemm_mma(const GemmParams& p, uint32_t base, uin
     if (acc == 0) acc_par ^= 1u;
   }
   mma_commit_pair(GemmSmem::drain(base), 0x1);
-  mbar_wait_drain(GemmSmem::drain(base), 0, kDrainNs);
+  mbar_wait_drain(GemmSmem::drain(base), 0, kDrainNs, p.status);
 }
 
 // Largest of 32 values, as a tree (depth 5, not a 32-step chain).

@@ -339,7 +339,12 @@ __global__ void __launch_bounds__(32 * kRingWarps)
   bool ok = true;
   for (long long r = gw; r < p.T; r += GW, ++i) {
     const int st = static_cast<int>(i % stages);
-    if (!mbar_wait(bar0 + 8u * st, static_cast<uint32_t>((i / stages) & 1), &abort_flag, p.status)) {
+    // Every lane waits, but the warp leaves together: a lane that saw the
+    // buffer land must not go on to the full-warp reductions below while a
+    // lane that saw another warp's abort has left.
+    const bool landed =
+        mbar_wait(bar0 + 8u * st, static_cast<uint32_t>((i / stages) & 1), &abort_flag, p.status);
+    if (!__all_sync(0xffffffffu, landed)) {
       ok = false;
       break;
     }
@@ -430,7 +435,7 @@ __global__ void __launch_bounds__(32 * kRingWarps)
     for (long long k = i; k < i + stages; ++k)
       if (gw + k * GW < p.T)
         mbar_wait_drain(bar0 + 8u * static_cast<uint32_t>(k % stages),
-                        static_cast<uint32_t>((k / stages) & 1), kDrainNs);
+                        static_cast<uint32_t>((k / stages) & 1), kDrainNs, p.status);
   }
 }
 
