@@ -51,17 +51,67 @@ def peaks():
         return dict(FALLBACK_PEAKS), "fallback"
 
 
+def pick_peak(pk: dict, region_s: float, clocks: dict | None):
+    """The bf16 peak a kernel timed in this region is measured against.
+
+    MEASURED_PEAKS.json holds cuBLAS as a burst (best of a few calls, at the
+    maximum clock) and as a seconds-long loop under the power cap.  A region
+    shorter than a second, or one whose median SM clock stayed within 5% of the
+    maximum, ran at burst clocks: the burst figure is its peak.  Only a region
+    of seconds that settled below that clock is held to the sustained figure.
+    Returns (peak TFLOP/s, regime, reason)."""
+    burst, sus = float(pk["bf16_tflops"]), float(pk["bf16_tflops_sustained"])
+    mhz = (clocks or {}).get("sm_mhz")
+    mx = (clocks or {}).get("sm_max_mhz") or pk.get("sm_max_mhz")
+    if region_s < 1.0:
+        return burst, "burst", f"timed region {region_s:.2f} s (< 1 s)"
+    if mhz and mx and mhz >= 0.95 * mx:
+        return burst, "burst", f"median SM clock {mhz:.0f} of {mx:.0f} MHz"
+    if not mhz:
+        return burst, "burst", "no clock samples; burst assumed"
+    return sus, "sustained", f"timed region {region_s:.1f} s at median {mhz:.0f} of {mx:.0f} MHz"
+
+
+def strip_comments(text: str) -> str:
+    """C/CUDA source without its // and /* */ comments; string and character
+    literals are copied as they are (a // inside a string is not a comment).
+    A block comment becomes one space, or its newlines if it spans lines."""
+    out, i, n = [], 0, len(text)
+    while i < n:
+        c = text[i]
+        if c in "\"'":
+            j = i + 1
+            while j < n and text[j] != c and text[j] != "\n":
+                j += 2 if text[j] == "\\" else 1
+            out.append(text[i:j + 1])
+            i = j + 1
+        elif text.startswith("//", i):
+            j = text.find("\n", i)
+            i = n if j < 0 else j
+        elif text.startswith("/*", i):
+            j = text.find("*/", i + 2)
+            j = n if j < 0 else j + 2
+            out.append("\n" * text.count("\n", i, j) or " ")
+            i = j
+        else:
+            out.append(c)
+            i += 1
+    return "".join(out)
+
+
 def source_hash(names) -> str:
-    """Hash of the code of C/CUDA source files, blind to comments and layout:
-    // and /* */ comments are dropped and whitespace runs collapsed, so only a
-    change that can change the compiled kernel changes the hash."""
+    """Hash of the code of C/CUDA source files, blind to comments and to the
+    spacing within a line: comments are dropped (strip_comments), runs of
+    spaces and tabs collapsed, blank lines dropped.  Line breaks are kept, so a
+    change that can change the compiled code (a token moved across the end of a
+    preprocessor line, say) changes the hash."""
     h = hashlib.sha256()
     for name in names:
         with open(os.path.join(ROOT, name), encoding="utf-8") as fh:
-            text = fh.read()
-        text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
-        text = re.sub(r"//[^\n]*", " ", text)
-        h.update(" ".join(text.split()).encode())
+            text = strip_comments(fh.read())
+        lines = (" ".join(l.split()) for l in text.splitlines())
+        h.update("\n".join(l for l in lines if l).encode())
+        h.update(b"\0")
     return h.hexdigest()[:16]
 
 
@@ -351,18 +401,25 @@ def gpu_arm(args, rank, world, local):
     launches, total_ms = kern[dom]
     flops_launch = KERNELS[dom] * (step_flops / 4) / (launches / args.steps)
     achieved = flops_launch / (total_ms / launches / 1e3) / 1e12
-    # The kernels are timed inside a loop of back-to-back steps, the regime in
-    # which the clock settles under the power cap: the sustained bf16 figure
-    # is the denominator; the burst figure is reported beside it.
-    peak = float(pk["bf16_tflops_sustained"])
-    burst = float(pk["bf16_tflops"])
+    burst, sus = float(pk["bf16_tflops"]), float(pk["bf16_tflops_sustained"])
+    peak, regime, why = pick_peak(pk, ms * args.steps / 1e3, clocks)
     roofline = {"bound": "tensor", "kernel": dom, "achieved": achieved, "peak": peak,
-                "unit": "TFLOP/s", "frac": achieved / peak, "frac_of_burst": achieved / burst,
-                "peak_source": (f"{pk_src} bf16 dense sustained (MEASURED_PEAKS.json; burst {burst})"
-                                if pk_src == "measured" else "fallback 1.7 PFLOP/s bf16 sustained"),
+                "unit": "TFLOP/s", "frac": achieved / peak, "peak_regime": regime,
+                "peak_why": why,
+                "peak_source": (f"{pk_src} dense bf16 {regime} (MEASURED_PEAKS.json: burst {burst}, "
+                                f"sustained {sus})" if pk_src == "measured"
+                                else f"fallback dense bf16 {regime}"),
                 "flops_per_launch": flops_launch,
                 "traffic": traffic_for(dom)}
     gpu_launches = sum(v[0] for v in kern.values())
+
+    # ---- the same step looped for seconds: the regime of a training run, in
+    # which the clock settles under the power cap
+    sustained = None
+    if args.sustain_s > 0:
+        nvtx.range_push("sustained_steps")
+        sustained = sustained_run(args, step, ms, stream, dev, pk, step_flops, wl, world)
+        nvtx.range_pop()
 
     # ---- evaluation metrics between sub-models (forward only), same inputs
     pairwise = None
@@ -382,8 +439,10 @@ def gpu_arm(args, rank, world, local):
         pw_ms = e0.elapsed_time(e1) / n_pw
         k_launches, k_ms = kp["pairwise"]
         k_tflops = (step_flops / 4) / (k_ms / k_launches / 1e3) / 1e12
+        pw_peak, pw_regime, _ = pick_peak(pk, pw_ms * n_pw / 1e3, None)
         pairwise = {"ms_per_call": pw_ms, "tokens_per_s": wl.T / (pw_ms / 1e3),
-                    "kernel_tflops": k_tflops, "kernel_frac_of_sustained": k_tflops / peak,
+                    "kernel_tflops": k_tflops, "kernel_frac": k_tflops / pw_peak,
+                    "peak_tflops": pw_peak, "peak_regime": pw_regime,
                     "flops_per_call": step_flops / 4,
                     "what": "per-token KL(p_i||p_j) for all ordered sub-model pairs, means and "
                             "top-1 agreement (forward only)"}
@@ -440,16 +499,61 @@ def gpu_arm(args, rank, world, local):
         + (f" with the teacher's x{wl.teacher_scale:g}" if wl.teacher_scale != 1.0 else "")
         + f", {wl.targets} targets; FineWeb-Edu not available)",
         "config": workload_config(wl, world),
-        "tensor_frac_step": step_flops / (ms_max / 1e3) / 1e12 / burst,
-        "tensor_frac_step_sustained": step_flops / (ms_max / 1e3) / 1e12 / peak,
+        # 8*T*V*sum(d) per step against the peak of the timed region's regime
+        "tensor_frac_step": step_flops / (ms_max / 1e3) / 1e12 / peak,
         # the model-FLOPs convention 6*T*V*sum(d), which leaves out the
         # backward's recompute of the logits
-        "tensor_frac_step_6tvd": 0.75 * step_flops / (ms_max / 1e3) / 1e12 / burst,
+        "tensor_frac_step_6tvd": 0.75 * step_flops / (ms_max / 1e3) / 1e12 / peak,
+        "peak_regime": {"regime": regime, "tflops": peak, "why": why},
         "roofline": roofline, "kernels": per_kernel, "gpu_launches": gpu_launches,
-        "clocks": clocks, "e2e": e2e, "cpu_baseline": cpu, "pairwise_eval": pairwise,
+        "clocks": clocks, "sustained": sustained, "e2e": e2e, "cpu_baseline": cpu,
+        "pairwise_eval": pairwise,
         "junction": junction, "spec_verify": spec, "parity_sample": parity,
     }
     print(json.dumps(line), flush=True)
+
+
+def sustained_run(args, step, ms_short, stream, dev, pk, step_flops, wl, world):
+    """Back-to-back steps for about args.sustain_s seconds (after the short
+    timed region), clocks sampled throughout.  The fractions are of the
+    sustained bf16 peak when the clock settled below its maximum, else of the
+    burst peak (pick_peak)."""
+    import torch
+
+    from paper_2608_09703_gb300 import binding as B
+
+    n = max(10, int(args.sustain_s * 1e3 / max(ms_short, 1e-3)))
+    sampler = ClockSampler(dev.index if dev.index is not None else 0)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    torch.cuda.synchronize()
+    sampler.start()
+    time.sleep(0.25)
+    B.mls_profile_enable(True)
+    e0.record(stream)
+    for _ in range(n):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    kern = B.mls_profile_read()
+    B.mls_profile_enable(False)
+    clocks = sampler.stop()
+    ms = e0.elapsed_time(e1) / n
+    ms_max, value = aggregate(ms, wl.T, world)
+    peak, regime, why = pick_peak(pk, ms * n / 1e3, clocks)
+    out = {"steps": n, "seconds": ms * n / 1e3, "ms_per_step": ms_max, "value": value,
+           "unit": UNIT, "tensor_frac_step": step_flops / (ms_max / 1e3) / 1e12 / peak,
+           "tensor_frac_step_of_burst": step_flops / (ms_max / 1e3) / 1e12 / float(pk["bf16_tflops"]),
+           "peak_regime": {"regime": regime, "tflops": peak, "why": why}, "clocks": clocks,
+           "kernels": {}}
+    for name, (launches, total_ms) in kern.items():
+        entry = {"ms_per_step": total_ms / n}
+        if name in KERNELS:
+            f = KERNELS[name] * (step_flops / 4) / (launches / n)
+            t = f / (total_ms / launches / 1e3) / 1e12
+            entry.update({"tflops": t, "frac": t / peak})
+        out["kernels"][name] = entry
+    return out
 
 
 def junction_run(args, wl, dev, hbm_gbs):
@@ -616,11 +720,13 @@ def spec_run(args, dev, pk):
         ms = e0.elapsed_time(e1) / n
         gemm_ms = kp["spec_logits"][1] / n
         f = flops if not greedy else 2 * wl.V * Pv * wl.d_verify
+        sp_peak, sp_regime, _ = pick_peak(pk, ms * n / 1e3, None)
         out[mode] = {
             "ms_per_call": ms, "positions_per_s": Pv / (ms / 1e3),
             "kernel_ms": {k: v[1] / n for k, v in kp.items()},
             "logits_tflops": f / (gemm_ms / 1e3) / 1e12,
-            "logits_frac_of_sustained": f / (gemm_ms / 1e3) / 1e12 / float(pk["bf16_tflops_sustained"]),
+            "logits_frac": f / (gemm_ms / 1e3) / 1e12 / sp_peak,
+            "peak_tflops": sp_peak, "peak_regime": sp_regime,
         }
         if not greedy:
             # the selection kernels against one read of every probability row
@@ -643,6 +749,8 @@ def main():
     ap.add_argument("--no-spec", action="store_true")
     ap.add_argument("--tokens", type=int, default=0, help="override T (profiling captures)")
     ap.add_argument("--vocab", type=int, default=0, help="override V (profiling captures)")
+    ap.add_argument("--sustain-s", type=float, default=3.0,
+                    help="seconds of back-to-back steps for the sustained sub-record (0: skip)")
     ap.add_argument("--vocab-group", type=int, default=0,
                     help="backward vocabulary group in columns (0 = the library's choice)")
     args = ap.parse_args()

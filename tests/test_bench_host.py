@@ -8,16 +8,38 @@ sys.path.insert(0, ROOT)
 import bench  # noqa: E402
 
 
-def test_source_hash_ignores_comments_and_layout(tmp_path):
+def test_source_hash_ignores_comments_and_spacing(tmp_path):
     a = tmp_path / "a.cu"
     b = tmp_path / "b.cu"
     c = tmp_path / "c.cu"
     a.write_text("// header\nint f(int x) {\n  return x + 1;  /* one */\n}\n")
-    b.write_text("/* other\n   words */ int f(int x)   { return x + 1; }  // trailing\n")
-    c.write_text("int f(int x) { return x + 2; }\n")
+    b.write_text("int f(int x)   {\n\treturn   x + 1;\n\n}  // trailing\n")
+    c.write_text("int f(int x) {\n  return x + 2;\n}\n")
     ha, hb, hc = (bench.source_hash([str(p)]) for p in (a, b, c))
     assert ha == hb
     assert ha != hc
+
+
+def test_source_hash_keeps_line_breaks_and_string_literals(tmp_path):
+    files = {
+        # a token moved onto a preprocessor line changes the code
+        "p1.cu": "#define K 4\nint k = K;\n",
+        "p2.cu": "#define K 4 int k = K;\n",
+        # text after // inside a string literal is code, not a comment
+        "s1.cu": 'const char* s = "a // b";\n',
+        "s2.cu": 'const char* s = "a // c";\n',
+        "q1.cu": "char c = '\"'; int x = 1; // x\n",
+        "q2.cu": "char c = '\"'; int x = 2; // x\n",
+    }
+    h = {}
+    for name, text in files.items():
+        f = tmp_path / name
+        f.write_text(text)
+        h[name] = bench.source_hash([str(f)])
+    assert h["p1.cu"] != h["p2.cu"]
+    assert h["s1.cu"] != h["s2.cu"]
+    assert h["q1.cu"] != h["q2.cu"]
+    assert bench.strip_comments('x = "/* no */"; /* yes */ y;') == 'x = "/* no */";   y;'
 
 
 def test_traffic_figures_are_tied_to_listed_sources():

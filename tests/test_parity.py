@@ -205,7 +205,9 @@ def _full_size(name, nsample, seed=21):
 
 @pytest.mark.parametrize("name", ["suite3", "suite3_big", "suite4", "stress", "suite3_paper"])
 def test_full_size_sampled(name):
-    _full_size(name, nsample=10)
+    """64 sampled tokens (the first and last among them) of each full-size
+    workload: per-token losses, statistics, argmax and their dH rows."""
+    _full_size(name, nsample=64)
 
 
 def test_empty_token_batch():

@@ -304,17 +304,19 @@ def test_spec_exact_ties_at_the_nucleus_boundary():
 
 def test_spec_suite_shape_sampled():
     """The benchmark's shape (batch 102, draft length 6, 1024/3072 widths,
-    V = 50304): every output in range, two calls identical, and a sample of
-    sequences against the oracle."""
+    V = 50304): every output in range, two calls identical, and 34 of the 102
+    sequences (the first, the last and 32 drawn at random) against the oracle,
+    at least three quarters of them decided."""
     wl = synth.SPEC_WORKLOADS["spec_suite3"]
     Hd, Wd, Hv, Wv = synth.make_spec_inputs(wl, 50)
     u = synth.make_uniforms(wl.B, wl.gamma, 50)
-    seqs = np.array([0, 17, 50, 101])
+    pick = np.random.default_rng(50).choice(np.arange(1, wl.B - 1), 32, replace=False)
+    seqs = np.unique(np.concatenate([[0, wl.B - 1], pick]))
     rows = (seqs[:, None] * wl.gamma + np.arange(wl.gamma)[None]).reshape(-1)
     zd = exact(Hd[torch.as_tensor(rows)], Wd)
     draft = np.random.default_rng(50).integers(0, wl.V, (wl.B, wl.gamma)).astype(np.int32)
     draft[seqs] = draw_drafts(zd, wl.gamma, wl.temperature, wl.top_p, 50)
-    n1, nx1, _ = check(wl, Hd, Wd, Hv, Wv, draft, u, seqs=seqs, min_checked=0.5)
+    n1, nx1, _ = check(wl, Hd, Wd, Hv, Wv, draft, u, seqs=seqs, min_checked=0.75)
     n2, nx2 = run_gpu(wl, Hd, Wd, Hv, Wv, draft, u)
     assert (n1 == n2).all() and (nx1 == nx2).all()
 

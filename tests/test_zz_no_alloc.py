@@ -6,19 +6,23 @@ workspace, or a steady-state loop that must not call cudaMalloc because it can
 synchronise the device and take memory from a pool another allocator owns.  For
 them the library keeps a fixed scratch array of its own and offers a forward
 that needs no workspace.  This file checks, through the C ABI, that two calls in
-a row give the same results as the ordinary forward with a workspace, and that
-a problem too large for the built-in scratch is refused before anything runs.
+a row give the same results as the ordinary forward with a workspace and as
+the fp64 oracle, and that a problem too large for the built-in scratch is
+refused before anything runs.
 (It is collected last so that a run stopping at the first failure has already
 run every other test.)
 """
+import types
+
 import numpy as np
 import pytest
 import torch
 
+from oracle import oracle
 from paper_2608_09703_gb300 import binding as B
 from paper_2608_09703_gb300 import synth
 
-from helpers import rel_close
+from helpers import check_forward, exact_logits, rel_close
 
 pytestmark = pytest.mark.gpu
 
@@ -56,6 +60,15 @@ def test_noalloc_forward_matches_workspace_forward_on_two_calls():
             ok, err = rel_close(out[key].cpu().double().numpy(), want.cpu().double().numpy())
             assert ok, f"call {i}: {key} differs from the workspace forward (rel err {err})"
         assert np.array_equal(out["argmax"].cpu().numpy(), ref.argmax.cpu().numpy())
+        # and directly against the oracle, on the same inputs
+        yc = y.cpu().numpy().astype(np.int32)
+        want = oracle.forward(synth.as_oracle_arrays(H), synth.as_oracle_arrays(W), yc,
+                              teacher=wl.teacher_index, tau=wl.tau, alpha=wl.alpha, w=wl.weights)
+        got = types.SimpleNamespace(tok_loss=out["tok_loss"], tok_diag=out["tok_diag"],
+                                    stats=out["stats"], argmax=out["argmax"])
+        check_forward(got, want, logits=exact_logits(H, W))
+        ok, err = rel_close([out["loss"].item()], [want["loss"]])
+        assert ok, f"call {i}: scalar loss differs from the oracle (rel err {err})"
 
 
 def test_noalloc_rejects_problems_beyond_the_scratch():
