@@ -197,7 +197,7 @@ Plan make_plan(const mls_problem* p, int pairs) {
   long long sum_d = 0;
   for (int m = 0; m < p->M; ++m) sum_d += p->d[m];
   pl.band = choose_band(pl.ntt, 2LL * kHeadBM * sum_d * pl.elt);
-  pl.merge_blocks = static_cast<int>(ceil_div(T, kMergeTokens));
+  pl.merge_blocks = static_cast<int>(ceil_div(T, merge_tokens_per_block(pl.nparts)));
   pl.eval_merge_blocks = static_cast<int>(ceil_div(T, kEvalMergeTokens));
   size_t o = 0;
   pl.off_part = o;
@@ -242,7 +242,7 @@ Plan make_plan(const mls_problem* p, int pairs) {
   }
   pl.bwd_bytes = o;
 
-  pl.eval_nvt = static_cast<int>(ceil_div(V, kEvalBN));
+  pl.eval_nvt = static_cast<int>(ceil_div(V, eval_tile_cols(p->M)));
   pl.eval_S = choose_splits(pl.ntt, pl.eval_nvt, pairs);
   o = 0;
   pl.off_epart = o;
@@ -425,6 +425,19 @@ extern "C" int mls_head_loss_fwd(const mls_problem* p, const void* const* H, con
   return timed("final", s, [&] { return launch_final(mp.block_sum, mp.block_cnt, pl.merge_blocks, loss, s); });
 }
 
+// The dH problems of a backward GEMM launch run in wide units
+// (GemmProblem::wide) when each of them has a reduction of at least this many
+// k-blocks of 128 bytes, an even number of column tiles (no single-tile
+// units, which would only lose the epilogue overlap) and nothing to
+// accumulate (the first vocabulary group): a wide unit's two accumulators are
+// drained while no MMA runs, which costs a share inversely proportional to
+// the reduction and doubles when dH is read back.  Measured on one GB300 in a
+// seconds-long loop under the power cap: the 3-level suite at T = 8192 (786
+// k-blocks) gains 2.6% on the GEMM, while the paper's 3B suite (9 and 17
+// column tiles) lost 5% and the 4-level suite (504 k-blocks, four groups)
+// 2% when they ran wide.
+constexpr long long kWideMinBlocks = 512;
+
 // Two-class schedule of a persistent GEMM launch whose first n_long tiles take
 // cost_long and the other n_short cost_short (K-blocks plus a per-tile
 // allowance): see GemmParams.  The pairs that get one long tile fewer take
@@ -600,16 +613,34 @@ extern "C" int mls_head_loss_bwd(const mls_problem* p, const void* const* H, con
       gb.prob[M + m] = S.prob[m];
       gb.prob[M + m].a_map = gb.prob[M + m].b_map = M + m;
       gb.prob[M + m].a_mn = dh_long ? 1 : 0;
-      gb.prob[M + m].tile_begin += L.total_tiles;
+    }
+    // dH with a long reduction runs in wide units (two column tiles sharing
+    // each A tile of G); the units are numbered problem by problem, the long
+    // class first.
+    bool wide = true;
+    for (int i = 0; i < 2 * M; ++i) {
+      const GemmProblem& q = gb.prob[i];
+      if (q.a_mn == 0)
+        wide = wide && q.accumulate == 0 && q.tiles_n % 2 == 0 && ceil_div(q.K, KE) >= kWideMinBlocks;
+    }
+    int units = 0, n_long = 0;
+    for (int i = 0; i < 2 * M; ++i) {
+      GemmProblem& q = gb.prob[i];
+      q.wide = (wide && q.a_mn == 0) ? 1 : 0;
+      q.tile_begin = units;
+      units += static_cast<int>(ceil_div(q.Mrows, 2 * kGemmBM)) * (q.wide ? (q.tiles_n + 1) / 2 : q.tiles_n);
+      if (i == M - 1) n_long = units;
     }
     gb.nprob = 2 * M;
-    gb.total_tiles = L.total_tiles + S.total_tiles;
+    gb.total_tiles = units;
     gb.status = dev->status;
     const int grid = 2 * (gb.total_tiles < pairs ? gb.total_tiles : pairs);
-    // cost of a tile: its K-blocks plus an allowance for draining its 256x256 accumulator
+    // cost of a unit: its K-blocks (twice for a wide one) plus an allowance for
+    // draining its 256x256 accumulators
     constexpr long long kDrainBlocks = 8;
-    schedule_two_class(gb, grid / 2, L.total_tiles, ceil_div(L.prob[0].K, KE) + kDrainBlocks,
-                       S.total_tiles, ceil_div(S.prob[0].K, KE) + kDrainBlocks);
+    const long long cost_l = (ceil_div(gb.prob[0].K, KE) + kDrainBlocks) * (gb.prob[0].wide ? 2 : 1);
+    const long long cost_s = (ceil_div(gb.prob[M].K, KE) + kDrainBlocks) * (gb.prob[M].wide ? 2 : 1);
+    schedule_two_class(gb, grid / 2, n_long, cost_l, units - n_long, cost_s);
     if ((rc = timed("gemm_bwd", s, [&] { return launch_gemm_mixed(gb, grid, s); }))) return rc;
   }
   return MLS_OK;
@@ -808,7 +839,7 @@ extern "C" int mls_head_pairwise(const mls_problem* p, const void* const* H, con
   const int KE = 128 / pl.elt;
   for (int m = 0; m < p->M; ++m) {
     if (encode(&ep.mapH[m], H[m], pl.elt, p->d[m], p->T, p->d[m], KE, kHeadBM) ||
-        encode(&ep.mapW[m], W[m], pl.elt, p->d[m], p->V, p->d[m], KE, kEvalBHalf))
+        encode(&ep.mapW[m], W[m], pl.elt, p->d[m], p->V, p->d[m], KE, eval_tile_cols(p->M) / 2))
       return MLS_ERR_CUDA;
     ep.nk[m] = static_cast<int>(ceil_div(p->d[m], KE));
   }

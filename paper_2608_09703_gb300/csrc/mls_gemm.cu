@@ -11,8 +11,10 @@
 // CTA pairs (clusters of 2) own 256x256 output tiles: each CTA loads the 128
 // rows of A and the 128 rows of B that are its half, the even CTA issues
 // 256x256xK pair MMAs (cta_group::2) and each CTA drains its 128 accumulator
-// rows.  Persistent pairs walk a list of tiles over up to four problems (one
-// per sub-model):
+// rows.  Persistent pairs walk a list of units over up to eight problems (dW
+// and dH of each sub-model); a unit is one output tile, or for a wide problem
+// two adjacent column tiles that share each stage's A tile and use both TMEM
+// accumulators (no epilogue overlap, so only long reductions are made wide):
 //   warp 4    TMA producer (each CTA its own halves; both CTAs' loads complete
 //             on the even CTA's barrier, which expects the bytes of both)
 //   warp 5    MMA issuer (even CTA)
@@ -42,7 +44,16 @@ struct GemmSmem {
   static __device__ __forceinline__ uint32_t drain(uint32_t b) {
     return b + kBar + 8u * (2 * kGemmStages + 4);
   }
-  static constexpr uint32_t kTmemSlot = kBar + 8u * (2 * kGemmStages + 5);
+  // Wide units: stage s holds A | B0 | B1 at s * kWideStage, over the memory of
+  // the plain stages; wfull / wempty are its barriers.
+  static constexpr uint32_t kWideStage = kGemmABytes + 2 * kGemmBBytes;
+  static __device__ __forceinline__ uint32_t wfull(uint32_t b, int s) {
+    return b + kBar + 8u * (2 * kGemmStages + 5 + s);
+  }
+  static __device__ __forceinline__ uint32_t wempty(uint32_t b, int s) {
+    return b + kBar + 8u * (2 * kGemmStages + 5 + kGemmWideStages + s);
+  }
+  static constexpr uint32_t kTmemSlot = kBar + 8u * (2 * kGemmStages + 5 + 2 * kGemmWideStages);
   static constexpr uint32_t kAbort = kTmemSlot + 4;
   static constexpr uint32_t kEnd = kAbort + 4;
   // kEpiSoftmax output staging: per epilogue warp two 32 x 32 fp32 chunks
@@ -52,6 +63,9 @@ struct GemmSmem {
   static constexpr uint32_t kStaging = (kEnd + 1023u) & ~1023u;
 };
 static_assert(GemmSmem::kEnd + 1024 <= kGemmSmem, "gemm shared memory map overflows");
+static_assert(kGemmWideStages * GemmSmem::kWideStage <= GemmSmem::kBar,
+              "wide stages must fit in the plain stages' memory");
+static_assert(GemmSmem::kWideStage % 1024 == 0, "wide stages must stay 1024-byte aligned");
 static_assert(GemmSmem::kStaging + kGemmEpiWarps * 2 * GemmSmem::kChunk + 1023 <= kGemmSmem,
               "gemm output staging overflows");
 
@@ -59,12 +73,12 @@ constexpr uint32_t kTmemCols = 512;
 constexpr uint64_t kDrainNs = 100000000ull;
 constexpr int kPairM = 2 * kGemmBM;  // output rows of a pair tile
 
-struct TileCoord {
-  int prob, tm, tn;
+struct UnitCoord {
+  int prob, tm, tn, nt;  // problem, tile row, first tile column, tiles (1 or 2)
 };
 
-// The j-th tile of this pair, or -1 when it has no more.
-__device__ __forceinline__ int pair_tile(const GemmParams& p, int pair, int npairs, int j) {
+// The j-th unit of this pair, or -1 when it has no more.
+__device__ __forceinline__ int pair_unit(const GemmParams& p, int pair, int npairs, int j) {
   if (!p.two_class) {
     const int t = pair + j * npairs;
     return t < p.total_tiles ? t : -1;
@@ -88,46 +102,79 @@ __device__ __forceinline__ bool a_mn_of(const GemmProblem& pr) {
   return kAMode == 2 ? pr.a_mn != 0 : kAMode == 1;
 }
 
-__device__ __forceinline__ TileCoord decode_tile(const GemmParams& p, int t) {
-  int i = 0;
-  while (i + 1 < p.nprob && t >= p.prob[i + 1].tile_begin) ++i;
-  const int local = t - p.prob[i].tile_begin;
-  if (p.prob[i].m_fast) return {i, local % p.prob[i].tiles_m, local / p.prob[i].tiles_m};
-  return {i, local / p.prob[i].tiles_n, local % p.prob[i].tiles_n};
+// Wide units exist only in the launch that mixes problems (launch_gemm_mixed).
+template <int kAMode>
+__device__ __forceinline__ bool wide_of(const GemmProblem& pr) {
+  return kAMode == 2 && pr.wide != 0;
 }
 
-// This CTA's loads: its 128 rows of A and its 128 rows of B for every k-block.
+template <int kAMode>
+__device__ __forceinline__ UnitCoord decode_unit(const GemmParams& p, int u) {
+  int i = 0;
+  while (i + 1 < p.nprob && u >= p.prob[i + 1].tile_begin) ++i;
+  const GemmProblem& pr = p.prob[i];
+  const int local = u - pr.tile_begin;
+  if (pr.m_fast) return {i, local % pr.tiles_m, local / pr.tiles_m, 1};
+  if (wide_of<kAMode>(pr)) {
+    const int un = (pr.tiles_n + 1) >> 1;
+    const int tn = (local % un) * 2;
+    return {i, local / un, tn, pr.tiles_n - tn < 2 ? 1 : 2};
+  }
+  return {i, local / pr.tiles_n, local % pr.tiles_n, 1};
+}
+
+// This CTA's loads: its 128 rows of A and its 128 rows of B (of both column
+// tiles in a wide unit) for every k-block.
 template <bool kTF32, int kAMode, bool kBMN>
 __device__ __forceinline__ void gemm_producer(const GemmParams& p, uint32_t base, uint32_t rank,
                                               volatile int* abort_flag) {
   constexpr int KE = kTF32 ? 32 : 64;  // elements per 128-byte row
   constexpr uint32_t kBox = KE * 128;  // bytes of one MN-major box {KE, KE}
   const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
-  int stage = 0;
+  // plain ring (kGemmStages) and wide ring (kGemmWideStages) over the same memory
+  int stage = 0, wstage = 0;
   uint32_t phase = 0, filled = 0, lastpar = 0;
+  uint32_t wphase = 0, wfilled = 0, wlastpar = 0;
+  int layout = -1;  // ring the stages were last filled in: 0 plain, 1 wide
   bool ok = true;
-  int t;
-  for (int j = 0; ok && (t = pair_tile(p, pair, npairs, j)) >= 0; ++j) {
-    const TileCoord tc = decode_tile(p, t);
-    const GemmProblem& pr = p.prob[tc.prob];
-    MLS_CHECK(p.status, t < p.total_tiles && tc.prob < p.nprob && pr.a_map < kGemmMaxProblems &&
-                            static_cast<long long>(tc.tm) * kPairM < pr.Mrows &&
-                            static_cast<long long>(tc.tn) * kGemmBN < pr.Ncols);
+  int u;
+  for (int j = 0; ok && (u = pair_unit(p, pair, npairs, j)) >= 0; ++j) {
+    const UnitCoord uc = decode_unit<kAMode>(p, u);
+    const GemmProblem& pr = p.prob[uc.prob];
+    MLS_CHECK(p.status, u < p.total_tiles && uc.prob < p.nprob && pr.a_map < kGemmMaxProblems &&
+                            static_cast<long long>(uc.tm) * kPairM < pr.Mrows &&
+                            static_cast<long long>(uc.tn + uc.nt - 1) * kGemmBN < pr.Ncols);
     const bool amn = a_mn_of<kAMode>(pr);
+    const bool wide = wide_of<kAMode>(pr);
+    // Before one ring's memory is refilled in the other layout, every stage
+    // filled in the old layout must have been consumed by the MMAs.
+    if (layout == (wide ? 0 : 1)) {
+      for (int s = 0; ok && s < (wide ? kGemmStages : kGemmWideStages); ++s) {
+        const uint32_t f = wide ? filled : wfilled, lp = wide ? lastpar : wlastpar;
+        if ((f >> s) & 1u)
+          ok = mbar_wait(wide ? GemmSmem::empty(base, s) : GemmSmem::wempty(base, s), (lp >> s) & 1u,
+                         abort_flag, p.status);
+      }
+      if (!ok) break;
+    }
+    layout = wide ? 1 : 0;
     const CUtensorMap* ma = &p.mapA[pr.a_map];
     const CUtensorMap* mb = &p.mapB[pr.b_map];
     const int nkb = (pr.K + KE - 1) / KE;
-    const int m0 = pr.a_m0 + tc.tm * kPairM + static_cast<int>(rank) * kGemmBM;
-    const int n0 = pr.b_n0 + tc.tn * kGemmBN + static_cast<int>(rank) * kGemmBHalf;
+    const int m0 = pr.a_m0 + uc.tm * kPairM + static_cast<int>(rank) * kGemmBM;
+    const int n0 = pr.b_n0 + uc.tn * kGemmBN + static_cast<int>(rank) * kGemmBHalf;
     for (int kb = 0; kb < nkb; ++kb) {
-      if (!mbar_wait(GemmSmem::empty(base, stage), phase ^ 1u, abort_flag, p.status)) {
+      const uint32_t empty_bar = wide ? GemmSmem::wempty(base, wstage) : GemmSmem::empty(base, stage);
+      if (!mbar_wait(empty_bar, (wide ? wphase : phase) ^ 1u, abort_flag, p.status)) {
         ok = false;
         break;
       }
-      const uint32_t fb = map_to_rank(GemmSmem::full(base, stage), 0);
-      if (rank == 0) mbar_arrive_expect_tx(GemmSmem::full(base, stage), 2 * (kGemmABytes + kGemmBBytes));
-      const uint32_t sa = base + GemmSmem::kA + stage * kGemmABytes;
-      const uint32_t sb = base + GemmSmem::kB + stage * kGemmBBytes;
+      const uint32_t full_bar = wide ? GemmSmem::wfull(base, wstage) : GemmSmem::full(base, stage);
+      const uint32_t fb = map_to_rank(full_bar, 0);
+      if (rank == 0)
+        mbar_arrive_expect_tx(full_bar, 2 * (kGemmABytes + static_cast<uint32_t>(uc.nt) * kGemmBBytes));
+      const uint32_t sa = wide ? base + wstage * GemmSmem::kWideStage : base + GemmSmem::kA + stage * kGemmABytes;
+      const uint32_t sb = wide ? sa + kGemmABytes : base + GemmSmem::kB + stage * kGemmBBytes;
       const int ka = pr.a_k0 + kb * KE, kbb = pr.b_k0 + kb * KE;
       if (amn) {
 #pragma unroll
@@ -135,34 +182,52 @@ __device__ __forceinline__ void gemm_producer(const GemmParams& p, uint32_t base
       } else {
         tma_load_2d_pair(sa, ma, fb, ka, m0);
       }
-      if (kBMN) {
+      for (int t = 0; t < uc.nt; ++t) {
+        const uint32_t sbt = sb + static_cast<uint32_t>(t) * kGemmBBytes;
+        const int n0t = n0 + t * kGemmBN;
+        if (kBMN) {
 #pragma unroll
-        for (int q = 0; q < kGemmBHalf / KE; ++q)
-          tma_load_2d_pair(sb + q * kBox, mb, fb, n0 + q * KE, kbb);
-      } else {
-        tma_load_2d_pair(sb, mb, fb, kbb, n0);
+          for (int q = 0; q < kGemmBHalf / KE; ++q) tma_load_2d_pair(sbt + q * kBox, mb, fb, n0t + q * KE, kbb);
+        } else {
+          tma_load_2d_pair(sbt, mb, fb, kbb, n0t);
+        }
       }
-      filled |= 1u << stage;
-      lastpar = (lastpar & ~(1u << stage)) | (phase << stage);
-      if (++stage == kGemmStages) {
-        stage = 0;
-        phase ^= 1u;
+      if (wide) {
+        wfilled |= 1u << wstage;
+        wlastpar = (wlastpar & ~(1u << wstage)) | (wphase << wstage);
+        if (++wstage == kGemmWideStages) {
+          wstage = 0;
+          wphase ^= 1u;
+        }
+      } else {
+        filled |= 1u << stage;
+        lastpar = (lastpar & ~(1u << stage)) | (phase << stage);
+        if (++stage == kGemmStages) {
+          stage = 0;
+          phase ^= 1u;
+        }
       }
     }
   }
-  if (!ok && filled) {
+  if (!ok && (filled | wfilled)) {
     // Loads already issued must land before this CTA's shared memory goes away.
     // The even CTA can watch its barriers; the odd CTA's loads are counted on
     // the even CTA's barriers, so it waits out a bound no TMA load approaches.
     if (rank == 0) {
       for (int s = 0; s < kGemmStages; ++s)
-        if ((filled >> s) & 1u) mbar_wait_drain(GemmSmem::full(base, s), (lastpar >> s) & 1u, kDrainNs, p.status);
+        if ((filled >> s) & 1u)
+          mbar_wait_drain(GemmSmem::full(base, s), (lastpar >> s) & 1u, kDrainNs, p.status);
+      for (int s = 0; s < kGemmWideStages; ++s)
+        if ((wfilled >> s) & 1u)
+          mbar_wait_drain(GemmSmem::wfull(base, s), (wlastpar >> s) & 1u, kDrainNs, p.status);
     } else {
       spin_ns(kDrainNs);
     }
   }
 }
 
+// Tile i of this pair (counted over its units) accumulates in TMEM
+// accumulator i & 1, whose (i >> 1)-th use it is.
 template <bool kTF32, int kAMode, bool kBMN>
 __device__ __forceinline__ void gemm_mma(const GemmParams& p, uint32_t base, uint32_t tmem,
                                          volatile int* abort_flag) {
@@ -174,43 +239,63 @@ __device__ __forceinline__ void gemm_mma(const GemmParams& p, uint32_t base, uin
   constexpr uint32_t kStepMN = ((32u / (kTF32 ? 4u : 2u)) * 128u) >> 4;
   constexpr uint16_t kBoth = 0x3;
   const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
-  int stage = 0;
-  uint32_t phase = 0, acc = 0, acc_par = 0;
+  int stage = 0, wstage = 0;
+  uint32_t phase = 0, wphase = 0, tiles = 0;
   bool ok = true;
-  int t;
-  for (int j = 0; ok && (t = pair_tile(p, pair, npairs, j)) >= 0; ++j) {
-    const TileCoord tc = decode_tile(p, t);
-    const int nkb = (p.prob[tc.prob].K + KE - 1) / KE;
-    const bool amn = a_mn_of<kAMode>(p.prob[tc.prob]);
+  int u;
+  for (int j = 0; ok && (u = pair_unit(p, pair, npairs, j)) >= 0; ++j) {
+    const UnitCoord uc = decode_unit<kAMode>(p, u);
+    const GemmProblem& pr = p.prob[uc.prob];
+    const int nkb = (pr.K + KE - 1) / KE;
+    const bool amn = a_mn_of<kAMode>(pr);
+    const bool wide = wide_of<kAMode>(pr);
     const uint32_t idesc = make_idesc(kPairM, kGemmBN, kTF32, amn, kBMN);
-    if (!mbar_wait(GemmSmem::acce(base, acc), acc_par ^ 1u, abort_flag, p.status)) {
-      ok = false;
-      break;
+    for (int t = 0; ok && t < uc.nt; ++t) {
+      const uint32_t i = tiles + static_cast<uint32_t>(t);
+      ok = mbar_wait(GemmSmem::acce(base, i & 1u), ((i >> 1) & 1u) ^ 1u, abort_flag, p.status);
     }
+    if (!ok) break;
     tc_fence_after();
-    const uint32_t d = tmem + acc * kGemmBN;
+    const uint32_t d0 = tmem + (tiles & 1u) * kGemmBN, d1 = tmem + ((tiles + 1u) & 1u) * kGemmBN;
     for (int kb = 0; kb < nkb; ++kb) {
-      if (!mbar_wait(GemmSmem::full(base, stage), phase, abort_flag, p.status)) {
+      const uint32_t full_bar = wide ? GemmSmem::wfull(base, wstage) : GemmSmem::full(base, stage);
+      if (!mbar_wait(full_bar, wide ? wphase : phase, abort_flag, p.status)) {
         ok = false;
         break;
       }
       tc_fence_after();
-      const uint64_t ad = make_sdesc(base + GemmSmem::kA + stage * kGemmABytes, amn ? kBox : 16u);
-      const uint64_t bd = make_sdesc(base + GemmSmem::kB + stage * kGemmBBytes, kBMN ? kBox : 16u);
+      const uint32_t sa = wide ? base + wstage * GemmSmem::kWideStage : base + GemmSmem::kA + stage * kGemmABytes;
+      const uint32_t sb = wide ? sa + kGemmABytes : base + GemmSmem::kB + stage * kGemmBBytes;
+      const uint64_t ad = make_sdesc(sa, amn ? kBox : 16u);
+      const uint64_t bd = make_sdesc(sb, kBMN ? kBox : 16u);
 #pragma unroll
       for (int kk = 0; kk < 4; ++kk)
-        mma_issue_pair<kTF32>(d, ad + kk * (amn ? kStepMN : kStepK),
+        mma_issue_pair<kTF32>(d0, ad + kk * (amn ? kStepMN : kStepK),
                               bd + kk * (kBMN ? kStepMN : kStepK), idesc, (kb | kk) != 0);
-      mma_commit_pair(GemmSmem::empty(base, stage), kBoth);
-      if (++stage == kGemmStages) {
-        stage = 0;
-        phase ^= 1u;
+      if (uc.nt == 2) {
+        const uint64_t bd1 = make_sdesc(sb + kGemmBBytes, kBMN ? kBox : 16u);  // second column tile
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk)
+          mma_issue_pair<kTF32>(d1, ad + kk * (amn ? kStepMN : kStepK),
+                                bd1 + kk * (kBMN ? kStepMN : kStepK), idesc, (kb | kk) != 0);
+      }
+      if (wide) {
+        mma_commit_pair(GemmSmem::wempty(base, wstage), kBoth);
+        if (++wstage == kGemmWideStages) {
+          wstage = 0;
+          wphase ^= 1u;
+        }
+      } else {
+        mma_commit_pair(GemmSmem::empty(base, stage), kBoth);
+        if (++stage == kGemmStages) {
+          stage = 0;
+          phase ^= 1u;
+        }
       }
     }
     if (!ok) break;
-    mma_commit_pair(GemmSmem::accf(base, acc), kBoth);
-    acc ^= 1u;
-    if (acc == 0) acc_par ^= 1u;
+    for (int t = 0; t < uc.nt; ++t) mma_commit_pair(GemmSmem::accf(base, (tiles + t) & 1u), kBoth);
+    tiles += static_cast<uint32_t>(uc.nt);
   }
   mma_commit_pair(GemmSmem::drain(base), 0x1);
   mbar_wait_drain(GemmSmem::drain(base), 0, kDrainNs, p.status);
@@ -334,63 +419,69 @@ __device__ __noinline__ void epilogue_stats(const GemmProblem& pr, const CUtenso
 // kStats: the launch may hold problems with a statistics epilogue (only the
 // verify step's logits GEMM); without it epilogue_stats is not in the kernel,
 // which keeps the training GEMMs at 64 registers instead of 119.
-template <bool kStats>
+template <int kAMode, bool kStats>
 __device__ __forceinline__ void gemm_epilogue(const GemmParams& p, uint32_t base, uint32_t tmem,
                                               uint32_t rank, int warp, int lane,
                                               volatile int* abort_flag) {
   const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
-  uint32_t acc = 0, acc_par = 0, stores = 0;
+  uint32_t tiles = 0, stores = 0;
   const uint32_t tl = tmem + (static_cast<uint32_t>(warp * 32) << 16);
   const uint32_t stage = base + GemmSmem::kStaging + static_cast<uint32_t>(warp) * 2 * GemmSmem::kChunk;
-  int t;
-  for (int j = 0; (t = pair_tile(p, pair, npairs, j)) >= 0; ++j) {
-    const TileCoord tc = decode_tile(p, t);
-    const GemmProblem& pr = p.prob[tc.prob];
-    const bool ok = mbar_wait(GemmSmem::accf(base, acc), acc_par, abort_flag, p.status);
-    if (!__all_sync(0xffffffffu, ok)) break;
-    tc_fence_after();
-    const long long row = static_cast<long long>(tc.tm) * kPairM + rank * kGemmBM + warp * 32 + lane;
-    const bool row_ok = row < pr.Mrows;
-    float v[32];
-    if (kStats && pr.epi != kEpiPlain) {
-      const int row0 = tc.tm * kPairM + static_cast<int>(rank) * kGemmBM + warp * 32;
-      epilogue_stats(pr, &p.mapC[tc.prob], stage, stores, tl + acc * kGemmBN, tc.tn, row, row_ok,
-                     row0, lane);
-    } else {
-    float* crow = pr.C + (row_ok ? row : 0) * pr.ldc;
+  bool aborted = false;
+  int u;
+  for (int j = 0; !aborted && (u = pair_unit(p, pair, npairs, j)) >= 0; ++j) {
+    const UnitCoord uc = decode_unit<kAMode>(p, u);
+    const GemmProblem& pr = p.prob[uc.prob];
+    for (int t = 0; t < uc.nt; ++t, ++tiles) {
+      const uint32_t acc = tiles & 1u;
+      const int tn = uc.tn + t;
+      const bool ok = mbar_wait(GemmSmem::accf(base, acc), (tiles >> 1) & 1u, abort_flag, p.status);
+      if (!__all_sync(0xffffffffu, ok)) {
+        aborted = true;
+        break;
+      }
+      tc_fence_after();
+      const long long row = static_cast<long long>(uc.tm) * kPairM + rank * kGemmBM + warp * 32 + lane;
+      const bool row_ok = row < pr.Mrows;
+      float v[32];
+      if (kStats && pr.epi != kEpiPlain) {
+        const int row0 = uc.tm * kPairM + static_cast<int>(rank) * kGemmBM + warp * 32;
+        epilogue_stats(pr, &p.mapC[uc.prob], stage, stores, tl + acc * kGemmBN, tn, row, row_ok,
+                       row0, lane);
+      } else {
+        float* crow = pr.C + (row_ok ? row : 0) * pr.ldc;
 #pragma unroll 1
-    for (int c = 0; c < kGemmBN / 32; ++c) {
-      tmem_ld32(tl + acc * kGemmBN + c * 32, v);
-      const int col = tc.tn * kGemmBN + c * 32;
-      if (row_ok && col < pr.Ncols) {
-        float* dst = crow + col;
-        if (col + 32 <= pr.Ncols) {
-          float4* d4 = reinterpret_cast<float4*>(dst);
+        for (int c = 0; c < kGemmBN / 32; ++c) {
+          tmem_ld32(tl + acc * kGemmBN + c * 32, v);
+          const int col = tn * kGemmBN + c * 32;
+          if (row_ok && col < pr.Ncols) {
+            float* dst = crow + col;
+            if (col + 32 <= pr.Ncols) {
+              float4* d4 = reinterpret_cast<float4*>(dst);
 #pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            float4 o = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
-            if (pr.accumulate) {
-              const float4 c4 = d4[i];
-              o.x += c4.x;
-              o.y += c4.y;
-              o.z += c4.z;
-              o.w += c4.w;
+              for (int i = 0; i < 8; ++i) {
+                float4 o = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+                if (pr.accumulate) {
+                  const float4 c4 = d4[i];
+                  o.x += c4.x;
+                  o.y += c4.y;
+                  o.z += c4.z;
+                  o.w += c4.w;
+                }
+                d4[i] = o;
+              }
+            } else {
+#pragma unroll
+              for (int i = 0; i < 32; ++i)
+                if (col + i < pr.Ncols) dst[i] = pr.accumulate ? dst[i] + v[i] : v[i];
             }
-            d4[i] = o;
           }
-        } else {
-#pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if (col + i < pr.Ncols) dst[i] = pr.accumulate ? dst[i] + v[i] : v[i];
         }
       }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_remote(map_to_rank(GemmSmem::acce(base, acc), 0));
     }
-    }
-    tc_fence_before();
-    __syncwarp();
-    if (lane == 0) mbar_arrive_remote(map_to_rank(GemmSmem::acce(base, acc), 0));
-    acc ^= 1u;
-    if (acc == 0) acc_par ^= 1u;
   }
   if (stores && lane == 0) bulk_wait_all();  // staging must outlive the stores reading it
 }
@@ -412,6 +503,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     for (int s = 0; s < kGemmStages; ++s) {
       mbar_init(GemmSmem::full(base, s), 1);
       mbar_init(GemmSmem::empty(base, s), 1);
+    }
+    for (int s = 0; s < kGemmWideStages; ++s) {
+      mbar_init(GemmSmem::wfull(base, s), 1);
+      mbar_init(GemmSmem::wempty(base, s), 1);
     }
     for (uint32_t a = 0; a < 2; ++a) {
       mbar_init(GemmSmem::accf(base, a), 1);
@@ -441,7 +536,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     if (lane == 0 && rank == 0) gemm_mma<kTF32, kAMode, kBMN>(p, base, tmem, abort_flag);
     __syncwarp();
   } else {
-    gemm_epilogue<kStats>(p, base, tmem, rank, warp, lane, abort_flag);
+    gemm_epilogue<kAMode, kStats>(p, base, tmem, rank, warp, lane, abort_flag);
   }
 
   tc_fence_before();

@@ -101,6 +101,8 @@ constexpr int kGemmBM = 128;       // rows of A (and of C) per CTA
 constexpr int kGemmBN = 256;       // columns of C per pair tile
 constexpr int kGemmBHalf = 128;    // rows of B per CTA
 constexpr int kGemmStages = 6;
+// Wide units (GemmProblem::wide): stages of A | B0 | B1 over the same memory.
+constexpr int kGemmWideStages = 4;
 constexpr int kGemmEpiWarps = 4;
 constexpr int kGemmThreads = (kGemmEpiWarps + 2) * 32;
 constexpr uint32_t kGemmABytes = kGemmBM * 128;
@@ -117,7 +119,8 @@ struct GemmProblem {
   long long ldc;
   int accumulate;                // C += A*B if 1, C = A*B if 0
   int tiles_n;                   // ceil(Ncols / kGemmBN)
-  int tile_begin;                // first linear pair tile (256 x kGemmBN) of this problem
+  int tile_begin;                // first unit of this problem in the launch's unit numbering
+                                 // (a unit is one pair tile of 256 x kGemmBN, or two if wide)
   int tiles_m;                   // ceil(Mrows / 256); used when m_fast is set
   int m_fast;                    // 1: consecutive tiles walk M first (pairs running at the
                                  //    same time share the B tile, read once from HBM)
@@ -131,6 +134,12 @@ struct GemmProblem {
   float* stats;
   long long stats_ld;
   int a_mn;                      // A is MN-major (read by launches that take the layout per problem)
+  // Wide units (launch_gemm_mixed only): a unit is two adjacent column tiles
+  // (tn, tn + 1) that share the A tile of each stage and take both TMEM
+  // accumulators, which halves the A operand's shared-memory traffic per FLOP
+  // and the number of passes over B.  The accumulators are then not double
+  // buffered, so this suits problems with a long reduction.
+  int wide;
 };
 enum GemmEpilogue { kEpiPlain = 0, kEpiSoftmax = 1, kEpiArgmax = 2 };
 
@@ -142,7 +151,7 @@ struct GemmParams {
   CUtensorMap mapC[kGemmMaxProblems];  // kEpiSoftmax: C fp32 [Mrows, Ncols], box {32, 32}, 128B swizzle
   int nprob;
   GemmProblem prob[kGemmMaxProblems];
-  int total_tiles;
+  int total_tiles;               // units of the launch (pair tiles, or pairs of them if wide)
   int* status;
   // Schedule.  two_class == 0: pair p takes tiles p, p + npairs, ...
   // two_class == 1: tiles [0, n_long) are the long ones (larger K) and go
@@ -158,31 +167,39 @@ struct GemmParams {
 
 // ------------------------------------------------------------------ pairwise evaluation
 // Forward-only evaluation metrics between sub-models.  A CTA pair owns 256
-// tokens; for every 128-column vocabulary tile it computes the logit tiles of
-// all M <= 4 sub-models into TMEM at once (M x 128 columns) and accumulates,
-// for every ordered pair (s, j), D_sj = sum_v exp(z_s[v] - max_s) (z_s[v] - z_j[v]).
-constexpr int kEvalBN = 128;     // vocabulary columns per tile
-constexpr int kEvalBHalf = 64;   // rows of W per CTA
-constexpr int kEvalStages = 9;
-constexpr uint32_t kEvalABytes = kHeadBM * 128;
-constexpr uint32_t kEvalBBytes = kEvalBHalf * 128;
+// tokens; for every vocabulary tile it computes the logit tiles of all M <= 4
+// sub-models into TMEM at once (M tiles of eval_tile_cols(M) columns, at most
+// the 512 TMEM columns) and accumulates, for every ordered pair (s, j),
+// D_sj = sum_v exp(z_s[v] - max_s) (z_s[v] - z_j[v]).  The tile is as wide as
+// TMEM allows: operand bytes per FLOP fall as the tile widens, and operand
+// delivery from L2 bounds this kernel.
+__host__ __device__ constexpr int eval_tile_cols(int M) { return M <= 2 ? 256 : (M == 3 ? 160 : 128); }
+constexpr uint32_t kEvalABytes = kHeadBM * 128;                    // A stage: 128 token rows
+__host__ __device__ constexpr uint32_t eval_b_bytes(int M) { return eval_tile_cols(M) / 2 * 128; }
+// As many stages as fit in 216 KB (9, 8, 6 and 6 for M = 4, 3, 2, 1).
+constexpr uint32_t kEvalStageBudget = 216 * 1024;
+__host__ __device__ constexpr int eval_stages(int M) {
+  return static_cast<int>(kEvalStageBudget / (kEvalABytes + eval_b_bytes(M)));
+}
+__host__ __device__ constexpr uint32_t eval_smem(int M) {
+  return static_cast<uint32_t>(eval_stages(M)) * (kEvalABytes + eval_b_bytes(M)) + 1024 + 1024;
+}
 // per token and split: max_s (4), sum_s (4), argmax_s (4), D_sj for j != s (4 x 3)
 constexpr int kEvalFields = 24;
 constexpr uint32_t kEvalXchg = kEvalFields * kHeadBM * 4;
 // The half-merge exchange is only used after the main loop, when the operand
 // stages are idle, so it shares their memory.
-constexpr uint32_t kEvalSmem = kEvalStages * (kEvalABytes + kEvalBBytes) + 1024 + 1024;
-static_assert(kEvalXchg <= kEvalStages * (kEvalABytes + kEvalBBytes), "exchange fits in the stages");
+static_assert(kEvalXchg <= 6 * (kEvalABytes + eval_b_bytes(2)), "exchange fits in the stages");
 
 struct EvalParams {
   CUtensorMap mapH[kMaxModels];  // H_m [T, d_m], box {128 B of K, kHeadBM rows}
-  CUtensorMap mapW[kMaxModels];  // W_m [V, d_m], box {128 B of K, kEvalBHalf rows}
+  CUtensorMap mapW[kMaxModels];  // W_m [V, d_m], box {128 B of K, eval_tile_cols(M) / 2 rows}
   int M;
   int order[kMaxModels];         // units of a vocabulary tile, widest sub-model first
   int pos[kMaxModels];           // pos[order[i]] = i
   int nk[kMaxModels];
   int ntt;                       // token tiles of 256 (one per CTA pair)
-  int nvt;                       // vocabulary tiles of kEvalBN
+  int nvt;                       // vocabulary tiles of eval_tile_cols(M) columns
   int S;                         // CTA pairs per token tile
   int band;                      // token tiles per band of the launch order (band_unit)
   long long T, V;
@@ -275,7 +292,15 @@ struct MergeParams {
   int* status;
 };
 
-constexpr int kMergeTokens = 8;        // tokens per merge block (8 warps share them)
+// Warps of a merge block per group of 8 tokens: 4 partial slots per warp, as
+// few warps as cover the partials (8 warps for more than 8 partials).
+__host__ __device__ inline int merge_warps_per_octet(int nparts) {
+  return nparts <= 4 ? 1 : nparts <= 8 ? 2 : 8;
+}
+// Tokens per merge block (8 warps): 8 octets of one warp, 4 of two, or 1 of eight.
+__host__ __device__ inline int merge_tokens_per_block(int nparts) {
+  return 8 * (8 / merge_warps_per_octet(nparts));
+}
 constexpr int kEvalMergeTokens = 128;  // tokens per evaluation-merge block: one thread per token
 
 // Launchers (return the cudaError_t of the launch).

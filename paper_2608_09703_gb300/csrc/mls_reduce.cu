@@ -1,7 +1,7 @@
 // Row reductions of the forward pass, the token count of the backward and an
 // fp32 transpose (used only for fp32 inputs, whose tf32 GEMMs read K-major copies).
 //
-// merge_kernel: a block of 8 warps combines, for 8 tokens, the partial row
+// merge_kernel: a block of 8 warps combines, for 8 to 64 tokens, the partial row
 // states that the head kernel wrote per (CTA, half tile) into
 //   lse_m    = logsumexp(z_m)            CE_m = lse_m - z_m[y]
 //   lset_m   = logsumexp(z_m / tau)
@@ -35,35 +35,43 @@ __device__ __forceinline__ double block_sum_double(double v, double* sh) {
   return s;  // valid in thread 0
 }
 
-// A block of 8 warps merges kMergeTokens = 8 consecutive tokens.  Lane l of
-// warp w takes token t0 + (l mod 8) and the partials k = 4 w + l / 8,
-// k + 32, ...: the 8 lanes of a group read 32 consecutive bytes (one sector)
-// of each (partial, field, sub-model).  Round 1 takes every sub-model's row
-// maximum, round 2 its sums.  The partials of a token are combined in a fixed
-// order (within a lane, across the 4 lane groups by butterflies, across the 8
-// warps in warp order), so results are deterministic.
+// A block of 8 warps merges 8 * (8 / kWT) consecutive tokens: each group of 8
+// tokens (an octet) takes kWT warps, i.e. 4 * kWT partial slots per token.
+// Lane l of warp w takes token (l mod 8) of octet w / kWT and the partials
+// k = 4 (w mod kWT) + l / 8, k + 4 kWT, ...: the 8 lanes of a group read 32
+// consecutive bytes (one sector) of each (partial, field, sub-model).  kWT
+// follows the number of partials (merge_warps_per_octet), so few partials
+// do not leave most lanes idle.  Round 1 takes every sub-model's row maximum,
+// round 2 its sums.  The partials of a token are combined in a fixed order
+// (within a lane, across the 4 lane groups by butterflies, across the octet's
+// warps in warp order), and the block's share of the loss over its octets in
+// octet order, so results are deterministic.
 constexpr int kMergeWarps = 8;
-static_assert(kMergeTokens == 8, "a lane group covers 8 tokens");
 
+template <int kWT>
 __global__ void __launch_bounds__(kMergeWarps * 32, 4) merge_kernel(const __grid_constant__ MergeParams p) {
-  __shared__ float sh_f[4][kMergeWarps][kMaxModels][kMergeTokens];  // max, then s1, st, acc, zy
-  __shared__ int sh_am[kMergeWarps][kMaxModels][kMergeTokens];
+  constexpr int kOct = kMergeWarps / kWT;  // token octets per block
+  constexpr int kSlots = 4 * kWT;          // partial slots per token
+  __shared__ float sh_f[4][kMergeWarps][kMaxModels][8];  // max, then s1, st, acc, zy
+  __shared__ int sh_am[kMergeWarps][kMaxModels][8];
+  __shared__ double sh_c[kOct][2];
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int j = lane & 7, grp = lane >> 3;  // token within the block, partial group
+  const int j = lane & 7, grp = lane >> 3;  // token within the octet, partial group
+  const int oct = w / kWT, ww = w % kWT;    // octet, warp within the octet
   const long long T = p.T;
-  const long long t = static_cast<long long>(blockIdx.x) * kMergeTokens + j;
+  const long long t = (static_cast<long long>(blockIdx.x) * kOct + oct) * 8 + j;
   const bool live = t < T;
   const long long MT = static_cast<long long>(p.M) * T;
   const long long PS = kPartFields * MT;  // stride between partials
   const int tc = p.teacher;
-  const int k0 = 4 * w + grp;
+  const int k0 = 4 * ww + grp;
 
   // ---- round 1: row maxima of every sub-model
   float mx[kMaxModels];
 #pragma unroll
   for (int m = 0; m < kMaxModels; ++m) mx[m] = -INFINITY;
   if (live)
-    for (int k = k0; k < p.nparts; k += 32) {
+    for (int k = k0; k < p.nparts; k += kSlots) {
 #pragma unroll
       for (int m = 0; m < kMaxModels; ++m)
         if (m < p.M) mx[m] = fmaxf(mx[m], p.part[k * PS + kPartMax * MT + m * T + t]);
@@ -78,7 +86,7 @@ __global__ void __launch_bounds__(kMergeWarps * 32, 4) merge_kernel(const __grid
 #pragma unroll
   for (int m = 0; m < kMaxModels; ++m) {
     float v = -INFINITY;
-    for (int ww = 0; ww < kMergeWarps; ++ww) v = fmaxf(v, sh_f[0][ww][m][j]);
+    for (int q = 0; q < kWT; ++q) v = fmaxf(v, sh_f[0][oct * kWT + q][m][j]);
     mx[m] = v;
   }
   float mT = -INFINITY;
@@ -100,7 +108,7 @@ __global__ void __launch_bounds__(kMergeWarps * 32, 4) merge_kernel(const __grid
     am[m] = INT_MAX;
   }
   if (live)
-    for (int k = k0; k < p.nparts; k += 32) {
+    for (int k = k0; k < p.nparts; k += kSlots) {
       const float mtk = p.part[k * PS + kPartMax * MT + static_cast<long long>(tc) * T + t];
 #pragma unroll
       for (int m = 0; m < kMaxModels; ++m) {
@@ -146,21 +154,21 @@ __global__ void __launch_bounds__(kMergeWarps * 32, 4) merge_kernel(const __grid
     }
   }
   __syncthreads();
-  if (w != 0) return;
 
-  // ---- warp 0, lanes 0-7: one token each
+  // ---- the octet's first warp, lanes 0-7: one token each
   double contrib = 0.0, cnt = 0.0;
-  if (lane < kMergeTokens && live) {
+  if (ww == 0 && lane < 8 && live) {
 #pragma unroll
     for (int m = 0; m < kMaxModels; ++m) {
       float a = 0.f, b = 0.f, c = 0.f, d = 0.f;
       int e = INT_MAX;
-      for (int ww = 0; ww < kMergeWarps; ++ww) {
-        a += sh_f[0][ww][m][j];
-        b += sh_f[1][ww][m][j];
-        c += sh_f[2][ww][m][j];
-        d += sh_f[3][ww][m][j];
-        e = min(e, sh_am[ww][m][j]);
+      for (int q = 0; q < kWT; ++q) {
+        const int wq = oct * kWT + q;
+        a += sh_f[0][wq][m][j];
+        b += sh_f[1][wq][m][j];
+        c += sh_f[2][wq][m][j];
+        d += sh_f[3][wq][m][j];
+        e = min(e, sh_am[wq][m][j]);
       }
       s1[m] = a;
       st[m] = b;
@@ -225,15 +233,26 @@ __global__ void __launch_bounds__(kMergeWarps * 32, 4) merge_kernel(const __grid
     }
     cnt = valid ? 1.0 : 0.0;
   }
-  // the block's share, over its tokens in a fixed order
+  // the block's share, over its tokens in a fixed order: within each octet,
+  // then over the octets
 #pragma unroll
   for (int o = 4; o > 0; o >>= 1) {
     contrib += __shfl_down_sync(0xffffffffu, contrib, o);
     cnt += __shfl_down_sync(0xffffffffu, cnt, o);
   }
-  if (lane == 0) {
-    p.block_sum[blockIdx.x] = contrib;
-    p.block_cnt[blockIdx.x] = static_cast<long long>(cnt);
+  if (ww == 0 && lane == 0) {
+    sh_c[oct][0] = contrib;
+    sh_c[oct][1] = cnt;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double bs = 0.0, bc = 0.0;
+    for (int o = 0; o < kOct; ++o) {
+      bs += sh_c[o][0];
+      bc += sh_c[o][1];
+    }
+    p.block_sum[blockIdx.x] = bs;
+    p.block_cnt[blockIdx.x] = static_cast<long long>(bc);
   }
 }
 
@@ -302,7 +321,11 @@ cudaError_t launch_transpose(const float* in, long long rows, long long cols, lo
 
 cudaError_t launch_merge(const MergeParams& p, int blocks, cudaStream_t s) {
   if (blocks <= 0) return cudaSuccess;
-  merge_kernel<<<blocks, kMergeWarps * 32, 0, s>>>(p);
+  switch (merge_warps_per_octet(p.nparts)) {
+    case 1: merge_kernel<1><<<blocks, kMergeWarps * 32, 0, s>>>(p); break;
+    case 2: merge_kernel<2><<<blocks, kMergeWarps * 32, 0, s>>>(p); break;
+    default: merge_kernel<8><<<blocks, kMergeWarps * 32, 0, s>>>(p); break;
+  }
   return cudaGetLastError();
 }
 

@@ -61,6 +61,30 @@ def test_vocab_groups_match(vocab_group):
     full_parity(wl, H, W, y, vocab_group=vocab_group)
 
 
+@pytest.mark.parametrize("T,V,vocab_group", [(520, 35000, 0), (300, 66000, 33024)])
+def test_wide_dh_units(T, V, vocab_group):
+    """A vocabulary group of at least 512 k-blocks that writes dH, with an even
+    number of column tiles in every sub-model, runs dH in wide units (two
+    column tiles sharing each A tile of G): widths of 2 and 4 column tiles (the
+    last ragged) over 3 or 2 token tiles (the last ragged).  In the second
+    case there are two groups of 33024 and 32976 columns: the first runs wide,
+    the second plain, accumulating into dH."""
+    wl = synth.Workload("wide", T=T, d=(320, 1008), V=V, tau=1.3, alpha=0.5, w_sigma=0.05)
+    H, W, y = synth.make_inputs(wl, seed=13)
+    full_parity(wl, H, W, y, vocab_group=vocab_group, argmax=False)
+
+
+@pytest.mark.parametrize("V", [700, 1800, 9000])
+def test_merge_partial_counts(V):
+    """1000 tokens (4 token tiles, the last ragged) against 3, 8 and 36
+    vocabulary tiles: about 3, 8 and 19 partial states per token, so the merge
+    runs with one, two and eight warps per group of 8 tokens."""
+    wl = synth.Workload("merge", T=1000, d=(64, 128), V=V, tau=0.9, alpha=0.5, w_sigma=0.05)
+    H, W, y = synth.make_inputs(wl, seed=14)
+    y[[5, 999]] = -1
+    full_parity(wl, H, W, y)
+
+
 def test_edge_shapes():
     # V below one vocabulary tile, a single token, a single sub-model
     for wl in (synth.Workload("v100", T=130, d=(32, 64), V=100, w_sigma=0.1),
