@@ -4,19 +4,20 @@
 //   KL(p_s || p_j) = E_{p_s}[z_s - z_j] - (lse_s - lse_j)
 // with p = softmax(z) at temperature 1.  The logits are never stored.
 //
-// A CTA pair owns 256 tokens and a strided set of 128-column vocabulary tiles.
-// For each tile the even CTA issues pair MMAs (cta_group::2, 256x128xK) for
-// every sub-model into its own 128 TMEM columns, so all M <= 4 logit tiles are
-// resident together; the epilogue then reads them chunk by chunk and
-// accumulates, per sub-model s, the running max, sum_v exp(z_s - max_s) and
+// A CTA pair owns 256 tokens and a strided set of vocabulary tiles of
+// N = eval_tile_cols(M) columns (256, 256, 160, 128 for M = 1..4: M tiles of
+// N columns fill TMEM).  For each tile the even CTA issues pair MMAs
+// (cta_group::2, 256 x N x K) for every sub-model into its own N TMEM columns,
+// widest sub-model first (unit position q holds sub-model order[q]), so all M
+// logit tiles are resident together; the epilogue then accumulates, per
+// sub-model s, the running max, sum_v exp(z_s - max_s) and
 // D_sj = sum_v exp(z_s - max_s) (z_s - z_j) for every j != s (the difference
 // is taken element by element, so nearly equal sub-models lose no precision).
-// TMEM is a ring of four 128-column slots: the u-th unit (one sub-model of one
-// vocabulary tile, widest sub-model first) goes to slot u mod 4 and waits only
-// for that slot's previous tile to be drained, so at M = 3 the next tile's
-// widest unit runs during the epilogue (M = 2: full double buffering; M = 4:
-// one tile at a time).  Roles: warp 8 TMA producer, warp 9 MMA issuer (even
-// CTA), warps 0-7 epilogue (one thread per token and 64 columns).
+// The epilogue first copies the widest sub-model's tile into registers and
+// releases its TMEM columns, so the next tile's widest (longest) MMAs run
+// while the rest of the epilogue reads the other sub-models from TMEM.
+// Roles: warp 8 TMA producer, warp 9 MMA issuer (even CTA), warps 0-7
+// epilogue (one thread per token and N / 2 columns).
 #include <climits>
 
 #include "mls_device.cuh"
@@ -25,31 +26,35 @@
 namespace mls {
 namespace {
 
+template <int kM>
 struct EvalSmem {
+  static constexpr int kN = eval_tile_cols(kM);
+  static constexpr int kStages = eval_stages(kM);
+  static constexpr uint32_t kBBytes = eval_b_bytes(kM);
   static constexpr uint32_t kA = 0;
-  static constexpr uint32_t kB = kEvalStages * kEvalABytes;
+  static constexpr uint32_t kB = kStages * kEvalABytes;
   static constexpr uint32_t kX = kA;  // half-merge exchange, after the main loop only
-  static constexpr uint32_t kBar = kB + kEvalStages * kEvalBBytes;
+  static constexpr uint32_t kBar = kB + kStages * kBBytes;
   static __device__ __forceinline__ uint32_t full(uint32_t b, int s) { return b + kBar + 8u * s; }
   static __device__ __forceinline__ uint32_t empty(uint32_t b, int s) {
-    return b + kBar + 8u * (kEvalStages + s);
+    return b + kBar + 8u * (kStages + s);
   }
-  // tile j's accumulators are complete: accf(j mod 4); slot s drained: slote(s)
+  // tile j's accumulators are complete: accf(j & 1)
   static __device__ __forceinline__ uint32_t accf(uint32_t b, int j) {
-    return b + kBar + 8u * (2 * kEvalStages + (j & 3));
+    return b + kBar + 8u * (2 * kStages + (j & 1));
   }
-  static __device__ __forceinline__ uint32_t slote(uint32_t b, int s) {
-    return b + kBar + 8u * (2 * kEvalStages + 4 + s);
-  }
-  static __device__ __forceinline__ uint32_t drain(uint32_t b) {
-    return b + kBar + 8u * (2 * kEvalStages + 8);
-  }
-  static constexpr uint32_t kTmemSlot = kBar + 8u * (2 * kEvalStages + 9);
+  // the widest sub-model's columns (free0) / all other columns (free1) were read
+  static __device__ __forceinline__ uint32_t free0(uint32_t b) { return b + kBar + 8u * (2 * kStages + 2); }
+  static __device__ __forceinline__ uint32_t free1(uint32_t b) { return b + kBar + 8u * (2 * kStages + 3); }
+  static __device__ __forceinline__ uint32_t drain(uint32_t b) { return b + kBar + 8u * (2 * kStages + 4); }
+  static constexpr uint32_t kTmemSlot = kBar + 8u * (2 * kStages + 5);
   static constexpr uint32_t kAbort = kTmemSlot + 4;
   static constexpr uint32_t kEnd = kAbort + 4;
+  static_assert(kEnd + 1024 <= eval_smem(kM), "eval shared memory map overflows");
+  static_assert(kM * kN <= 512, "all sub-models' tiles must fit in TMEM");
+  static_assert(kBBytes % 1024 == 0, "B stages must stay 1024-byte aligned");
+  static_assert((kN / 2) % 16 == 0, "an epilogue thread reads 16-column chunks");
 };
-static_assert(EvalSmem::kEnd + 1024 <= kEvalSmem, "eval shared memory map overflows");
-static_assert(kMaxModels * kEvalBN <= 512, "all sub-models' tiles must fit in TMEM");
 
 constexpr uint32_t kTmemCols = 512;
 constexpr uint64_t kDrainNs = 100000000ull;
@@ -58,29 +63,30 @@ constexpr int kD = 12;  // field offset of D_sj
 // field index of D_sj (j != s) in the partial state
 __host__ __device__ constexpr int dfield(int s, int j) { return kD + s * 3 + (j < s ? j : j - 1); }
 
-template <bool kTF32>
+template <bool kTF32, int kM>
 __device__ __forceinline__ void eval_producer(const EvalParams& p, uint32_t base, int row0,
                                               uint32_t rank, int split, volatile int* abort_flag) {
+  using Sm = EvalSmem<kM>;
   constexpr int KE = kTF32 ? 32 : 64;
   int stage = 0;
   uint32_t phase = 0, filled = 0, lastpar = 0;
   bool ok = true;
   for (int vt = split; ok && vt < p.nvt; vt += p.S) {
-    for (int i = 0; ok && i < p.M; ++i) {
+    for (int i = 0; ok && i < kM; ++i) {
       const int m = p.order[i];
       for (int kb = 0; kb < p.nk[m]; ++kb) {
-        if (!mbar_wait(EvalSmem::empty(base, stage), phase ^ 1u, abort_flag, p.status)) {
+        if (!mbar_wait(Sm::empty(base, stage), phase ^ 1u, abort_flag, p.status)) {
           ok = false;
           break;
         }
-        if (rank == 0) mbar_arrive_expect_tx(EvalSmem::full(base, stage), 2 * (kEvalABytes + kEvalBBytes));
-        const uint32_t fb = map_to_rank(EvalSmem::full(base, stage), 0);
-        tma_load_2d_pair(base + EvalSmem::kA + stage * kEvalABytes, &p.mapH[m], fb, kb * KE, row0);
-        tma_load_2d_pair(base + EvalSmem::kB + stage * kEvalBBytes, &p.mapW[m], fb, kb * KE,
-                         vt * kEvalBN + static_cast<int>(rank) * kEvalBHalf);
+        if (rank == 0) mbar_arrive_expect_tx(Sm::full(base, stage), 2 * (kEvalABytes + Sm::kBBytes));
+        const uint32_t fb = map_to_rank(Sm::full(base, stage), 0);
+        tma_load_2d_pair(base + Sm::kA + stage * kEvalABytes, &p.mapH[m], fb, kb * KE, row0);
+        tma_load_2d_pair(base + Sm::kB + stage * Sm::kBBytes, &p.mapW[m], fb, kb * KE,
+                         vt * Sm::kN + static_cast<int>(rank) * (Sm::kN / 2));
         filled |= 1u << stage;
         lastpar = (lastpar & ~(1u << stage)) | (phase << stage);
-        if (++stage == kEvalStages) {
+        if (++stage == Sm::kStages) {
           stage = 0;
           phase ^= 1u;
         }
@@ -89,102 +95,103 @@ __device__ __forceinline__ void eval_producer(const EvalParams& p, uint32_t base
   }
   if (!ok && filled) {
     if (rank == 0) {
-      for (int s = 0; s < kEvalStages; ++s)
-        if ((filled >> s) & 1u) mbar_wait_drain(EvalSmem::full(base, s), (lastpar >> s) & 1u, kDrainNs, p.status);
+      for (int s = 0; s < Sm::kStages; ++s)
+        if ((filled >> s) & 1u) mbar_wait_drain(Sm::full(base, s), (lastpar >> s) & 1u, kDrainNs, p.status);
     } else {
       spin_ns(kDrainNs);
     }
   }
 }
 
-template <bool kTF32>
+// Unit q of tile j goes to TMEM columns [q N, (q + 1) N).  The widest unit
+// (q = 0) of tile j waits for the epilogue to have copied tile j - 1's columns
+// of q = 0 (free0); the others wait for it to have finished tile j - 1 (free1).
+template <bool kTF32, int kM>
 __device__ __forceinline__ void eval_mma(const EvalParams& p, uint32_t base, uint32_t tmem,
                                          int split, volatile int* abort_flag) {
-  constexpr uint32_t kIdesc = make_idesc(2 * kHeadBM, kEvalBN, kTF32, false, false);
+  using Sm = EvalSmem<kM>;
+  constexpr uint32_t kIdesc = make_idesc(2 * kHeadBM, Sm::kN, kTF32, false, false);
   int stage = 0;
   uint32_t phase = 0;
-  int uses[4] = {0, 0, 0, 0};  // times each TMEM slot has been handed out
   bool ok = true;
   int j = 0;
   for (int vt = split; ok && vt < p.nvt; vt += p.S, ++j) {
-    for (int i = 0; ok && i < p.M; ++i) {
+    for (int i = 0; ok && i < kM; ++i) {
       const int m = p.order[i];
-      const int slot = (j * p.M + i) & 3;
-      // the n-th use of a slot waits for its (n-1)-th drain
-      if (uses[slot] > 0 &&
-          !mbar_wait(EvalSmem::slote(base, slot), static_cast<uint32_t>(uses[slot] - 1) & 1u,
+      if (j > 0 && i <= 1 &&
+          !mbar_wait(i == 0 ? Sm::free0(base) : Sm::free1(base), static_cast<uint32_t>(j - 1) & 1u,
                      abort_flag, p.status)) {
         ok = false;
         break;
       }
-      ++uses[slot];
       tc_fence_after();
-      const uint32_t d = tmem + static_cast<uint32_t>(slot) * kEvalBN;
+      const uint32_t d = tmem + static_cast<uint32_t>(i * Sm::kN);
       for (int kb = 0; kb < p.nk[m]; ++kb) {
-        if (!mbar_wait(EvalSmem::full(base, stage), phase, abort_flag, p.status)) {
+        if (!mbar_wait(Sm::full(base, stage), phase, abort_flag, p.status)) {
           ok = false;
           break;
         }
         tc_fence_after();
-        const uint64_t ad = make_sdesc(base + EvalSmem::kA + stage * kEvalABytes, 16);
-        const uint64_t bd = make_sdesc(base + EvalSmem::kB + stage * kEvalBBytes, 16);
+        const uint64_t ad = make_sdesc(base + Sm::kA + stage * kEvalABytes, 16);
+        const uint64_t bd = make_sdesc(base + Sm::kB + stage * Sm::kBBytes, 16);
 #pragma unroll
         for (int kk = 0; kk < 4; ++kk)
           mma_issue_pair<kTF32>(d, ad + 2u * kk, bd + 2u * kk, kIdesc, (kb | kk) != 0);
-        mma_commit_pair(EvalSmem::empty(base, stage), 0x3);
-        if (++stage == kEvalStages) {
+        mma_commit_pair(Sm::empty(base, stage), 0x3);
+        if (++stage == Sm::kStages) {
           stage = 0;
           phase ^= 1u;
         }
       }
     }
     if (!ok) break;
-    mma_commit_pair(EvalSmem::accf(base, j), 0x3);
+    mma_commit_pair(Sm::accf(base, j), 0x3);
   }
-  mma_commit_pair(EvalSmem::drain(base), 0x1);
-  mbar_wait_drain(EvalSmem::drain(base), 0, kDrainNs, p.status);
+  mma_commit_pair(Sm::drain(base), 0x1);
+  mbar_wait_drain(Sm::drain(base), 0, kDrainNs, p.status);
 }
 
+// Running state of one thread, indexed by unit position q (sub-model order[q]).
+template <int kM>
 struct EvalState {
-  float m[kMaxModels], s[kMaxModels];
-  int am[kMaxModels];
-  float d[kMaxModels][kMaxModels];
+  float m[kM], s[kM];
+  int am[kM];
+  float d[kM][kM];
 };
 
-// One 32-column chunk of every sub-model's tile (z[s][i] = z_s at column col0 + i).
-template <bool kMasked>
-__device__ __forceinline__ void eval_chunk(const float (&z)[kMaxModels][32], int M, int nvalid,
-                                           long long col0, float L1, EvalState& st) {
+// 16 columns of every unit's tile: z[q][i] = z_{order[q]} at column col0 + i.
+template <int kM, bool kMasked>
+__device__ __forceinline__ void eval_chunk(const float (&z)[kM][16], int nvalid, long long col0,
+                                           float L1, EvalState<kM>& st) {
 #pragma unroll
-  for (int s = 0; s < kMaxModels; ++s) {
-    if (s >= M) continue;
+  for (int q = 0; q < kM; ++q) {
     float cmax = -INFINITY;
     int carg = 0;
 #pragma unroll
-    for (int i = 0; i < 32; ++i) {
+    for (int i = 0; i < 16; ++i) {
       const bool ok = !kMasked || i < nvalid;
-      if (ok && z[s][i] > cmax) {
-        cmax = z[s][i];
+      if (ok && z[q][i] > cmax) {
+        cmax = z[q][i];
         carg = i;
       }
     }
-    if (cmax > st.m[s]) {
-      st.am[s] = static_cast<int>(col0 + carg);
-      const float f = st.m[s] == -INFINITY ? 0.f : fast_exp2((st.m[s] - cmax) * L1);
-      st.s[s] *= f;
+    if (cmax > st.m[q]) {
+      st.am[q] = static_cast<int>(col0 + carg);
+      const float f = st.m[q] == -INFINITY ? 0.f : fast_exp2((st.m[q] - cmax) * L1);
+      st.s[q] *= f;
 #pragma unroll
-      for (int j = 0; j < kMaxModels; ++j) st.d[s][j] *= f;
-      st.m[s] = cmax;
+      for (int r = 0; r < kM; ++r) st.d[q][r] *= f;
+      st.m[q] = cmax;
     }
-    const float nb = -st.m[s] * L1;
+    const float nb = -st.m[q] * L1;
 #pragma unroll
-    for (int i = 0; i < 32; ++i) {
+    for (int i = 0; i < 16; ++i) {
       const bool ok = !kMasked || i < nvalid;
-      const float e = ok ? fast_exp2(fmaf(z[s][i], L1, nb)) : 0.f;
-      st.s[s] += e;
+      const float e = ok ? fast_exp2(fmaf(z[q][i], L1, nb)) : 0.f;
+      st.s[q] += e;
 #pragma unroll
-      for (int j = 0; j < kMaxModels; ++j)
-        if (j != s && j < M) st.d[s][j] = fmaf(e, z[s][i] - z[j][i], st.d[s][j]);
+      for (int r = 0; r < kM; ++r)
+        if (r != q) st.d[q][r] = fmaf(e, z[q][i] - z[r][i], st.d[q][r]);
     }
   }
 }
@@ -193,94 +200,109 @@ __device__ __forceinline__ float scale_to(float from, float to, float L1) {
   return from == -INFINITY ? 0.f : fast_exp2((from - to) * L1);
 }
 
+// Frees TMEM columns for the MMA issuer: every epilogue warp of both CTAs
+// arrives on the even CTA's barrier once its reads have completed.
+__device__ __forceinline__ void eval_release(uint32_t bar, int lane) {
+  tc_fence_before();
+  __syncwarp();
+  if (lane == 0) mbar_arrive_remote(map_to_rank(bar, 0));
+}
+
+template <int kM>
 __device__ __forceinline__ void eval_epilogue(const EvalParams& p, uint32_t base, uint32_t tmem,
                                               float* xchg, int row_base, int split, int warp,
                                               int lane, volatile int* abort_flag) {
+  using Sm = EvalSmem<kM>;
+  constexpr int kHalf = Sm::kN / 2;  // columns per thread
+  constexpr int kChunks = kHalf / 16;
   const int quad = warp & 3, half = warp >> 2;
   const int r = quad * 32 + lane;
   const long long row = static_cast<long long>(row_base) + r;
-  const uint32_t tl = tmem + (static_cast<uint32_t>(quad * 32) << 16) + static_cast<uint32_t>(half * 64);
-  const int M = p.M;
+  const uint32_t tl = tmem + (static_cast<uint32_t>(quad * 32) << 16) + static_cast<uint32_t>(half * kHalf);
   const float L1 = p.L1;
-  EvalState st;
+  EvalState<kM> st;
 #pragma unroll
-  for (int s = 0; s < kMaxModels; ++s) {
-    st.m[s] = -INFINITY;
-    st.s[s] = 0.f;
-    st.am[s] = 0;
+  for (int q = 0; q < kM; ++q) {
+    st.m[q] = -INFINITY;
+    st.s[q] = 0.f;
+    st.am[q] = 0;
 #pragma unroll
-    for (int j = 0; j < kMaxModels; ++j) st.d[s][j] = 0.f;
+    for (int j = 0; j < kM; ++j) st.d[q][j] = 0.f;
   }
-  float z[kMaxModels][32];
   int j = 0;
   for (int vt = split; vt < p.nvt; vt += p.S, ++j) {
-    const bool ok = mbar_wait(EvalSmem::accf(base, j), static_cast<uint32_t>(j >> 2) & 1u,
-                              abort_flag, p.status);
+    const bool ok = mbar_wait(Sm::accf(base, j), static_cast<uint32_t>(j >> 1) & 1u, abort_flag, p.status);
     if (!__all_sync(0xffffffffu, ok)) break;
     tc_fence_after();
+    // the widest unit's columns into registers, then its TMEM columns are free
+    float z0[kChunks][16];
 #pragma unroll
-    for (int c = 0; c < 2; ++c) {
-      const long long col0 = static_cast<long long>(vt) * kEvalBN + half * 64 + c * 32;
-      const int nvalid = static_cast<int>(max(0LL, min(32LL, p.V - col0)));
+    for (int c = 0; c < kChunks; ++c) tmem_ld16(tl + static_cast<uint32_t>(c * 16), z0[c]);
+    eval_release(Sm::free0(base), lane);
+#pragma unroll
+    for (int c = 0; c < kChunks; ++c) {
+      const long long col0 = static_cast<long long>(vt) * Sm::kN + half * kHalf + c * 16;
+      const int nvalid = static_cast<int>(max(0LL, min(16LL, p.V - col0)));
       if (nvalid == 0) continue;  // warp-uniform
+      float z[kM][16];
 #pragma unroll
-      for (int s = 0; s < kMaxModels; ++s)
-        if (s < M) {
-          const uint32_t slot = static_cast<uint32_t>(j * M + p.pos[s]) & 3u;
-          tmem_ld32(tl + slot * kEvalBN + static_cast<uint32_t>(c * 32), z[s]);
-        }
-      if (nvalid == 32)
-        eval_chunk<false>(z, M, 32, col0, L1, st);
+      for (int i = 0; i < 16; ++i) z[0][i] = z0[c][i];
+#pragma unroll
+      for (int q = 1; q < kM; ++q) tmem_ld16(tl + static_cast<uint32_t>(q * Sm::kN + c * 16), z[q]);
+      if (nvalid == 16)
+        eval_chunk<kM, false>(z, 16, col0, L1, st);
       else
-        eval_chunk<true>(z, M, nvalid, col0, L1, st);
+        eval_chunk<kM, true>(z, nvalid, col0, L1, st);
     }
-    tc_fence_before();
-    __syncwarp();
-    if (lane == 0)
-      for (int i = 0; i < M; ++i)
-        mbar_arrive_remote(map_to_rank(EvalSmem::slote(base, (j * M + i) & 3), 0));
+    eval_release(Sm::free1(base), lane);
   }
 
-  // the two column halves of a token combine through shared memory
+  // The two column halves of a token combine through shared memory; fields
+  // are indexed by sub-model (order[q]).
   auto X = [&](int f) -> float& { return xchg[f * kHeadBM + r]; };
   if (half == 1) {
 #pragma unroll
-    for (int s = 0; s < kMaxModels; ++s) {
-      X(s) = st.m[s];
-      X(4 + s) = st.s[s];
-      X(8 + s) = __int_as_float(st.am[s]);
+    for (int q = 0; q < kM; ++q) {
+      const int s = p.order[q];
+      X(s) = st.m[q];
+      X(4 + s) = st.s[q];
+      X(8 + s) = __int_as_float(st.am[q]);
 #pragma unroll
-      for (int j = 0; j < kMaxModels; ++j)
-        if (j != s) X(dfield(s, j)) = st.d[s][j];
+      for (int q2 = 0; q2 < kM; ++q2)
+        if (q2 != q) X(dfield(s, p.order[q2])) = st.d[q][q2];
     }
   }
   named_bar_sync(1, kHeadEpiWarps * 32);
   if (half == 1 || row >= p.T) return;
   float* P = p.part + static_cast<long long>(split) * kEvalFields * p.T + row;
 #pragma unroll
-  for (int s = 0; s < kMaxModels; ++s) {
-    if (s >= M) continue;
-    const float m1 = X(s), mm = fmaxf(st.m[s], m1);
-    const float fa = scale_to(st.m[s], mm, L1), fb = scale_to(m1, mm, L1);
+  for (int q = 0; q < kM; ++q) {
+    const int s = p.order[q];
+    const float m1 = X(s), mm = fmaxf(st.m[q], m1);
+    const float fa = scale_to(st.m[q], mm, L1), fb = scale_to(m1, mm, L1);
     const int a1 = __float_as_int(X(8 + s));
     P[s * p.T] = mm;
-    P[(4 + s) * p.T] = st.s[s] * fa + X(4 + s) * fb;
-    P[(8 + s) * p.T] = __int_as_float(m1 > st.m[s] ? a1 : (st.m[s] > m1 ? st.am[s] : min(st.am[s], a1)));
+    P[(4 + s) * p.T] = st.s[q] * fa + X(4 + s) * fb;
+    P[(8 + s) * p.T] = __int_as_float(m1 > st.m[q] ? a1 : (st.m[q] > m1 ? st.am[q] : min(st.am[q], a1)));
 #pragma unroll
-    for (int j = 0; j < kMaxModels; ++j)
-      if (j != s && j < M) P[dfield(s, j) * p.T] = st.d[s][j] * fa + X(dfield(s, j)) * fb;
+    for (int q2 = 0; q2 < kM; ++q2)
+      if (q2 != q) {
+        const int f = dfield(s, p.order[q2]);
+        P[f * p.T] = st.d[q][q2] * fa + X(f) * fb;
+      }
   }
 }
 
-template <bool kTF32>
+template <bool kTF32, int kM>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kHeadThreads, 1)
     eval_kernel(const __grid_constant__ EvalParams p) {
+  using Sm = EvalSmem<kM>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t* gbase = smem_raw + (base - raw);
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(gbase + EvalSmem::kAbort);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + EvalSmem::kTmemSlot);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(gbase + Sm::kAbort);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + Sm::kTmemSlot);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = cluster_ctarank();
   int tt, split;
@@ -289,23 +311,22 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kHeadThreads, 1)
 
   if (threadIdx.x == 0) {
     *abort_flag = 0;
-    for (int s = 0; s < kEvalStages; ++s) {
-      mbar_init(EvalSmem::full(base, s), 1);
-      mbar_init(EvalSmem::empty(base, s), 1);
+    for (int s = 0; s < Sm::kStages; ++s) {
+      mbar_init(Sm::full(base, s), 1);
+      mbar_init(Sm::empty(base, s), 1);
     }
-    for (int q = 0; q < 4; ++q) {
-      mbar_init(EvalSmem::accf(base, q), 1);
-      mbar_init(EvalSmem::slote(base, q), 2 * kHeadEpiWarps);
-    }
-    mbar_init(EvalSmem::drain(base), 1);
+    for (int q = 0; q < 2; ++q) mbar_init(Sm::accf(base, q), 1);
+    mbar_init(Sm::free0(base), 2 * kHeadEpiWarps);
+    mbar_init(Sm::free1(base), 2 * kHeadEpiWarps);
+    mbar_init(Sm::drain(base), 1);
     fence_barrier_init();
   }
   if (warp == kHeadEpiWarps + 1) {
-    tmem_alloc_pair(base + EvalSmem::kTmemSlot, kTmemCols);
+    tmem_alloc_pair(base + Sm::kTmemSlot, kTmemCols);
     tmem_relinquish_pair();
   }
   if (warp == kHeadEpiWarps && lane == 0) {
-    for (int m = 0; m < p.M; ++m) {
+    for (int m = 0; m < kM; ++m) {
       tma_prefetch_desc(&p.mapH[m]);
       tma_prefetch_desc(&p.mapW[m]);
     }
@@ -318,15 +339,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kHeadThreads, 1)
   if (warp >= kHeadEpiWarps) {
     regs_decrease<kHeadCtlRegs>();
     if (warp == kHeadEpiWarps) {
-      if (lane == 0) eval_producer<kTF32>(p, base, row_base, rank, split, abort_flag);
+      if (lane == 0) eval_producer<kTF32, kM>(p, base, row_base, rank, split, abort_flag);
     } else if (warp == kHeadEpiWarps + 1) {
-      if (lane == 0 && rank == 0) eval_mma<kTF32>(p, base, tmem, split, abort_flag);
+      if (lane == 0 && rank == 0) eval_mma<kTF32, kM>(p, base, tmem, split, abort_flag);
       __syncwarp();
     }
   } else {
     regs_increase<kHeadEpiRegs>();
-    eval_epilogue(p, base, tmem, reinterpret_cast<float*>(gbase + EvalSmem::kX), row_base, split,
-                  warp, lane, abort_flag);
+    eval_epilogue<kM>(p, base, tmem, reinterpret_cast<float*>(gbase + Sm::kX), row_base, split,
+                      warp, lane, abort_flag);
   }
 
   tc_fence_before();
@@ -436,14 +457,24 @@ __global__ void __launch_bounds__(kEvalFinalThreads)
 
 }  // namespace
 
+template <int kM>
+cudaError_t launch_eval_m(const EvalParams& p, bool tf32, int grid, cudaStream_t s) {
+  if (tf32)
+    eval_kernel<true, kM><<<grid, kHeadThreads, eval_smem(kM), s>>>(p);
+  else
+    eval_kernel<false, kM><<<grid, kHeadThreads, eval_smem(kM), s>>>(p);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_eval(const EvalParams& p, bool tf32, cudaStream_t s) {
   const int grid = 2 * p.ntt * p.S;
   if (grid <= 0) return cudaSuccess;
-  if (tf32)
-    eval_kernel<true><<<grid, kHeadThreads, kEvalSmem, s>>>(p);
-  else
-    eval_kernel<false><<<grid, kHeadThreads, kEvalSmem, s>>>(p);
-  return cudaGetLastError();
+  switch (p.M) {
+    case 1: return launch_eval_m<1>(p, tf32, grid, s);
+    case 2: return launch_eval_m<2>(p, tf32, grid, s);
+    case 3: return launch_eval_m<3>(p, tf32, grid, s);
+    default: return launch_eval_m<4>(p, tf32, grid, s);
+  }
 }
 
 cudaError_t launch_eval_merge(const EvalMergeParams& p, int blocks, cudaStream_t s) {
@@ -460,19 +491,25 @@ cudaError_t launch_eval_final(const double* block_acc, const long long* block_cn
 
 cudaError_t setup_eval_kernels() {
   cudaError_t e;
-#define MLS_SET(TF)                                                                           \
-  e = cudaFuncSetAttribute(eval_kernel<TF>, cudaFuncAttributeMaxDynamicSharedMemorySize,      \
-                           kEvalSmem);                                                        \
+#define MLS_SET(TF, M)                                                                        \
+  e = cudaFuncSetAttribute(eval_kernel<TF, M>, cudaFuncAttributeMaxDynamicSharedMemorySize,   \
+                           eval_smem(M));                                                     \
   if (e != cudaSuccess) return e;                                                             \
   {                                                                                           \
     cudaFuncAttributes fa;                                                                    \
-    e = cudaFuncGetAttributes(&fa, eval_kernel<TF>);                                          \
+    e = cudaFuncGetAttributes(&fa, eval_kernel<TF, M>);                                       \
     if (e != cudaSuccess) return e;                                                           \
     if (fa.maxThreadsPerBlock < kHeadThreads || fa.numRegs != kHeadLaunchRegs)                \
       return cudaErrorLaunchOutOfResources;                                                   \
   }
-  MLS_SET(true)
-  MLS_SET(false)
+  MLS_SET(true, 1)
+  MLS_SET(true, 2)
+  MLS_SET(true, 3)
+  MLS_SET(true, 4)
+  MLS_SET(false, 1)
+  MLS_SET(false, 2)
+  MLS_SET(false, 3)
+  MLS_SET(false, 4)
 #undef MLS_SET
   return cudaSuccess;
 }

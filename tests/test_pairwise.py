@@ -88,3 +88,22 @@ def test_pairwise_suite3_full_size_sampled():
     rng = np.random.default_rng(35)
     rows = np.unique(np.concatenate([rng.integers(0, wl.T, 8), [0, wl.T - 1]]))
     check(wl, H, W, y, rows=rows)
+
+
+def test_pairwise_single_model():
+    """M = 1: no pairs; the argmax and the (zero) KL matrix still come out."""
+    wl = synth.Workload("pw1", T=300, d=(96,), V=777, w_sigma=0.1)
+    H, W, y = synth.make_inputs(wl, seed=36)
+    kl, _, stats = check(wl, H, W, y)
+    assert np.abs(kl).max() == 0.0 and stats[1][0, 0] == 1.0
+
+
+@pytest.mark.parametrize("M", [2, 3, 4])
+def test_pairwise_many_tiles_per_pair(M):
+    """16 token tiles and a ragged vocabulary of 4999 columns: each CTA pair
+    walks several vocabulary tiles (256, 160 or 128 columns wide for M = 2, 3,
+    4), so the epilogue's early release of the widest sub-model's columns and
+    the accumulator barriers go through several phases."""
+    wl = synth.Workload("pwm", T=4096, d=(64, 192, 128, 320)[:M], V=4999, w_sigma=0.08)
+    H, W, y = synth.make_inputs(wl, seed=37 + M)
+    check(wl, H, W, y)
