@@ -109,7 +109,8 @@ long long ceil_div(long long a, long long b) { return (a + b - 1) / b; }
 struct Plan {
   int elt = 2;
   int ntt = 0, nvt = 0;
-  int band = 1;  // token tiles per band of the head and evaluation kernels' launch order
+  int band = 1;      // token tiles per band of the forward and evaluation launch order
+  int band_bwd = 1;  // the same for the backward head kernel
   // forward
   int S = 1, nparts = 0, merge_blocks = 0, eval_merge_blocks = 0;
   size_t off_part = 0, off_bsum = 0, off_bcnt = 0, fwd_bytes = 0;
@@ -154,12 +155,15 @@ int choose_splits(int ntt, long long tiles, int pairs) {
 // the band's tokens once per vocabulary tile, so a band's H is kept within a
 // share of L2 that stays resident while W streams past it.  Fewer token tiles
 // per band mean more passes over W (one per band); the bands are made equal.
-#ifndef MLS_HEAD_BAND_BYTES
-#define MLS_HEAD_BAND_BYTES (48ll << 20)
-#endif
-int choose_band(int ntt, long long h_bytes_per_tile) {
+// The backward streams its dL/dz stores through L2 as well, so its band's H
+// gets a smaller share (measured on the 3-level suite: 48 MB gave the
+// forward its least traffic at no cost in time; 32 MB, with the stores
+// marked evict-first, cut the backward's DRAM reads from 4.8 to 3.3 GB).
+constexpr long long kBandBytesFwd = 48ll << 20;
+constexpr long long kBandBytesBwd = 32ll << 20;
+int choose_band(int ntt, long long h_bytes_per_tile, long long budget) {
   if (ntt < 1) return 1;
-  long long band = MLS_HEAD_BAND_BYTES / (h_bytes_per_tile > 0 ? h_bytes_per_tile : 1);
+  long long band = budget / (h_bytes_per_tile > 0 ? h_bytes_per_tile : 1);
   if (band < 1) band = 1;
   if (band >= ntt) return ntt;
   const long long nbands = (ntt + band - 1) / band;
@@ -196,7 +200,8 @@ Plan make_plan(const mls_problem* p, int pairs) {
   pl.nparts = pl.S;
   long long sum_d = 0;
   for (int m = 0; m < p->M; ++m) sum_d += p->d[m];
-  pl.band = choose_band(pl.ntt, 2LL * kHeadBM * sum_d * pl.elt);
+  pl.band = choose_band(pl.ntt, 2LL * kHeadBM * sum_d * pl.elt, kBandBytesFwd);
+  pl.band_bwd = choose_band(pl.ntt, 2LL * kHeadBM * sum_d * pl.elt, kBandBytesBwd);
   pl.merge_blocks = static_cast<int>(ceil_div(T, merge_tokens_per_block(pl.nparts)));
   pl.eval_merge_blocks = static_cast<int>(ceil_div(T, kEvalMergeTokens));
   size_t o = 0;
@@ -547,7 +552,7 @@ extern "C" int mls_head_loss_bwd(const mls_problem* p, const void* const* H, con
     hp.vt_begin = static_cast<int>(g * tiles_per_group);
     hp.vt_end = static_cast<int>(ceil_div(c0 + gc, kHeadBN));
     hp.S = choose_splits(pl.ntt, hp.vt_end - hp.vt_begin, dev->head_pairs);
-    hp.band = pl.band;
+    hp.band = pl.band_bwd;
     hp.g_col0 = c0;
     if ((rc = timed("head_bwd", s, [&] { return launch_head_bwd(hp, tf32, p->tau == 1.0f, s); }))) return rc;
     if (tf32)

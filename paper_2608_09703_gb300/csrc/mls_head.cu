@@ -505,7 +505,9 @@ __device__ __forceinline__ void put_chunk(const GOut& o, int gcol, int ch, const
     fence_proxy_async_smem();
     __syncwarp();
     if (lane == 0) {
-      tma_store_2d(o.map, buf, gcol + ch * 32, o.row0);
+      // dL/dz is read back by the GEMMs only after the whole launch, so its
+      // lines are the first to go from L2, ahead of the band's H and W.
+      tma_store_2d_hint(o.map, buf, gcol + ch * 32, o.row0, l2_policy_evict_first());
       bulk_commit();
     }
     *o.count += 1;
