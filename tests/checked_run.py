@@ -33,6 +33,25 @@ def main(path):
     for m in range(wl.M):
         out[f"dH{m}"] = op.dH[m].cpu().numpy()
         out[f"dW{m}"] = op.dW[m].cpu().numpy()
+    # the backward GEMM's wide dH units (one group of 516 k-blocks, even
+    # column-tile counts), 8 partial states per token (two merge warps per 8
+    # tokens), and the pairwise metrics at M = 2 and M = 4 (their own tile
+    # widths)
+    for tag, wl2 in (("w", synth.Workload("chkw", T=1100, d=(320, 1008), V=33000, w_sigma=0.05)),
+                     ("m4", synth.Workload("chk4", T=2048, d=(64, 128, 64, 192), V=2000, w_sigma=0.1))):
+        H2, W2, y2 = synth.make_inputs(wl2, seed=75)
+        H2, W2, y2 = [h.to(dev) for h in H2], [w.to(dev) for w in W2], y2.to(dev).to(torch.int32)
+        op2 = B.HeadLoss(wl2.d, wl2.T, wl2.V, device=dev)
+        op2.forward(H2, W2, y2)
+        op2.backward(H2, W2, y2)
+        kl2, _, ps2 = op2.pairwise(H2, W2, y2)
+        torch.cuda.synchronize()
+        out[f"status_{tag}"] = np.array(B.mls_get_status())
+        out[f"{tag}_tok_loss"], out[f"{tag}_kl"], out[f"{tag}_ps"] = (
+            t.cpu().numpy() for t in (op2.tok_loss, kl2, ps2))
+        for m in range(wl2.M):
+            out[f"{tag}_dH{m}"] = op2.dH[m].cpu().numpy()
+            out[f"{tag}_dW{m}"] = op2.dW[m].cpu().numpy()
     # junction
     g = torch.Generator().manual_seed(72)
     o = torch.randn(130, 64, generator=g).to(torch.bfloat16).to(dev)
