@@ -107,3 +107,22 @@ def test_pairwise_many_tiles_per_pair(M):
     wl = synth.Workload("pwm", T=4096, d=(64, 192, 128, 320)[:M], V=4999, w_sigma=0.08)
     H, W, y = synth.make_inputs(wl, seed=37 + M)
     check(wl, H, W, y)
+
+
+def test_pairwise_fp32_three_models():
+    """fp32 inputs (tf32 products) at M = 3: 160-column tiles read with
+    32-element k-blocks, over a ragged vocabulary and two token tiles.  The
+    heads have the fp32 workload's scale (sigma 0.02): tf32 rounds each
+    product to ~2^-11, which the KL tolerance covers at logits of that size
+    (with sigma 0.1 the largest KL error reached 1.6e-3)."""
+    wl = synth.Workload("pwf", T=300, d=(32, 96, 64), V=1234, dtype="fp32", w_sigma=0.02)
+    H, W, y = synth.make_inputs(wl, seed=41)
+    check(wl, H, W, y)
+
+
+def test_pairwise_token_bands():
+    """The suite's widths over 24 token tiles: the evaluation kernel's pairs run
+    in 2 bands of 12 token tiles; every token compared with the oracle."""
+    wl = synth.Workload("pwb", T=6000, d=(1024, 2048, 3072), V=700, w_sigma=0.02)
+    H, W, y = synth.make_inputs(wl, seed=42)
+    check(wl, H, W, y)

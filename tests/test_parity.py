@@ -74,6 +74,18 @@ def test_wide_dh_units(T, V, vocab_group):
     full_parity(wl, H, W, y, vocab_group=vocab_group, argmax=False)
 
 
+def test_token_bands_full_parity():
+    """The suite's widths over 24 token tiles (the last ragged) and a small
+    vocabulary: the head kernels' pairs run in bands of token tiles (2 bands of
+    12 in the forward, 3 of 8 in the backward), every token and every
+    gradient entry compared with the oracle."""
+    wl = synth.Workload("bands", T=6000, d=(1024, 2048, 3072), V=700, tau=1.0, alpha=0.5,
+                        w_sigma=0.02)
+    H, W, y = synth.make_inputs(wl, seed=15)
+    y[[0, 3100, 5999]] = -1
+    full_parity(wl, H, W, y, argmax=False)
+
+
 @pytest.mark.parametrize("V", [700, 1800, 9000])
 def test_merge_partial_counts(V):
     """1000 tokens (4 token tiles, the last ragged) against 3, 8 and 36
