@@ -5,17 +5,20 @@
 // with p = softmax(z) at temperature 1.  The logits are never stored.
 //
 // A CTA pair owns 256 tokens and a strided set of vocabulary tiles of
-// N = eval_tile_cols(M) columns (256, 256, 160, 128 for M = 1..4: M tiles of
-// N columns fill TMEM).  For each tile the even CTA issues pair MMAs
-// (cta_group::2, 256 x N x K) for every sub-model into its own N TMEM columns,
-// widest sub-model first (unit position q holds sub-model order[q]), so all M
-// logit tiles are resident together; the epilogue then accumulates, per
-// sub-model s, the running max, sum_v exp(z_s - max_s) and
-// D_sj = sum_v exp(z_s - max_s) (z_s - z_j) for every j != s (the difference
-// is taken element by element, so nearly equal sub-models lose no precision).
-// The epilogue first copies the widest sub-model's tile into registers and
-// releases its TMEM columns, so the next tile's widest (longest) MMAs run
-// while the rest of the epilogue reads the other sub-models from TMEM.
+// N = eval_tile_cols(M) columns (256 for M <= 3, 128 for M = 4).  For each tile
+// the even CTA issues pair MMAs (cta_group::2, 256 x N x K) for every
+// sub-model, widest first (unit position q holds sub-model order[q]); the
+// epilogue accumulates, per sub-model s, the running max, sum_v exp(z_s - max_s)
+// and D_sj = sum_v exp(z_s - max_s) (z_s - z_j) for every j != s (the
+// difference is taken element by element, so nearly equal sub-models lose no
+// precision).  The epilogue first copies the widest sub-model's tile into
+// registers and releases its TMEM columns, so the next MMAs run while it reads
+// the other sub-models from TMEM.  Two TMEM schedules:
+//   - all resident (M = 1, 2, 4): unit q in columns [qN, (q+1)N), M N <= 512;
+//     the next tile's widest unit runs under the rest of the epilogue;
+//   - slots (M = 3): the two narrower units in two 256-column slots; the
+//     epilogue passes over them pair by pair and frees one slot before its
+//     last pass (eval_mma_slots, eval_slots_main).
 // Roles: warp 8 TMA producer, warp 9 MMA issuer (even CTA), warps 0-7
 // epilogue (one thread per token and N / 2 columns).
 #include <climits>
@@ -39,19 +42,29 @@ struct EvalSmem {
   static __device__ __forceinline__ uint32_t empty(uint32_t b, int s) {
     return b + kBar + 8u * (kStages + s);
   }
-  // tile j's accumulators are complete: accf(j & 1)
-  static __device__ __forceinline__ uint32_t accf(uint32_t b, int j) {
-    return b + kBar + 8u * (2 * kStages + (j & 1));
+  // eight barriers for the accumulators, used as below by each schedule
+  static __device__ __forceinline__ uint32_t tb(uint32_t b, int i) {
+    return b + kBar + 8u * (2 * kStages + i);
   }
+  // all-resident schedule (M != 3): tile j's accumulators are complete: accf(j & 1);
   // the widest sub-model's columns (free0) / all other columns (free1) were read
-  static __device__ __forceinline__ uint32_t free0(uint32_t b) { return b + kBar + 8u * (2 * kStages + 2); }
-  static __device__ __forceinline__ uint32_t free1(uint32_t b) { return b + kBar + 8u * (2 * kStages + 3); }
-  static __device__ __forceinline__ uint32_t drain(uint32_t b) { return b + kBar + 8u * (2 * kStages + 4); }
-  static constexpr uint32_t kTmemSlot = kBar + 8u * (2 * kStages + 5);
+  static __device__ __forceinline__ uint32_t accf(uint32_t b, int j) { return tb(b, j & 1); }
+  static __device__ __forceinline__ uint32_t free0(uint32_t b) { return tb(b, 2); }
+  static __device__ __forceinline__ uint32_t free1(uint32_t b) { return tb(b, 3); }
+  // slot schedule (M = 3): unit q of the tile is complete (q = 0, 1, 2); unit 0
+  // was copied out (copied); the first (pass_a) and second (pass_b) epilogue
+  // passes over the last unit are done
+  static __device__ __forceinline__ uint32_t unit_full(uint32_t b, int q) { return tb(b, q); }
+  static __device__ __forceinline__ uint32_t copied(uint32_t b) { return tb(b, 3); }
+  static __device__ __forceinline__ uint32_t pass_a(uint32_t b) { return tb(b, 4); }
+  static __device__ __forceinline__ uint32_t pass_b(uint32_t b) { return tb(b, 5); }
+  static __device__ __forceinline__ uint32_t drain(uint32_t b) { return tb(b, 7); }
+  static constexpr uint32_t kTmemSlot = kBar + 8u * (2 * kStages + 8);
   static constexpr uint32_t kAbort = kTmemSlot + 4;
   static constexpr uint32_t kEnd = kAbort + 4;
   static_assert(kEnd + 1024 <= eval_smem(kM), "eval shared memory map overflows");
-  static_assert(kM * kN <= 512, "all sub-models' tiles must fit in TMEM");
+  static_assert(eval_slotted(kM) ? 2 * kN <= 512 : kM * kN <= 512,
+                "the resident tiles must fit in TMEM");
   static_assert(kBBytes % 1024 == 0, "B stages must stay 1024-byte aligned");
   static_assert((kN / 2) % 16 == 0, "an epilogue thread reads 16-column chunks");
 };
@@ -151,6 +164,61 @@ __device__ __forceinline__ void eval_mma(const EvalParams& p, uint32_t base, uin
   mbar_wait_drain(Sm::drain(base), 0, kDrainNs, p.status);
 }
 
+// Slot schedule (M = 3).  Tile j's units go to two 256-column TMEM slots,
+// a_j = (j & 1) * 256 and b_j = 256 - a_j:
+//   unit 0 (widest) -> a_j, after the epilogue's first pass over tile j - 1's
+//                      last unit has freed a_j (= b_{j-1})         [pass_a]
+//   unit 1          -> b_j, after its second pass has freed b_j      [pass_b]
+//   unit 2          -> a_j, once unit 0 has been copied to registers [copied]
+// so unit 0 of the next tile, the longest, runs under the end of the epilogue.
+template <bool kTF32>
+__device__ __forceinline__ void eval_mma_slots(const EvalParams& p, uint32_t base, uint32_t tmem,
+                                               int split, volatile int* abort_flag) {
+  using Sm = EvalSmem<3>;
+  constexpr uint32_t kIdesc = make_idesc(2 * kHeadBM, Sm::kN, kTF32, false, false);
+  int stage = 0;
+  uint32_t phase = 0;
+  bool ok = true;
+  int j = 0;
+  for (int vt = split; ok && vt < p.nvt; vt += p.S, ++j) {
+    const uint32_t sa = static_cast<uint32_t>(j & 1) * Sm::kN, sb = Sm::kN - sa;
+    for (int i = 0; ok && i < 3; ++i) {
+      const int m = p.order[i];
+      const uint32_t prev = static_cast<uint32_t>(j - 1) & 1u;
+      bool go = true;
+      if (i == 0 && j > 0) go = mbar_wait(Sm::pass_a(base), prev, abort_flag, p.status);
+      if (i == 1 && j > 0) go = mbar_wait(Sm::pass_b(base), prev, abort_flag, p.status);
+      if (i == 2) go = mbar_wait(Sm::copied(base), static_cast<uint32_t>(j) & 1u, abort_flag, p.status);
+      if (!go) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t d = tmem + (i == 1 ? sb : sa);
+      for (int kb = 0; kb < p.nk[m]; ++kb) {
+        if (!mbar_wait(Sm::full(base, stage), phase, abort_flag, p.status)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint64_t ad = make_sdesc(base + Sm::kA + stage * kEvalABytes, 16);
+        const uint64_t bd = make_sdesc(base + Sm::kB + stage * Sm::kBBytes, 16);
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk)
+          mma_issue_pair<kTF32>(d, ad + 2u * kk, bd + 2u * kk, kIdesc, (kb | kk) != 0);
+        mma_commit_pair(Sm::empty(base, stage), 0x3);
+        if (++stage == Sm::kStages) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+      if (ok) mma_commit_pair(Sm::unit_full(base, i), 0x3);
+    }
+  }
+  mma_commit_pair(Sm::drain(base), 0x1);
+  mbar_wait_drain(Sm::drain(base), 0, kDrainNs, p.status);
+}
+
 // Running state of one thread, indexed by unit position q (sub-model order[q]).
 template <int kM>
 struct EvalState {
@@ -208,6 +276,154 @@ __device__ __forceinline__ void eval_release(uint32_t bar, int lane) {
   if (lane == 0) mbar_arrive_remote(map_to_rank(bar, 0));
 }
 
+// Online maximum and first argmax of unit q over a 16-column chunk; a new
+// maximum rescales the unit's sum and its D_q*.
+template <int kM, bool kMasked>
+__device__ __forceinline__ void eval_max(const float (&z)[16], int nvalid, long long col0,
+                                         float L1, EvalState<kM>& st, int q) {
+  float cmax = -INFINITY;
+  int carg = 0;
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    const bool ok = !kMasked || i < nvalid;
+    if (ok && z[i] > cmax) {
+      cmax = z[i];
+      carg = i;
+    }
+  }
+  if (cmax > st.m[q]) {
+    st.am[q] = static_cast<int>(col0 + carg);
+    const float f = st.m[q] == -INFINITY ? 0.f : fast_exp2((st.m[q] - cmax) * L1);
+    st.s[q] *= f;
+#pragma unroll
+    for (int r = 0; r < kM; ++r) st.d[q][r] *= f;
+    st.m[q] = cmax;
+  }
+}
+
+// One pair (a, b) over a 16-column chunk, with both units' maxima already
+// covering it: D_ab += e_a (z_a - z_b), D_ba += e_b (z_b - z_a), and the sums
+// of e_a / e_b where asked.
+template <int kM, bool kMasked, bool kSumA, bool kSumB>
+__device__ __forceinline__ void eval_pair(const float (&za)[16], const float (&zb)[16], int nvalid,
+                                          float L1, EvalState<kM>& st, int a, int b) {
+  const float na = -st.m[a] * L1, nb = -st.m[b] * L1;
+  float sa = 0.f, sb = 0.f, dab = 0.f, dba = 0.f;
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    const bool ok = !kMasked || i < nvalid;
+    const float ea = ok ? fast_exp2(fmaf(za[i], L1, na)) : 0.f;
+    const float eb = ok ? fast_exp2(fmaf(zb[i], L1, nb)) : 0.f;
+    const float dz = za[i] - zb[i];
+    if (kSumA) sa += ea;
+    if (kSumB) sb += eb;
+    dab = fmaf(ea, dz, dab);
+    dba = fmaf(eb, -dz, dba);
+  }
+  if (kSumA) st.s[a] += sa;
+  if (kSumB) st.s[b] += sb;
+  st.d[a][b] += dab;
+  st.d[b][a] += dba;
+}
+
+// The slot schedule's epilogue (M = 3; slots as in eval_mma_slots).  Per tile:
+//   copy    unit 0 into registers, release (copied)
+//   pass 1  (units 0, 1)  maxima and sums of both, D_01, D_10   [under unit 2's MMAs]
+//   pass 2a (units 1, 2)  maximum and sum of unit 2, D_12, D_21; release b_j
+//   pass 2b (units 0, 2)  D_02, D_20; release a_j               [under the next unit 0]
+template <bool kMasked>
+__device__ __forceinline__ void eval_pass1(const float (&z0)[16], uint32_t t1, int nvalid,
+                                           long long col0, float L1, EvalState<3>& st) {
+  float z1[16];
+  tmem_ld16(t1, z1);
+  eval_max<3, kMasked>(z0, nvalid, col0, L1, st, 0);
+  eval_max<3, kMasked>(z1, nvalid, col0, L1, st, 1);
+  eval_pair<3, kMasked, true, true>(z0, z1, nvalid, L1, st, 0, 1);
+}
+template <bool kMasked>
+__device__ __forceinline__ void eval_pass2a(uint32_t t1, uint32_t t2, int nvalid, long long col0,
+                                            float L1, EvalState<3>& st) {
+  float z1[16], z2[16];
+  tmem_ld16(t1, z1);
+  tmem_ld16(t2, z2);
+  eval_max<3, kMasked>(z2, nvalid, col0, L1, st, 2);
+  eval_pair<3, kMasked, false, true>(z1, z2, nvalid, L1, st, 1, 2);
+}
+template <bool kMasked>
+__device__ __forceinline__ void eval_pass2b(const float (&z0)[16], uint32_t t2, int nvalid,
+                                            float L1, EvalState<3>& st) {
+  float z2[16];
+  tmem_ld16(t2, z2);
+  eval_pair<3, kMasked, false, false>(z0, z2, nvalid, L1, st, 0, 2);
+}
+
+__device__ __forceinline__ bool eval_slots_main(const EvalParams& p, uint32_t base, uint32_t tl,
+                                                int split, int half, int lane,
+                                                volatile int* abort_flag, EvalState<3>& st) {
+  using Sm = EvalSmem<3>;
+  constexpr int kHalf = Sm::kN / 2;  // 128 columns per thread
+  constexpr int kChunks = kHalf / 16;
+  const float L1 = p.L1;
+  int j = 0;
+  for (int vt = split; vt < p.nvt; vt += p.S, ++j) {
+    const uint32_t par = static_cast<uint32_t>(j) & 1u;
+    const uint32_t sa = par * Sm::kN, sb = Sm::kN - sa;
+    const long long tcol = static_cast<long long>(vt) * Sm::kN + half * kHalf;
+    bool ok = mbar_wait(Sm::unit_full(base, 0), par, abort_flag, p.status);
+    if (!__all_sync(0xffffffffu, ok)) return false;
+    tc_fence_after();
+    float z0[kChunks][16];
+#pragma unroll
+    for (int c = 0; c < kChunks; ++c) tmem_ld16(tl + sa + static_cast<uint32_t>(c * 16), z0[c]);
+    eval_release(Sm::copied(base), lane);
+
+    ok = mbar_wait(Sm::unit_full(base, 1), par, abort_flag, p.status);
+    if (!__all_sync(0xffffffffu, ok)) return false;
+    tc_fence_after();
+#pragma unroll
+    for (int c = 0; c < kChunks; ++c) {
+      const long long col0 = tcol + c * 16;
+      const int nvalid = static_cast<int>(max(0LL, min(16LL, p.V - col0)));
+      if (nvalid == 0) continue;  // warp-uniform
+      const uint32_t t1 = tl + sb + static_cast<uint32_t>(c * 16);
+      if (nvalid == 16)
+        eval_pass1<false>(z0[c], t1, 16, col0, L1, st);
+      else
+        eval_pass1<true>(z0[c], t1, nvalid, col0, L1, st);
+    }
+
+    ok = mbar_wait(Sm::unit_full(base, 2), par, abort_flag, p.status);
+    if (!__all_sync(0xffffffffu, ok)) return false;
+    tc_fence_after();
+#pragma unroll
+    for (int c = 0; c < kChunks; ++c) {
+      const long long col0 = tcol + c * 16;
+      const int nvalid = static_cast<int>(max(0LL, min(16LL, p.V - col0)));
+      if (nvalid == 0) continue;
+      const uint32_t t1 = tl + sb + static_cast<uint32_t>(c * 16);
+      const uint32_t t2 = tl + sa + static_cast<uint32_t>(c * 16);
+      if (nvalid == 16)
+        eval_pass2a<false>(t1, t2, 16, col0, L1, st);
+      else
+        eval_pass2a<true>(t1, t2, nvalid, col0, L1, st);
+    }
+    eval_release(Sm::pass_a(base), lane);
+#pragma unroll
+    for (int c = 0; c < kChunks; ++c) {
+      const long long col0 = tcol + c * 16;
+      const int nvalid = static_cast<int>(max(0LL, min(16LL, p.V - col0)));
+      if (nvalid == 0) continue;
+      const uint32_t t2 = tl + sa + static_cast<uint32_t>(c * 16);
+      if (nvalid == 16)
+        eval_pass2b<false>(z0[c], t2, 16, L1, st);
+      else
+        eval_pass2b<true>(z0[c], t2, nvalid, L1, st);
+    }
+    eval_release(Sm::pass_b(base), lane);
+  }
+  return true;
+}
+
 template <int kM>
 __device__ __forceinline__ void eval_epilogue(const EvalParams& p, uint32_t base, uint32_t tmem,
                                               float* xchg, int row_base, int split, int warp,
@@ -229,6 +445,9 @@ __device__ __forceinline__ void eval_epilogue(const EvalParams& p, uint32_t base
 #pragma unroll
     for (int j = 0; j < kM; ++j) st.d[q][j] = 0.f;
   }
+  if constexpr (eval_slotted(kM)) {
+    eval_slots_main(p, base, tl, split, half, lane, abort_flag, st);
+  } else {
   int j = 0;
   for (int vt = split; vt < p.nvt; vt += p.S, ++j) {
     const bool ok = mbar_wait(Sm::accf(base, j), static_cast<uint32_t>(j >> 1) & 1u, abort_flag, p.status);
@@ -255,6 +474,7 @@ __device__ __forceinline__ void eval_epilogue(const EvalParams& p, uint32_t base
         eval_chunk<kM, true>(z, nvalid, col0, L1, st);
     }
     eval_release(Sm::free1(base), lane);
+  }
   }
 
   // The two column halves of a token combine through shared memory; fields
@@ -315,9 +535,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kHeadThreads, 1)
       mbar_init(Sm::full(base, s), 1);
       mbar_init(Sm::empty(base, s), 1);
     }
-    for (int q = 0; q < 2; ++q) mbar_init(Sm::accf(base, q), 1);
-    mbar_init(Sm::free0(base), 2 * kHeadEpiWarps);
-    mbar_init(Sm::free1(base), 2 * kHeadEpiWarps);
+    if constexpr (eval_slotted(kM)) {
+      for (int q = 0; q < 3; ++q) mbar_init(Sm::unit_full(base, q), 1);
+      mbar_init(Sm::copied(base), 2 * kHeadEpiWarps);
+      mbar_init(Sm::pass_a(base), 2 * kHeadEpiWarps);
+      mbar_init(Sm::pass_b(base), 2 * kHeadEpiWarps);
+    } else {
+      for (int q = 0; q < 2; ++q) mbar_init(Sm::accf(base, q), 1);
+      mbar_init(Sm::free0(base), 2 * kHeadEpiWarps);
+      mbar_init(Sm::free1(base), 2 * kHeadEpiWarps);
+    }
     mbar_init(Sm::drain(base), 1);
     fence_barrier_init();
   }
@@ -341,7 +568,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kHeadThreads, 1)
     if (warp == kHeadEpiWarps) {
       if (lane == 0) eval_producer<kTF32, kM>(p, base, row_base, rank, split, abort_flag);
     } else if (warp == kHeadEpiWarps + 1) {
-      if (lane == 0 && rank == 0) eval_mma<kTF32, kM>(p, base, tmem, split, abort_flag);
+      if (lane == 0 && rank == 0) {
+        if constexpr (eval_slotted(kM))
+          eval_mma_slots<kTF32>(p, base, tmem, split, abort_flag);
+        else
+          eval_mma<kTF32, kM>(p, base, tmem, split, abort_flag);
+      }
       __syncwarp();
     }
   } else {

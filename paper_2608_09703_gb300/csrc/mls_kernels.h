@@ -168,15 +168,20 @@ struct GemmParams {
 // ------------------------------------------------------------------ pairwise evaluation
 // Forward-only evaluation metrics between sub-models.  A CTA pair owns 256
 // tokens; for every vocabulary tile it computes the logit tiles of all M <= 4
-// sub-models into TMEM at once (M tiles of eval_tile_cols(M) columns, at most
-// the 512 TMEM columns) and accumulates, for every ordered pair (s, j),
-// D_sj = sum_v exp(z_s[v] - max_s) (z_s[v] - z_j[v]).  The tile is as wide as
-// TMEM allows: operand bytes per FLOP fall as the tile widens, and operand
-// delivery from L2 bounds this kernel.
-__host__ __device__ constexpr int eval_tile_cols(int M) { return M <= 2 ? 256 : (M == 3 ? 160 : 128); }
+// sub-models and accumulates, for every ordered pair (s, j),
+// D_sj = sum_v exp(z_s[v] - max_s) (z_s[v] - z_j[v]), which needs every
+// sub-model's logit at the same column.  Operand bytes per FLOP fall as the
+// tile widens, and operand delivery from L2 bounds this kernel, so the tile is
+// as wide as the 512 TMEM columns and the epilogue's registers allow:
+//   - M = 1, 2, 4: all M tiles resident in TMEM at once (256, 256, 128 columns);
+//   - M = 3 (eval_slotted): 256 columns; the widest sub-model's tile is copied
+//     into the epilogue's registers as soon as it is complete, the other two
+//     occupy two 256-column TMEM slots whose roles alternate from tile to tile.
+__host__ __device__ constexpr bool eval_slotted(int M) { return M == 3; }
+__host__ __device__ constexpr int eval_tile_cols(int M) { return M <= 3 ? 256 : 128; }
 constexpr uint32_t kEvalABytes = kHeadBM * 128;                    // A stage: 128 token rows
 __host__ __device__ constexpr uint32_t eval_b_bytes(int M) { return eval_tile_cols(M) / 2 * 128; }
-// As many stages as fit in 216 KB (9, 8, 6 and 6 for M = 4, 3, 2, 1).
+// As many stages as fit in 216 KB (9 for M = 4, 6 for M = 1, 2, 3).
 constexpr uint32_t kEvalStageBudget = 216 * 1024;
 __host__ __device__ constexpr int eval_stages(int M) {
   return static_cast<int>(kEvalStageBudget / (kEvalABytes + eval_b_bytes(M)));

@@ -101,16 +101,17 @@ def test_pairwise_single_model():
 @pytest.mark.parametrize("M", [2, 3, 4])
 def test_pairwise_many_tiles_per_pair(M):
     """16 token tiles and a ragged vocabulary of 4999 columns: each CTA pair
-    walks several vocabulary tiles (256, 160 or 128 columns wide for M = 2, 3,
-    4), so the epilogue's early release of the widest sub-model's columns and
-    the accumulator barriers go through several phases."""
+    walks several vocabulary tiles (256, 256 or 128 columns wide for M = 2, 3,
+    4), so the epilogue's early release of the widest sub-model's columns, the
+    two alternating TMEM slots at M = 3 and the accumulator barriers go through
+    several phases."""
     wl = synth.Workload("pwm", T=4096, d=(64, 192, 128, 320)[:M], V=4999, w_sigma=0.08)
     H, W, y = synth.make_inputs(wl, seed=37 + M)
     check(wl, H, W, y)
 
 
 def test_pairwise_fp32_three_models():
-    """fp32 inputs (tf32 products) at M = 3: 160-column tiles read with
+    """fp32 inputs (tf32 products) at M = 3: 256-column tiles read with
     32-element k-blocks, over a ragged vocabulary and two token tiles.  The
     heads have the fp32 workload's scale (sigma 0.02): tf32 rounds each
     product to ~2^-11, which the KL tolerance covers at logits of that size
