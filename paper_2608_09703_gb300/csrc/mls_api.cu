@@ -858,6 +858,13 @@ extern "C" int mls_head_pairwise(const mls_problem* p, const void* const* H, con
         ep.order[i] = ep.order[k];
         ep.order[k] = t;
       }
+  // Slot schedule (M = 3): the narrower of the two TMEM-slot units goes first,
+  // so the epilogue's first pass runs under the longer MMAs of the other.
+  if (eval_slotted(p->M)) {
+    const int t = ep.order[1];
+    ep.order[1] = ep.order[2];
+    ep.order[2] = t;
+  }
   for (int i = 0; i < p->M; ++i) ep.pos[ep.order[i]] = i;
   ep.ntt = pl.ntt;
   ep.nvt = pl.eval_nvt;

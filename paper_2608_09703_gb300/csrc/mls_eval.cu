@@ -168,9 +168,10 @@ __device__ __forceinline__ void eval_mma(const EvalParams& p, uint32_t base, uin
 // a_j = (j & 1) * 256 and b_j = 256 - a_j:
 //   unit 0 (widest) -> a_j, after the epilogue's first pass over tile j - 1's
 //                      last unit has freed a_j (= b_{j-1})         [pass_a]
-//   unit 1          -> b_j, after its second pass has freed b_j      [pass_b]
+//   unit 1 (narrowest) -> b_j, after its second pass has freed b_j   [pass_b]
 //   unit 2          -> a_j, once unit 0 has been copied to registers [copied]
-// so unit 0 of the next tile, the longest, runs under the end of the epilogue.
+// so unit 0 of the next tile, the longest, runs under the end of the epilogue,
+// and the pass over units 0 and 1 under unit 2's MMAs.
 template <bool kTF32>
 __device__ __forceinline__ void eval_mma_slots(const EvalParams& p, uint32_t base, uint32_t tmem,
                                                int split, volatile int* abort_flag) {
@@ -276,87 +277,147 @@ __device__ __forceinline__ void eval_release(uint32_t bar, int lane) {
   if (lane == 0) mbar_arrive_remote(map_to_rank(bar, 0));
 }
 
-// Online maximum and first argmax of unit q over a 16-column chunk; a new
-// maximum rescales the unit's sum and its D_q*.
-template <int kM, bool kMasked>
-__device__ __forceinline__ void eval_max(const float (&z)[16], int nvalid, long long col0,
-                                         float L1, EvalState<kM>& st, int q) {
-  float cmax = -INFINITY;
-  int carg = 0;
+// ---- slot schedule epilogue (M = 3)
+// Columns past V take this logit: exp2 of it underflows to 0 against any real
+// maximum, it never wins a maximum over a chunk that has a valid column, and
+// two of them differ by 0, so every accumulation ignores them without a
+// second (masked) copy of the code.
+constexpr float kPadLogit = -1e30f;
+
+// This thread's 16 columns at TMEM address t; columns from nvalid on padded.
+__device__ __forceinline__ void ld_chunk(uint32_t t, int nvalid, float (&z)[16]) {
+  tmem_ld16(t, z);
+  if (nvalid < 16) {
 #pragma unroll
-  for (int i = 0; i < 16; ++i) {
-    const bool ok = !kMasked || i < nvalid;
-    if (ok && z[i] > cmax) {
-      cmax = z[i];
-      carg = i;
+    for (int i = 0; i < 16; ++i)
+      if (i >= nvalid) z[i] = kPadLogit;
+  }
+}
+// Two chunks in one wait: na (nb) of a's (b's) columns are valid.
+__device__ __forceinline__ void ld_chunk2(uint32_t ta, uint32_t tb, int na, int nb, float (&a)[16],
+                                          float (&b)[16]) {
+  tmem_ld16x2(ta, tb, a, b);
+  if (na < 16 || nb < 16) {
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      if (i >= na) a[i] = kPadLogit;
+      if (i >= nb) b[i] = kPadLogit;
     }
   }
-  if (cmax > st.m[q]) {
-    st.am[q] = static_cast<int>(col0 + carg);
-    const float f = st.m[q] == -INFINITY ? 0.f : fast_exp2((st.m[q] - cmax) * L1);
+}
+
+// Maximum of a chunk and the first column attaining it, by a tree whose left
+// operand always holds the lower columns (ties keep the left one).
+__device__ __forceinline__ void chunk_argmax(const float (&z)[16], float& vmax, int& imax) {
+  float v[8];
+  int ix[8];
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    const bool r = z[2 * k + 1] > z[2 * k];
+    v[k] = r ? z[2 * k + 1] : z[2 * k];
+    ix[k] = r ? 2 * k + 1 : 2 * k;
+  }
+#pragma unroll
+  for (int w = 4; w >= 1; w >>= 1) {
+#pragma unroll
+    for (int k = 0; k < w; ++k) {
+      const bool r = v[2 * k + 1] > v[2 * k];
+      v[k] = r ? v[2 * k + 1] : v[2 * k];
+      ix[k] = r ? ix[2 * k + 1] : ix[2 * k];
+    }
+  }
+  vmax = v[0];
+  imax = ix[0];
+}
+
+// Folds a tile's maximum (tmax at column tcol) into unit q's running state:
+// a new maximum rescales the unit's sum and its D_q*.
+__device__ __forceinline__ void fold_max(EvalState<3>& st, int q, float tmax, long long tcol, float L1) {
+  if (tmax > st.m[q]) {
+    st.am[q] = static_cast<int>(tcol);
+    const float f = st.m[q] == -INFINITY ? 0.f : fast_exp2((st.m[q] - tmax) * L1);
     st.s[q] *= f;
 #pragma unroll
-    for (int r = 0; r < kM; ++r) st.d[q][r] *= f;
-    st.m[q] = cmax;
+    for (int r = 0; r < 3; ++r) st.d[q][r] *= f;
+    st.m[q] = tmax;
   }
 }
 
-// One pair (a, b) over a 16-column chunk, with both units' maxima already
-// covering it: D_ab += e_a (z_a - z_b), D_ba += e_b (z_b - z_a), and the sums
-// of e_a / e_b where asked.
-template <int kM, bool kMasked, bool kSumA, bool kSumB>
-__device__ __forceinline__ void eval_pair(const float (&za)[16], const float (&zb)[16], int nvalid,
-                                          float L1, EvalState<kM>& st, int a, int b) {
-  const float na = -st.m[a] * L1, nb = -st.m[b] * L1;
-  float sa = 0.f, sb = 0.f, dab = 0.f, dba = 0.f;
+// Tile maximum of a unit held in TMEM at t (this thread's 128 columns).
+__device__ __forceinline__ void tmem_tile_max(uint32_t t, long long tcol, long long V, float& tmax,
+                                              long long& targ) {
+  tmax = -INFINITY;
+  targ = 0;
 #pragma unroll
-  for (int i = 0; i < 16; ++i) {
-    const bool ok = !kMasked || i < nvalid;
-    const float ea = ok ? fast_exp2(fmaf(za[i], L1, na)) : 0.f;
-    const float eb = ok ? fast_exp2(fmaf(zb[i], L1, nb)) : 0.f;
-    const float dz = za[i] - zb[i];
-    if (kSumA) sa += ea;
-    if (kSumB) sb += eb;
-    dab = fmaf(ea, dz, dab);
-    dba = fmaf(eb, -dz, dba);
+  for (int c = 0; c < 8; c += 2) {
+    const long long col0 = tcol + c * 16;
+    if (col0 >= V) continue;  // warp-uniform
+    float za[16], zb[16];
+    ld_chunk2(t + static_cast<uint32_t>(c * 16), t + static_cast<uint32_t>(c * 16 + 16),
+              static_cast<int>(min(16LL, V - col0)), static_cast<int>(max(0LL, min(16LL, V - col0 - 16))),
+              za, zb);
+    float va, vb;
+    int ia, ib;
+    chunk_argmax(za, va, ia);
+    chunk_argmax(zb, vb, ib);
+    if (col0 + 16 >= V) vb = -INFINITY;  // the second chunk is past V
+    if (va > tmax) {
+      tmax = va;
+      targ = col0 + ia;
+    }
+    if (vb > tmax) {
+      tmax = vb;
+      targ = col0 + 16 + ib;
+    }
   }
-  if (kSumA) st.s[a] += sa;
-  if (kSumB) st.s[b] += sb;
-  st.d[a][b] += dab;
-  st.d[b][a] += dba;
 }
 
-// The slot schedule's epilogue (M = 3; slots as in eval_mma_slots).  Per tile:
-//   copy    unit 0 into registers, release (copied)
-//   pass 1  (units 0, 1)  maxima and sums of both, D_01, D_10   [under unit 2's MMAs]
-//   pass 2a (units 1, 2)  maximum and sum of unit 2, D_12, D_21; release b_j
-//   pass 2b (units 0, 2)  D_02, D_20; release a_j               [under the next unit 0]
-template <bool kMasked>
-__device__ __forceinline__ void eval_pass1(const float (&z0)[16], uint32_t t1, int nvalid,
-                                           long long col0, float L1, EvalState<3>& st) {
-  float z1[16];
-  tmem_ld16(t1, z1);
-  eval_max<3, kMasked>(z0, nvalid, col0, L1, st, 0);
-  eval_max<3, kMasked>(z1, nvalid, col0, L1, st, 1);
-  eval_pair<3, kMasked, true, true>(z0, z1, nvalid, L1, st, 0, 1);
-}
-template <bool kMasked>
-__device__ __forceinline__ void eval_pass2a(uint32_t t1, uint32_t t2, int nvalid, long long col0,
-                                            float L1, EvalState<3>& st) {
-  float z1[16], z2[16];
-  tmem_ld16(t1, z1);
-  tmem_ld16(t2, z2);
-  eval_max<3, kMasked>(z2, nvalid, col0, L1, st, 2);
-  eval_pair<3, kMasked, false, true>(z1, z2, nvalid, L1, st, 1, 2);
-}
-template <bool kMasked>
-__device__ __forceinline__ void eval_pass2b(const float (&z0)[16], uint32_t t2, int nvalid,
-                                            float L1, EvalState<3>& st) {
-  float z2[16];
-  tmem_ld16(t2, z2);
-  eval_pair<3, kMasked, false, false>(z0, z2, nvalid, L1, st, 0, 2);
+// Partial sums of one pass over one pair (a, b) with both maxima fixed.
+struct PairSums {
+  float sa0, sa1, sb0, sb1, dab0, dab1, dba0, dba1;
+};
+
+// One 16-column chunk of pair (a, b): e_a, e_b against the fixed maxima
+// (na = -m_a log2 e, nb = -m_b log2 e); two interleaved partials per sum.
+template <bool kSumA, bool kSumB>
+__device__ __forceinline__ void pair_chunk(const float (&za)[16], const float (&zb)[16], float L1,
+                                           float na, float nb, PairSums& ps) {
+#pragma unroll
+  for (int i = 0; i < 16; i += 2) {
+    const float ea0 = fast_exp2(fmaf(za[i], L1, na)), ea1 = fast_exp2(fmaf(za[i + 1], L1, na));
+    const float eb0 = fast_exp2(fmaf(zb[i], L1, nb)), eb1 = fast_exp2(fmaf(zb[i + 1], L1, nb));
+    const float d0 = za[i] - zb[i], d1 = za[i + 1] - zb[i + 1];
+    if (kSumA) {
+      ps.sa0 += ea0;
+      ps.sa1 += ea1;
+    }
+    if (kSumB) {
+      ps.sb0 += eb0;
+      ps.sb1 += eb1;
+    }
+    ps.dab0 = fmaf(ea0, d0, ps.dab0);
+    ps.dab1 = fmaf(ea1, d1, ps.dab1);
+    ps.dba0 = fmaf(eb0, -d0, ps.dba0);
+    ps.dba1 = fmaf(eb1, -d1, ps.dba1);
+  }
 }
 
+template <bool kSumA, bool kSumB>
+__device__ __forceinline__ void fold_pair(EvalState<3>& st, int a, int b, const PairSums& ps) {
+  if (kSumA) st.s[a] += ps.sa0 + ps.sa1;
+  if (kSumB) st.s[b] += ps.sb0 + ps.sb1;
+  st.d[a][b] += ps.dab0 + ps.dab1;
+  st.d[b][a] += ps.dba0 + ps.dba1;
+}
+
+// Per tile (slots as in eval_mma_slots):
+//   copy    unit 0 into registers (padded past V), its tile maximum; release (copied)
+//   pass 1  (units 0, 1)  unit 1's tile maximum, then the sums of both, D_01, D_10
+//           [under unit 2's MMAs]
+//   pass 2a (units 1, 2)  unit 2's tile maximum, then its sum, D_12, D_21; release b_j
+//   pass 2b (units 0, 2)  D_02, D_20; release a_j    [under the next tile's unit 0]
+// Every pass runs with its units' maxima already folded in, so its chunks are
+// independent of one another.
 __device__ __forceinline__ bool eval_slots_main(const EvalParams& p, uint32_t base, uint32_t tl,
                                                 int split, int half, int lane,
                                                 volatile int* abort_flag, EvalState<3>& st) {
@@ -364,6 +425,7 @@ __device__ __forceinline__ bool eval_slots_main(const EvalParams& p, uint32_t ba
   constexpr int kHalf = Sm::kN / 2;  // 128 columns per thread
   constexpr int kChunks = kHalf / 16;
   const float L1 = p.L1;
+  const long long V = p.V;
   int j = 0;
   for (int vt = split; vt < p.nvt; vt += p.S, ++j) {
     const uint32_t par = static_cast<uint32_t>(j) & 1u;
@@ -374,50 +436,89 @@ __device__ __forceinline__ bool eval_slots_main(const EvalParams& p, uint32_t ba
     tc_fence_after();
     float z0[kChunks][16];
 #pragma unroll
-    for (int c = 0; c < kChunks; ++c) tmem_ld16(tl + sa + static_cast<uint32_t>(c * 16), z0[c]);
+    for (int c = 0; c < kChunks; c += 2)
+      tmem_ld16x2(tl + sa + static_cast<uint32_t>(c * 16), tl + sa + static_cast<uint32_t>(c * 16 + 16),
+                  z0[c], z0[c + 1]);
     eval_release(Sm::copied(base), lane);
+    {
+      float tmax = -INFINITY;
+      long long targ = 0;
+#pragma unroll
+      for (int c = 0; c < kChunks; ++c) {
+        const long long col0 = tcol + c * 16;
+        if (col0 + 16 > V) {
+#pragma unroll
+          for (int i = 0; i < 16; ++i)
+            if (col0 + i >= V) z0[c][i] = kPadLogit;
+        }
+        if (col0 >= V) continue;
+        float v;
+        int ix;
+        chunk_argmax(z0[c], v, ix);
+        if (v > tmax) {
+          tmax = v;
+          targ = col0 + ix;
+        }
+      }
+      fold_max(st, 0, tmax, targ, L1);
+    }
 
     ok = mbar_wait(Sm::unit_full(base, 1), par, abort_flag, p.status);
     if (!__all_sync(0xffffffffu, ok)) return false;
     tc_fence_after();
+    {
+      float tmax;
+      long long targ;
+      tmem_tile_max(tl + sb, tcol, V, tmax, targ);
+      fold_max(st, 1, tmax, targ, L1);
+      const float n0 = -st.m[0] * L1, n1 = -st.m[1] * L1;
+      PairSums ps = {};
 #pragma unroll
-    for (int c = 0; c < kChunks; ++c) {
-      const long long col0 = tcol + c * 16;
-      const int nvalid = static_cast<int>(max(0LL, min(16LL, p.V - col0)));
-      if (nvalid == 0) continue;  // warp-uniform
-      const uint32_t t1 = tl + sb + static_cast<uint32_t>(c * 16);
-      if (nvalid == 16)
-        eval_pass1<false>(z0[c], t1, 16, col0, L1, st);
-      else
-        eval_pass1<true>(z0[c], t1, nvalid, col0, L1, st);
+      for (int c = 0; c < kChunks; ++c) {
+        const long long col0 = tcol + c * 16;
+        if (col0 >= V) continue;  // warp-uniform
+        float z1[16];
+        ld_chunk(tl + sb + static_cast<uint32_t>(c * 16), static_cast<int>(min(16LL, V - col0)), z1);
+        pair_chunk<true, true>(z0[c], z1, L1, n0, n1, ps);
+      }
+      fold_pair<true, true>(st, 0, 1, ps);
     }
 
     ok = mbar_wait(Sm::unit_full(base, 2), par, abort_flag, p.status);
     if (!__all_sync(0xffffffffu, ok)) return false;
     tc_fence_after();
+    {
+      float tmax;
+      long long targ;
+      tmem_tile_max(tl + sa, tcol, V, tmax, targ);
+      fold_max(st, 2, tmax, targ, L1);
+      const float n1 = -st.m[1] * L1, n2 = -st.m[2] * L1;
+      PairSums ps = {};
 #pragma unroll
-    for (int c = 0; c < kChunks; ++c) {
-      const long long col0 = tcol + c * 16;
-      const int nvalid = static_cast<int>(max(0LL, min(16LL, p.V - col0)));
-      if (nvalid == 0) continue;
-      const uint32_t t1 = tl + sb + static_cast<uint32_t>(c * 16);
-      const uint32_t t2 = tl + sa + static_cast<uint32_t>(c * 16);
-      if (nvalid == 16)
-        eval_pass2a<false>(t1, t2, 16, col0, L1, st);
-      else
-        eval_pass2a<true>(t1, t2, nvalid, col0, L1, st);
+      for (int c = 0; c < kChunks; ++c) {
+        const long long col0 = tcol + c * 16;
+        if (col0 >= V) continue;
+        float z1[16], z2[16];
+        const int nv = static_cast<int>(min(16LL, V - col0));
+        ld_chunk2(tl + sb + static_cast<uint32_t>(c * 16), tl + sa + static_cast<uint32_t>(c * 16), nv, nv,
+                  z1, z2);
+        pair_chunk<false, true>(z1, z2, L1, n1, n2, ps);
+      }
+      fold_pair<false, true>(st, 1, 2, ps);
     }
     eval_release(Sm::pass_a(base), lane);
+    {
+      const float n0 = -st.m[0] * L1, n2 = -st.m[2] * L1;
+      PairSums ps = {};
 #pragma unroll
-    for (int c = 0; c < kChunks; ++c) {
-      const long long col0 = tcol + c * 16;
-      const int nvalid = static_cast<int>(max(0LL, min(16LL, p.V - col0)));
-      if (nvalid == 0) continue;
-      const uint32_t t2 = tl + sa + static_cast<uint32_t>(c * 16);
-      if (nvalid == 16)
-        eval_pass2b<false>(z0[c], t2, 16, L1, st);
-      else
-        eval_pass2b<true>(z0[c], t2, nvalid, L1, st);
+      for (int c = 0; c < kChunks; ++c) {
+        const long long col0 = tcol + c * 16;
+        if (col0 >= V) continue;
+        float z2[16];
+        ld_chunk(tl + sa + static_cast<uint32_t>(c * 16), static_cast<int>(min(16LL, V - col0)), z2);
+        pair_chunk<false, false>(z0[c], z2, L1, n0, n2, ps);
+      }
+      fold_pair<false, false>(st, 0, 2, ps);
     }
     eval_release(Sm::pass_b(base), lane);
   }

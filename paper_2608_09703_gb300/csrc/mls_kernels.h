@@ -200,7 +200,8 @@ struct EvalParams {
   CUtensorMap mapH[kMaxModels];  // H_m [T, d_m], box {128 B of K, kHeadBM rows}
   CUtensorMap mapW[kMaxModels];  // W_m [V, d_m], box {128 B of K, eval_tile_cols(M) / 2 rows}
   int M;
-  int order[kMaxModels];         // units of a vocabulary tile, widest sub-model first
+  int order[kMaxModels];         // units of a vocabulary tile, widest sub-model first (M = 3:
+                                 // widest, narrowest, middle)
   int pos[kMaxModels];           // pos[order[i]] = i
   int nk[kMaxModels];
   int ntt;                       // token tiles of 256 (one per CTA pair)
