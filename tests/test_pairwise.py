@@ -110,6 +110,17 @@ def test_pairwise_many_tiles_per_pair(M):
     check(wl, H, W, y)
 
 
+def test_pairwise_three_models_partial_last_half():
+    """M = 3 with V = 4900: the last 256-column tile holds 36 columns, so the
+    first column half of its threads is cut inside a 16-column chunk and the
+    second half has no valid column at all; three token tiles, the last ragged,
+    and a width tie (two sub-models of 128)."""
+    wl = synth.Workload("pwh", T=520, d=(128, 64, 128), V=4900, w_sigma=0.08)
+    H, W, y = synth.make_inputs(wl, seed=43)
+    y[[0, 519]] = -1
+    check(wl, H, W, y)
+
+
 def test_pairwise_fp32_three_models():
     """fp32 inputs (tf32 products) at M = 3: 256-column tiles read with
     32-element k-blocks, over a ragged vocabulary and two token tiles.  The
