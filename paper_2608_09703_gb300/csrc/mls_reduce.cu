@@ -41,8 +41,8 @@ __device__ __forceinline__ double block_sum_double(double v, double* sh) {
 // k = 4 (w mod kWT) + l / 8, k + 4 kWT, ...: the 8 lanes of a group read 32
 // consecutive bytes (one sector) of each (partial, field, sub-model).  kWT
 // follows the number of partials (merge_warps_per_octet), so few partials
-// do not leave most lanes idle.  Round 1 takes every sub-model's row maximum,
-// round 2 its sums.  The partials of a token are combined in a fixed order
+// do not leave most lanes idle.  Pass 1 takes every sub-model's row maximum,
+// pass 2 its sums.  The partials of a token are combined in a fixed order
 // (within a lane, across the 4 lane groups by butterflies, across the octet's
 // warps in warp order), and the block's share of the loss over its octets in
 // octet order, so results are deterministic.
@@ -66,7 +66,7 @@ __global__ void __launch_bounds__(kMergeWarps * 32, 4) merge_kernel(const __grid
   const int tc = p.teacher;
   const int k0 = 4 * ww + grp;
 
-  // ---- round 1: row maxima of every sub-model
+  // ---- pass 1: row maxima of every sub-model
   float mx[kMaxModels];
 #pragma unroll
   for (int m = 0; m < kMaxModels; ++m) mx[m] = -INFINITY;
@@ -95,7 +95,7 @@ __global__ void __launch_bounds__(kMergeWarps * 32, 4) merge_kernel(const __grid
     if (m == tc) mT = mx[m];
   __syncthreads();  // sh_f[0] is reused below
 
-  // ---- round 2: sums.  The teacher's weighted sum is relative to its own
+  // ---- pass 2: sums.  The teacher's weighted sum is relative to its own
   // maximum: B_k = sum q~ (z - m_k) log2(e)/tau; moving it to the row maximum
   // mT adds (m_k - mT) log2(e)/tau per unit of weight before the weights are
   // rescaled.  A student's A_k is relative to the teacher's maximum of the
