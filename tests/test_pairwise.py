@@ -90,6 +90,30 @@ def test_pairwise_suite3_full_size_sampled():
     check(wl, H, W, y, rows=rows)
 
 
+@pytest.mark.parametrize("name", ["suite4", "stress"])
+def test_pairwise_large_vocab_sampled(name):
+    """The 4-level suite (M = 4, V = 128256: four resident 128-column tiles)
+    and the stress shape (M = 3, V = 256000, teacher head x8: the slot
+    schedule over 1000 vocabulary tiles) at full size; ten sampled tokens (the
+    first and last among them) against the oracle, their argmax against fp64
+    logits computed on the device."""
+    wl = synth.WORKLOADS[name]
+    H, W, y = synth.make_inputs(wl, seed=44, device="cuda")
+    kl, am, stats = run_pairwise(wl, H, W, y)
+    rng = np.random.default_rng(44)
+    rows = np.unique(np.concatenate([rng.integers(0, wl.T, 8), [0, wl.T - 1]]))
+    ri = torch.as_tensor(rows, device=H[0].device)
+    ref = oracle.pairwise(synth.as_oracle_arrays([h[ri] for h in H]), synth.as_oracle_arrays(W))
+    err = np.abs(kl[:, :, rows] - ref["kl"]) / np.maximum(1.0, np.abs(ref["kl"]))
+    assert err.max() <= KL_TOL, f"KL err {err.max()}"
+    for m in range(wl.M):
+        zz = (H[m][ri].double() @ W[m].double().T).cpu().numpy()
+        top = np.sort(zz, -1)[:, -2:]
+        decided = (top[:, 1] - top[:, 0]) > 1e-4 * np.maximum(1.0, np.abs(top[:, 1]))
+        assert (am[m][rows][decided] == np.argmax(zz, -1)[decided]).all()
+    assert np.isfinite(stats).all()
+
+
 def test_pairwise_single_model():
     """M = 1: no pairs; the argmax and the (zero) KL matrix still come out."""
     wl = synth.Workload("pw1", T=300, d=(96,), V=777, w_sigma=0.1)
