@@ -131,17 +131,24 @@ struct Plan {
 // walks ceil(tiles / S) vocabulary tiles and `pairs` pairs are resident at a
 // time, so the kernel lasts about waves * (tiles per pair + a fixed per-pair
 // cost); S minimises that.
-int choose_splits(int ntt, long long tiles, int pairs) {
+// cta_cost: what one CTA pair costs beyond its tiles, in vocabulary tiles
+// (prologue, pipeline fill and drain, the exposed epilogue of its last tile).
+constexpr double kHeadCtaCost = 0.25;
+// The evaluation kernel's last tile exposes its whole epilogue (every pass) and
+// the partial-state write.  Measured at the 3-level suite (T = 8192, 197
+// vocabulary tiles): 33 splits (the head kernels' choice) 3.39 ms per call,
+// 7 splits 3.24 ms, which puts its per-pair cost near 1.2 tiles.
+constexpr double kEvalCtaCost = 1.25;
+int choose_splits(int ntt, long long tiles, int pairs, double cta_cost = kHeadCtaCost) {
   if (ntt < 1) ntt = 1;
   if (tiles < 1) return 1;
-  const double kCtaCost = 0.25;  // prologue + pipeline drain, in vocabulary tiles
   long long best = 1;
   double best_cost = 1e300;
   for (long long S = 1; S <= tiles && S <= 512; ++S) {
     const long long per = (tiles + S - 1) / S;
     if (S > 1 && (per - 1) * S >= tiles) continue;  // same tiles per CTA with fewer CTAs
     const long long waves = (ntt * S + pairs - 1) / pairs;
-    const double cost = waves * (per + kCtaCost);
+    const double cost = waves * (per + cta_cost);
     if (cost < best_cost - 1e-9) {
       best_cost = cost;
       best = S;
@@ -248,7 +255,7 @@ Plan make_plan(const mls_problem* p, int pairs) {
   pl.bwd_bytes = o;
 
   pl.eval_nvt = static_cast<int>(ceil_div(V, eval_tile_cols(p->M)));
-  pl.eval_S = choose_splits(pl.ntt, pl.eval_nvt, pairs);
+  pl.eval_S = choose_splits(pl.ntt, pl.eval_nvt, pairs, kEvalCtaCost);
   o = 0;
   pl.off_epart = o;
   o = align_up(o + sizeof(float) * static_cast<size_t>(pl.eval_S) * kEvalFields * T);
