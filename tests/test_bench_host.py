@@ -52,3 +52,15 @@ def test_traffic_figures_are_tied_to_listed_sources():
         got = bench.traffic_for(kernel)
         # either the figure (code unchanged since the capture) or None
         assert got in (None, e["traffic_bytes_per_launch"])
+
+
+def test_pick_peak_follows_the_clock_regime():
+    pk = {"bf16_tflops": 1904.5, "bf16_tflops_sustained": 1717.4, "sm_max_mhz": 2070.0}
+    # a sub-second region runs at burst clocks whatever the samples say
+    assert bench.pick_peak(pk, 0.24, {"sm_mhz": 1400.0, "sm_max_mhz": 2070.0})[:2] == (1904.5, "burst")
+    # a long region that held its clock near the maximum is still burst
+    assert bench.pick_peak(pk, 3.0, {"sm_mhz": 2000.0, "sm_max_mhz": 2070.0})[:2] == (1904.5, "burst")
+    # a long region that settled under the power cap is held to the sustained figure
+    assert bench.pick_peak(pk, 3.0, {"sm_mhz": 1460.0, "sm_max_mhz": 2070.0})[:2] == (1717.4, "sustained")
+    # no clock samples: the burst figure (the larger denominator)
+    assert bench.pick_peak(pk, 3.0, None)[:2] == (1904.5, "burst")
